@@ -1,0 +1,81 @@
+"""The seeded input generators (CPU): laws, determinism, quotas."""
+
+import numpy as np
+import pytest
+
+import synth
+
+
+def test_rows_deterministic_and_normal_like():
+    a = synth.rows_cpu(12345, 256, np.arange(400))
+    b = synth.rows_range_cpu(12345, 256, 0, 400, threads=3)
+    assert np.array_equal(a, b)
+    c = synth.rows_cpu(12345, 256, np.array([399, 7]))
+    assert np.array_equal(c, a[[399, 7]])
+    x = a.astype(np.uint32) << 16
+    v = x.view(np.float32).astype(np.float64)
+    assert abs(v.mean()) < 5e-4 and abs(v.std() - 0.02) < 5e-4
+    assert np.abs(v).max() < 0.02 * 3.5          # Irwin-Hall(4) support is +-sqrt(12)
+    assert not np.array_equal(a, synth.rows_cpu(12346, 256, np.arange(400)))
+
+
+def test_zipf_matches_inverse_cdf():
+    """Tokens equal upper_bound(cdf, u) with u the top 53 bits of each draw."""
+    w = synth.WORKLOADS["tiny"]
+    seed = 99
+    n = 5000
+    tok = synth.zipf_tokens(w, seed, n, inject=False)
+    r = np.arange(1, w.vocab + 1, dtype=np.float64)
+    cdf = np.cumsum(r ** -w.zipf_s)
+    cdf /= cdf[-1]
+    cdf[-1] = 1.0
+    lib = synth._load()
+    u = np.array([(lib.synth_draw(seed, i) >> 11) * 2.0 ** -53 for i in range(n)])
+    ref = np.searchsorted(cdf, u, side="right")
+    assert np.array_equal(tok, ref)
+    # rank-1 frequency close to 1 / H(V, s)
+    p1 = 1.0 / np.sum(r ** -w.zipf_s)
+    assert abs((tok == 0).mean() - p1) < 0.02
+
+
+def test_fgram_set_first_seen_distinct():
+    w = synth.WORKLOADS["tiny"].scaled("tiny_fg", quotas=((2, 500), (3, 300)))
+    tok, ln, used = synth.fgram_set(w)
+    assert tok.shape == (800, 3) and (np.bincount(ln)[2:] == [500, 300]).all()
+    grams = [tuple(tok[r, :ln[r]]) for r in range(800)]
+    assert len(set(grams)) == 800
+    assert (tok[ln == 2, 2] == -1).all()
+    # re-derive from the source stream: first-seen order, lengths interleaved by position
+    src = synth.zipf_tokens(w, synth.stream_seed(w, synth.S_SOURCE), used)
+    seen = {2: set(), 3: set()}
+    have = {2: 0, 3: 0}
+    quota = {2: 500, 3: 300}
+    exp = []
+    for p in range(used - 3 + 1):
+        for n in (2, 3):
+            if have[n] < quota[n]:
+                g = tuple(src[p:p + n])
+                if g not in seen[n]:
+                    seen[n].add(g)
+                    have[n] += 1
+                    exp.append(g)
+        if len(exp) == 800:
+            break
+    assert grams == [tuple(int(x) for x in g) for g in exp]
+
+
+def test_phrase_injection_rate():
+    w = synth.WORKLOADS["stress_k5"]
+    pt, pl = synth.phrase_pool(w)
+    assert pt.shape == (4096, 8) and pl.min() == 4 and pl.max() == 8
+    base = synth.zipf_tokens(w, 7, 200000, inject=False)
+    inj = synth.zipf_tokens(w, 7, 200000, inject=True)
+    frac = (base != inj).mean()
+    assert 0.03 < frac < 0.06
+
+
+def test_decode_inputs_shapes():
+    w = synth.WORKLOADS["offload_decode"].scaled("dec_small", dec_S=8, dec_steps=5)
+    hist, hl, new = synth.decode_inputs(w)
+    assert hist.shape == (8, 2) and (hl == 2).all() and new.shape == (5, 8)
+    assert (hist >= 0).all() and (new >= 0).all() and (new < w.vocab).all()
