@@ -1,0 +1,218 @@
+/*
+ * scone.h — C ABI of the SCONE inference-time input-embedding path on one
+ * NVIDIA GB300 (sm_103a).
+ *
+ * The path (Algorithm 1, inference branch, Sec. 3 of "Scaling Embedding
+ * Layers in Language Models"): for every position i of a token sequence
+ * (sigma_1 .. sigma_m), take the smallest j < i such that the n-gram
+ * (sigma_j .. sigma_i) is an f-gram, i.e. the longest f-gram ending at i,
+ * and emit that f-gram's precomputed embedding F(sigma_j .. sigma_i); if no
+ * f-gram ends at i, emit the token embedding T(sigma_i). f-grams have
+ * lengths 2..K (V_fgram is a subset of V_token^[2,K], Sec. 3).
+ *
+ * F is stored as "a dense embedding matrix paired with a hash dictionary
+ * that maps f-grams to matrix indices" (Sec. 2, "Efficient Indexing for
+ * Large Embedding Layers"). Here the dictionary is a GPU open-addressing
+ * table built once by scone_table_build; the dense matrix stays caller-owned
+ * in HBM or in host-pinned, device-mapped memory (the paper's off-accelerator
+ * tier, Sec. 4.3).
+ *
+ * Conventions shared by every call
+ *  - Pointers are plain addresses; "device" means a CUDA device address
+ *    (cudaMalloc / torch CUDA tensor), "host" an ordinary host address.
+ *    No call takes ownership of a caller buffer.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default).
+ *    Calls marked "async" only enqueue work on it and return.
+ *  - Embedding rows are bf16, passed as raw 16-bit words (scone_bf16), rows
+ *    of d elements, row-major, no padding between rows.
+ *  - Token batches are dense [B x L] int32, sequence-major. n-grams never
+ *    cross a sequence boundary; the first position of every sequence always
+ *    takes T.
+ *  - Errors the host can see (null or misaligned pointers, bad sizes, K or
+ *    vocab that the key format cannot hold) are returned at once and nothing
+ *    is enqueued. Errors only the device can see (a token outside
+ *    [0, vocab), a lookup that exceeded the probe limit) never trap: the
+ *    position gets a zero row, row = -1 and len = 0, and a sticky status
+ *    word in the table records the first such error; scone_status reads it.
+ *  - Return values are SCONE_OK (0) or a negative scone_err code.
+ */
+#ifndef SCONE_H_
+#define SCONE_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct scone_table scone_table;   /* opaque; owns its slot array and status word */
+typedef struct scone_decode scone_decode; /* opaque; owns the device history ring */
+typedef uint16_t scone_bf16;              /* raw bf16 bits */
+
+enum scone_err {
+  SCONE_OK = 0,
+  SCONE_ERR_INVALID_ARG = -1,     /* bad pointer, size, alignment or location */
+  SCONE_ERR_TOKEN_RANGE = -2,     /* a token outside [0, vocab) (device-detected, sticky) */
+  SCONE_ERR_DUPLICATE_FGRAM = -3, /* the f-gram list holds the same n-gram twice */
+  SCONE_ERR_TABLE_FULL = -4,      /* an insert found no free slot (cannot happen below LF 1) */
+  SCONE_ERR_PROBE_LIMIT = -5,     /* a lookup read more buckets than the limit (sticky) */
+  SCONE_ERR_UNSUPPORTED = -6,     /* K * ceil(log2 vocab) does not fit the key format */
+  SCONE_ERR_CUDA = -7,            /* a CUDA runtime call failed */
+  SCONE_ERR_NOMEM = -8            /* device or host allocation failed */
+};
+
+enum scone_rows_location {
+  SCONE_ROWS_DEVICE = 0,      /* F is device memory (HBM) */
+  SCONE_ROWS_HOST_MAPPED = 1  /* F is host memory from cudaHostAlloc(..., cudaHostAllocMapped)
+                                 or cudaHostRegister(..., Mapped); the GPU reads it over the
+                                 host link */
+};
+
+/*
+ * scone_table_build — the f-gram dictionary of Sec. 2 ("hash dictionary that
+ * maps f-grams to matrix indices"), built on the GPU. Synchronous.
+ *
+ *  fgram_tok  host int32 [n_fgrams * K]: f-gram r is fgram_tok[r*K .. r*K+len-1],
+ *             oldest token first; entries past the length are ignored.
+ *  fgram_len  host uint8 [n_fgrams], each in [2, K] (1-grams are not f-grams, Sec. 3).
+ *  n_fgrams   >= 0. Row r of F belongs to f-gram r (its index in this list).
+ *  K          maximum f-gram length, 2..8.
+ *  vocab      token ids are [0, vocab); every f-gram token must be in range.
+ *  d          embedding width (elements per row), >= 1.
+ *  F          [n_fgrams * d] bf16 rows; a device address, or a host address of
+ *             mapped pinned memory when F_location = SCONE_ROWS_HOST_MAPPED.
+ *             May be NULL only when n_fgrams = 0.
+ *  T          device [vocab * d] bf16 token embeddings (Sec. 2: T stays on the
+ *             accelerator).
+ *  load_factor  target fill of the slot array, in (0, 0.95]; 0 selects 0.5.
+ *  stream     used for the build kernels; the call synchronizes it.
+ *  out        receives the table.
+ *
+ * The table borrows F and T (they must outlive it) and owns only its slot
+ * array (16 or 32 bytes per slot, 32-byte buckets) and a status word. Errors:
+ * INVALID_ARG (bad list, length, token or pointer), DUPLICATE_FGRAM,
+ * UNSUPPORTED (key does not fit: K*ceil(log2 vocab) > 220), NOMEM, CUDA.
+ */
+int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_len, int64_t n_fgrams,
+                      int32_t K, int32_t vocab, int32_t d, const scone_bf16* F,
+                      int32_t F_location, const scone_bf16* T, float load_factor, void* stream,
+                      scone_table** out);
+
+/* Frees the slot array and status word (after a device synchronize). NULL is a no-op. */
+int scone_table_destroy(scone_table* table);
+
+/* Host-side description of a built table (sizes are in bytes). */
+typedef struct scone_table_info {
+  int64_t n_fgrams;
+  int64_t n_slots;
+  int64_t n_buckets;
+  int32_t slot_bytes;        /* 16 or 32 */
+  int32_t key_bits;          /* K * bits_per_token + 4 length bits */
+  int32_t bits_per_token;
+  int32_t K;
+  int32_t vocab;
+  int32_t d;
+  int32_t F_location;
+  int32_t max_insert_probe;  /* most buckets any f-gram insert read */
+  int64_t table_bytes;       /* slot array */
+  int64_t F_bytes;           /* n_fgrams * d * 2 (borrowed) */
+  int64_t T_bytes;           /* vocab * d * 2 (borrowed) */
+} scone_table_info;
+
+int scone_table_get_info(const scone_table* table, scone_table_info* info);
+
+/*
+ * Diagnostic: caps the buckets one lookup may read (default: all of them).
+ * A lookup that reaches the cap records SCONE_ERR_PROBE_LIMIT and treats the
+ * position as an error position. max_buckets >= 1.
+ */
+int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
+
+/*
+ * scone_match — the selection step of Algorithm 1 (Sec. 3): for each
+ * position, the length of the longest f-gram ending there and its row of F.
+ * Probes lengths 2..min(K, i+1), i.e. at most K-1 lookups per token, the
+ * bound Sec. 4.3 states ("up to four queries per token" for K = 5). Async.
+ *
+ *  tok  device int32 [B * L]; row device int32 [B * L] (F row, or -1 when T
+ *  is used or on error); len device uint8 [B * L] or NULL (n in 2..K for an
+ *  f-gram, 1 for the token fallback, 0 for an error position).
+ */
+int scone_match(const scone_table* table, const int32_t* tok, int32_t B, int32_t L,
+                int32_t* row, uint8_t* len, void* stream);
+
+/*
+ * scone_embed_gather — the emission step of Algorithm 1 (Sec. 3): for each
+ * of n_tok positions, out[t] = F[row[t]] if row[t] >= 0, else T[tok[t]]
+ * (a zero row when tok[t] is out of range or row[t] >= n_fgrams, which also
+ * sets the sticky status). tok, row device [n_tok]; out device [n_tok * d].
+ * Async.
+ */
+int scone_embed_gather(const scone_table* table, const int32_t* tok, const int32_t* row,
+                       int64_t n_tok, scone_bf16* out, void* stream);
+
+/*
+ * scone_embed — Algorithm 1 end to end (Sec. 3, inference branch) in one
+ * launch: match and gather fused, no intermediate row array in memory.
+ * tok device [B * L]; out device [B * L * d]; row / len as in scone_match,
+ * each may be NULL. Async.
+ */
+int scone_embed(const scone_table* table, const int32_t* tok, int32_t B, int32_t L,
+                scone_bf16* out, int32_t* row, uint8_t* len, void* stream);
+
+/*
+ * Decode (Sec. 3.2: T stays on the accelerator "for decoding", F is looked
+ * up per generated token). A decode state holds, per live sequence, its last
+ * K-1 tokens on the device, which is all Algorithm 1 needs for the next
+ * position.
+ *
+ * scone_decode_create: S live sequences. hist host int32 [S * (K-1)]: the
+ * sequence's known tokens right-aligned in its row (entries left of the last
+ * hist_len[s] are ignored); hist_len host int32 [S] in [0, K-1]. Synchronous.
+ */
+int scone_decode_create(const scone_table* table, int32_t S, const int32_t* hist,
+                        const int32_t* hist_len, scone_decode** out);
+
+/*
+ * scone_decode_step: appends new_tok[s] (device int32 [S]) to sequence s,
+ * embeds it by Algorithm 1 over the sequence so far, and writes
+ * out device [S * d]; row device int32 [S] and len device uint8 [S] may be
+ * NULL. Async; steps on one state must be ordered on one stream.
+ */
+int scone_decode_step(scone_decode* state, const int32_t* new_tok, scone_bf16* out, int32_t* row,
+                      uint8_t* len, void* stream);
+
+/* Copies the device history back: hist host [S * (K-1)], hist_len host [S]. Synchronous. */
+int scone_decode_get_history(const scone_decode* state, int32_t* hist, int32_t* hist_len);
+
+int scone_decode_destroy(scone_decode* state);
+
+/*
+ * scone_status: synchronizes `stream`, returns the first device-detected
+ * error recorded since the last call (SCONE_OK if none) and clears it.
+ */
+int scone_status(const scone_table* table, void* stream);
+
+/*
+ * Host memory for the offloaded tier: pinned and mapped into the device
+ * address space (cudaHostAlloc with cudaHostAllocMapped | cudaHostAllocPortable),
+ * so kernels read it over the host link. Use it for F with
+ * SCONE_ROWS_HOST_MAPPED. Synchronous. Errors: INVALID_ARG (bytes < 1 or
+ * out NULL), NOMEM (the pinned allocation failed; *out is NULL).
+ */
+int scone_host_alloc(int64_t bytes, void** out);
+
+/* Frees memory from scone_host_alloc (after a device synchronize). NULL is a no-op. */
+int scone_host_free(void* p);
+
+/* Static description of an error code. */
+const char* scone_strerror(int code);
+
+/* ABI version, (major << 16) | minor. */
+int scone_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SCONE_H_ */

@@ -1,0 +1,319 @@
+"""SCONE inference-time input embedding on one GB300 (sm_103a).
+
+Thin Python binding over the C ABI in ``include/scone.h`` (``libscone.so``,
+built next to this file by ``__graft_entry__.build()``). Every function has
+the C name and only marshals arguments: torch tensors become device
+addresses, the current CUDA stream is passed through, and every step of the
+path runs in the library's kernels. There is no CPU fallback: if the
+library is missing or a call fails, an exception is raised.
+
+Tensors carrying bf16 rows may be ``torch.bfloat16`` or ``torch.int16``
+(raw bits); token tensors are ``torch.int32``.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libscone.so")
+
+SCONE_OK = 0
+SCONE_ERR_INVALID_ARG = -1
+SCONE_ERR_TOKEN_RANGE = -2
+SCONE_ERR_DUPLICATE_FGRAM = -3
+SCONE_ERR_TABLE_FULL = -4
+SCONE_ERR_PROBE_LIMIT = -5
+SCONE_ERR_UNSUPPORTED = -6
+SCONE_ERR_CUDA = -7
+SCONE_ERR_NOMEM = -8
+SCONE_ROWS_DEVICE = 0
+SCONE_ROWS_HOST_MAPPED = 1
+
+EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_get_info",
+           "scone_table_set_probe_limit", "scone_match", "scone_embed_gather", "scone_embed",
+           "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
+           "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
+           "scone_strerror", "scone_version")
+
+_lib = None
+_vp = ctypes.c_void_p
+_i32, _i64 = ctypes.c_int32, ctypes.c_int64
+
+
+class SconeError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        msg = load_library().scone_strerror(code).decode()
+        super().__init__(f"{what}: {msg} ({code})")
+        self.code = code
+
+
+class scone_table_info(ctypes.Structure):
+    _fields_ = [("n_fgrams", _i64), ("n_slots", _i64), ("n_buckets", _i64),
+                ("slot_bytes", _i32), ("key_bits", _i32), ("bits_per_token", _i32),
+                ("K", _i32), ("vocab", _i32), ("d", _i32), ("F_location", _i32),
+                ("max_insert_probe", _i32), ("table_bytes", _i64), ("F_bytes", _i64),
+                ("T_bytes", _i64)]
+
+    def as_dict(self):
+        return {k: getattr(self, k) for k, _ in self._fields_}
+
+
+def load_library():
+    """Loads libscone.so (raises if it was not built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: run __graft_entry__.build() "
+                           "(there is no CPU fallback)")
+    lib = ctypes.CDLL(LIB_PATH)
+    lib.scone_table_build.argtypes = [_vp, _vp, _i64, _i32, _i32, _i32, _vp, _i32, _vp,
+                                      ctypes.c_float, _vp, ctypes.POINTER(_vp)]
+    lib.scone_table_destroy.argtypes = [_vp]
+    lib.scone_table_get_info.argtypes = [_vp, ctypes.POINTER(scone_table_info)]
+    lib.scone_table_set_probe_limit.argtypes = [_vp, _i64]
+    lib.scone_match.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp]
+    lib.scone_embed_gather.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
+    lib.scone_embed.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]
+    lib.scone_decode_create.argtypes = [_vp, _i32, _vp, _vp, ctypes.POINTER(_vp)]
+    lib.scone_decode_step.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp]
+    lib.scone_decode_get_history.argtypes = [_vp, _vp, _vp]
+    lib.scone_decode_destroy.argtypes = [_vp]
+    lib.scone_status.argtypes = [_vp, _vp]
+    lib.scone_host_alloc.argtypes = [_i64, ctypes.POINTER(_vp)]
+    lib.scone_host_free.argtypes = [_vp]
+    lib.scone_strerror.argtypes = [ctypes.c_int]
+    lib.scone_strerror.restype = ctypes.c_char_p
+    lib.scone_version.argtypes = []
+    for name in EXPORTS:
+        if name != "scone_strerror":
+            getattr(lib, name).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def _check(rc: int, what: str):
+    if rc != SCONE_OK:
+        raise SconeError(rc, what)
+
+
+def _stream(stream) -> int:
+    import torch
+
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _ptr(t) -> Optional[int]:
+    """Address of a tensor, numpy array, raw int address, or None."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if isinstance(t, np.ndarray):
+        assert t.flags["C_CONTIGUOUS"]
+        return t.ctypes.data
+    assert t.is_contiguous(), "tensors must be contiguous"
+    return t.data_ptr()
+
+
+class Table:
+    """A built f-gram table (owns the C handle; borrows F and T)."""
+
+    def __init__(self, handle: ctypes.c_void_p, keep):
+        self._h = handle
+        self._keep = keep   # F and T must outlive the table
+
+    @property
+    def handle(self) -> ctypes.c_void_p:
+        if self._h is None:
+            raise RuntimeError("table was closed")
+        return self._h
+
+    def info(self) -> dict:
+        return scone_table_get_info(self)
+
+    def close(self):
+        if self._h is not None:
+            load_library().scone_table_destroy(self._h)
+            self._h = None
+            self._keep = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def scone_table_build(fgram_tok: np.ndarray, fgram_len: np.ndarray, K: int, vocab: int, d: int,
+                      F, T, F_location: int = SCONE_ROWS_DEVICE, load_factor: float = 0.0,
+                      stream=None) -> Table:
+    """Builds the f-gram table. fgram_tok host [N, K] int32, fgram_len host [N] uint8.
+
+    F is a device tensor [N, d] (or a host-mapped address when F_location is
+    SCONE_ROWS_HOST_MAPPED); T a device tensor [vocab, d].
+    """
+    lib = load_library()
+    ft = np.ascontiguousarray(fgram_tok, dtype=np.int32).reshape(-1)
+    fl = np.ascontiguousarray(fgram_len, dtype=np.uint8).reshape(-1)
+    n = fl.shape[0]
+    if ft.shape[0] != n * K:
+        raise ValueError("fgram_tok must be [n_fgrams, K]")
+    h = _vp()
+    rc = lib.scone_table_build(_ptr(ft) if n else None, _ptr(fl) if n else None, n, K, vocab, d,
+                               _ptr(F), F_location, _ptr(T), load_factor, _stream(stream),
+                               ctypes.byref(h))
+    _check(rc, "scone_table_build")
+    return Table(h, (F, T))
+
+
+def scone_table_destroy(table: Table) -> None:
+    table.close()
+
+
+def scone_table_get_info(table: Table) -> dict:
+    info = scone_table_info()
+    _check(load_library().scone_table_get_info(table.handle, ctypes.byref(info)),
+           "scone_table_get_info")
+    return info.as_dict()
+
+
+def scone_table_set_probe_limit(table: Table, max_buckets: int) -> None:
+    _check(load_library().scone_table_set_probe_limit(table.handle, max_buckets),
+           "scone_table_set_probe_limit")
+
+
+def _bl(tok):
+    if tok.dim() == 2:
+        return tok.shape[0], tok.shape[1]
+    return 1, tok.shape[0]
+
+
+def scone_match(table: Table, tok, row, len=None, stream=None) -> None:
+    """tok [B, L] (or [n]) int32 device; row int32 and len uint8 of the same count."""
+    B, L = _bl(tok)
+    _check(load_library().scone_match(table.handle, _ptr(tok), B, L, _ptr(row), _ptr(len),
+                                      _stream(stream)), "scone_match")
+
+
+def scone_embed_gather(table: Table, tok, row, out, stream=None) -> None:
+    _check(load_library().scone_embed_gather(table.handle, _ptr(tok), _ptr(row), tok.numel(),
+                                             _ptr(out), _stream(stream)), "scone_embed_gather")
+
+
+def scone_embed(table: Table, tok, out, row=None, len=None, stream=None) -> None:
+    """Fused Algorithm 1: out [B*L, d] bf16 rows; row / len optional."""
+    B, L = _bl(tok)
+    _check(load_library().scone_embed(table.handle, _ptr(tok), B, L, _ptr(out), _ptr(row),
+                                      _ptr(len), _stream(stream)), "scone_embed")
+
+
+class DecodeState:
+    def __init__(self, handle, table: Table, S: int, H: int):
+        self._h = handle
+        self._table = table
+        self.S, self.H = S, H
+
+    @property
+    def handle(self):
+        if self._h is None:
+            raise RuntimeError("decode state was closed")
+        return self._h
+
+    def close(self):
+        if self._h is not None:
+            load_library().scone_decode_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def scone_decode_create(table: Table, hist: np.ndarray, hist_len: np.ndarray) -> DecodeState:
+    """hist host [S, K-1] int32 right-aligned; hist_len host [S] int32 in [0, K-1]."""
+    hist = np.ascontiguousarray(hist, dtype=np.int32)
+    hl = np.ascontiguousarray(hist_len, dtype=np.int32)
+    S = hl.shape[0]
+    h = _vp()
+    _check(load_library().scone_decode_create(table.handle, S, _ptr(hist), _ptr(hl),
+                                              ctypes.byref(h)), "scone_decode_create")
+    return DecodeState(h, table, S, hist.shape[1] if hist.ndim == 2 else 0)
+
+
+def scone_decode_step(state: DecodeState, new_tok, out, row=None, len=None, stream=None) -> None:
+    _check(load_library().scone_decode_step(state.handle, _ptr(new_tok), _ptr(out), _ptr(row),
+                                            _ptr(len), _stream(stream)), "scone_decode_step")
+
+
+def scone_decode_get_history(state: DecodeState):
+    hist = np.empty((state.S, state.H), np.int32)
+    hl = np.empty(state.S, np.int32)
+    _check(load_library().scone_decode_get_history(state.handle, _ptr(hist), _ptr(hl)),
+           "scone_decode_get_history")
+    return hist, hl
+
+
+def scone_decode_destroy(state: DecodeState) -> None:
+    state.close()
+
+
+def scone_status(table: Table, stream=None, raise_on_error: bool = True) -> int:
+    """Synchronizes the stream; returns (or raises) the sticky device error."""
+    rc = load_library().scone_status(table.handle, _stream(stream))
+    if raise_on_error:
+        _check(rc, "device status")
+    return rc
+
+
+class HostBuffer:
+    """Pinned, device-mapped host memory from scone_host_alloc (for an offloaded F)."""
+
+    def __init__(self, nbytes: int):
+        p = _vp()
+        _check(load_library().scone_host_alloc(nbytes, ctypes.byref(p)), "scone_host_alloc")
+        self.ptr = p.value
+        self.nbytes = nbytes
+
+    def numpy(self, dtype=np.uint16) -> np.ndarray:
+        """Host view of the buffer (no copy)."""
+        buf = (ctypes.c_char * self.nbytes).from_address(self.ptr)
+        return np.frombuffer(buf, dtype=dtype)
+
+    def free(self):
+        if self.ptr:
+            load_library().scone_host_free(self.ptr)
+            self.ptr = 0
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def scone_host_alloc(nbytes: int) -> HostBuffer:
+    return HostBuffer(nbytes)
+
+
+def scone_host_free(buf: HostBuffer) -> None:
+    buf.free()
+
+
+def scone_strerror(code: int) -> str:
+    return load_library().scone_strerror(code).decode()
+
+
+def scone_version() -> int:
+    return load_library().scone_version()

@@ -1,0 +1,216 @@
+// Decode step: one new token per live sequence (Sec. 3.2: at inference F is
+// looked up per generated token while T stays on the accelerator).
+//
+// Algorithm 1 only needs the last K-1 tokens before a position, so the state
+// keeps, per sequence, a device ring of its last K-1 tokens (right-aligned,
+// oldest first) and how many of them are known. One warp serves one
+// sequence: lane j probes the window of length j + 2 ending at the new token
+// (a full linear-probe lookup each), a warp ballot keeps the longest hit,
+// the lanes shift the new token into the history, and the warp copies the
+// selected row (F over the host link in the offloaded tier, or T from HBM)
+// with every lane's loads issued at once.
+
+#include <new>
+
+#include "scone_host.h"
+
+namespace scone {
+
+constexpr int kDecThreads = 128;
+constexpr int kDecWarps = kDecThreads / 32;
+
+namespace {
+
+template <int FMT>
+__device__ __forceinline__ int32_t lookup(const TableView& t, const KeyBits<Fmt<FMT>::kWords>& k,
+                                          int* err) {
+  uint64_t q = fastrange(key_hash<FMT>(k), t.n_buckets);
+  int32_t r = check_bucket<FMT>(ld_bucket(t.slots + q * kBucketBytes), k);
+  int64_t reads = 1;
+  while (r == -2) {
+    if (reads >= t.probe_limit) {
+      *err = SCONE_ERR_PROBE_LIMIT;
+      return -1;
+    }
+    q = (q + 1 == t.n_buckets) ? 0 : q + 1;
+    r = check_bucket<FMT>(ld_bucket(t.slots + q * kBucketBytes), k);
+    ++reads;
+  }
+  return r;
+}
+
+template <int FMT, int W>
+__global__ void __launch_bounds__(kDecThreads)
+    decode_kernel(const TableView t, int32_t* __restrict__ hist, int32_t* __restrict__ hist_len,
+                  const int32_t* __restrict__ new_tok, int32_t S, int32_t H,
+                  uint8_t* __restrict__ out, int32_t* __restrict__ row_out,
+                  uint8_t* __restrict__ len_out, int width) {
+  constexpr int NW = Fmt<FMT>::kWords;
+  __shared__ const void* src_s[kDecWarps][1];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int row_bytes = t.d * 2;
+  for (int64_t s = (int64_t)blockIdx.x * kDecWarps + warp; s < S;
+       s += (int64_t)gridDim.x * kDecWarps) {
+    const int32_t x = __ldg(new_tok + s);
+    const int32_t h = hist_len[s];
+    int32_t* hs = hist + s * H;
+    const bool xvalid = valid_token(x, t.vocab);
+    const int n = lane + 2;
+    int32_t r_lane = -1;
+    int err = 0;
+    if (xvalid && n <= t.K && n <= h + 1) {
+      KeyBits<NW> k;
+#pragma unroll
+      for (int q = 0; q < NW; ++q) k.w[q] = 0;
+      k.w[0] = (uint32_t)x;
+      bool ok = true;
+      for (int m = 1; m < n; ++m) {
+        const int32_t y = hs[H - m];
+        ok = ok && valid_token(y, t.vocab);
+        put_field<NW>(k, m * t.bits, (uint32_t)y, t.bits);
+      }
+      put_len<FMT>(k, n);
+      if (ok) r_lane = lookup<FMT>(t, k, &err);
+    }
+    const unsigned hits = __ballot_sync(0xFFFFFFFFu, r_lane >= 0);
+    const unsigned errs = __ballot_sync(0xFFFFFFFFu, err != 0);
+    const int best = hits ? 31 - __clz(hits) : -1;
+    int32_t r = __shfl_sync(0xFFFFFFFFu, r_lane, best >= 0 ? best : 0);
+    // a probe-limit error matters only at a length longer than the best hit,
+    // the same outcome as the longest-first scan of the prefill path
+    const bool probe_err = (best >= 0 ? (errs >> (best + 1)) : errs) != 0;
+    int len;
+    const void* src = nullptr;
+    if (!xvalid || probe_err) {
+      r = -1;
+      len = 0;
+    } else {
+      if (best < 0) r = -1;
+      len = best >= 0 ? best + 2 : 1;
+      src = r >= 0 ? static_cast<const void*>(t.F + (int64_t)r * t.d)
+                   : static_cast<const void*>(t.T + (int64_t)x * t.d);
+    }
+    // shift the new token into the history (all lanes have read it above)
+    int32_t keep = 0;
+    if (lane < H) keep = lane + 1 < H ? hs[lane + 1] : x;
+    __syncwarp();
+    if (lane < H) hs[lane] = keep;
+    if (lane == 0) {
+      hist_len[s] = h + 1 < H ? h + 1 : H;
+      if (row_out) row_out[s] = r;
+      if (len_out) len_out[s] = (uint8_t)len;
+      if (!xvalid) record_error(t.status, SCONE_ERR_TOKEN_RANGE);
+      else if (probe_err) record_error(t.status, SCONE_ERR_PROBE_LIMIT);
+      src_s[warp][0] = src;
+    }
+    __syncwarp();
+    warp_copy_rows_w<W>(src_s[warp], out + s * (int64_t)row_bytes, 1, row_bytes, width, lane);
+    __syncwarp();
+  }
+}
+
+using DecodeFn = void (*)(TableView, int32_t*, int32_t*, const int32_t*, int32_t, int32_t,
+                          uint8_t*, int32_t*, uint8_t*, int);
+
+DecodeFn pick_decode(int fmt, int width) {
+  if (fmt == FMT16) return width == 16 ? decode_kernel<FMT16, 16> : decode_kernel<FMT16, 0>;
+  return width == 16 ? decode_kernel<FMT32, 16> : decode_kernel<FMT32, 0>;
+}
+
+int decode_width(const TableView& t, const void* out) {
+  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)(t.d * 2);
+  if (t.n_fgrams > 0) a |= (uintptr_t)t.F;
+  if ((a & 15) == 0) return 16;
+  if ((a & 7) == 0) return 8;
+  if ((a & 3) == 0) return 4;
+  return 2;
+}
+
+}  // namespace
+
+}  // namespace scone
+
+using namespace scone;
+
+extern "C" int scone_decode_create(const scone_table* tb, int32_t S, const int32_t* hist,
+                                   const int32_t* hist_len, scone_decode** out) {
+  if (!out) return SCONE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!tb || S < 0 || (S > 0 && (!hist || !hist_len))) return SCONE_ERR_INVALID_ARG;
+  const int32_t H = tb->view.K - 1;
+  for (int32_t s = 0; s < S; ++s)
+    if (hist_len[s] < 0 || hist_len[s] > H) return SCONE_ERR_INVALID_ARG;
+  DeviceGuard g(tb->device);
+  scone_decode* st = new (std::nothrow) scone_decode();
+  if (!st) return SCONE_ERR_NOMEM;
+  st->table = tb;
+  st->S = S;
+  st->H = H;
+  if (S > 0) {
+    if (cudaMalloc(&st->hist, (size_t)S * H * sizeof(int32_t)) != cudaSuccess ||
+        cudaMalloc(&st->hist_len, (size_t)S * sizeof(int32_t)) != cudaSuccess) {
+      cudaGetLastError();
+      scone_decode_destroy(st);
+      return SCONE_ERR_NOMEM;
+    }
+    if (cudaMemcpy(st->hist, hist, (size_t)S * H * sizeof(int32_t), cudaMemcpyHostToDevice) !=
+            cudaSuccess ||
+        cudaMemcpy(st->hist_len, hist_len, (size_t)S * sizeof(int32_t),
+                   cudaMemcpyHostToDevice) != cudaSuccess) {
+      cudaGetLastError();
+      scone_decode_destroy(st);
+      return SCONE_ERR_CUDA;
+    }
+  }
+  *out = st;
+  return SCONE_OK;
+}
+
+extern "C" int scone_decode_step(scone_decode* st, const int32_t* new_tok, scone_bf16* out,
+                                 int32_t* row, uint8_t* len, void* stream) {
+  if (!st || !st->table) return SCONE_ERR_INVALID_ARG;
+  if (st->S == 0) return SCONE_OK;
+  if (!new_tok || !out || ((uintptr_t)new_tok & 3) || ((uintptr_t)out & 1) ||
+      (row && ((uintptr_t)row & 3)))
+    return SCONE_ERR_INVALID_ARG;
+  const scone_table* tb = st->table;
+  DeviceGuard g(tb->device);
+  const int width = decode_width(tb->view, out);
+  const DecodeFn fn = pick_decode(tb->fmt, width);
+  const int64_t need = (st->S + kDecWarps - 1) / kDecWarps;
+  const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)fn, kDecThreads, 0);
+  const int grid = (int)(need < cap ? need : cap);
+  fn<<<grid, kDecThreads, 0, (cudaStream_t)stream>>>(tb->view, st->hist, st->hist_len, new_tok,
+                                                     st->S, st->H,
+                                                     reinterpret_cast<uint8_t*>(out), row, len,
+                                                     width);
+  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}
+
+extern "C" int scone_decode_get_history(const scone_decode* st, int32_t* hist,
+                                        int32_t* hist_len) {
+  if (!st || (st->S > 0 && (!hist || !hist_len))) return SCONE_ERR_INVALID_ARG;
+  if (st->S == 0) return SCONE_OK;
+  DeviceGuard g(st->table->device);
+  if (cudaDeviceSynchronize() != cudaSuccess ||
+      cudaMemcpy(hist, st->hist, (size_t)st->S * st->H * sizeof(int32_t),
+                 cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemcpy(hist_len, st->hist_len, (size_t)st->S * sizeof(int32_t),
+                 cudaMemcpyDeviceToHost) != cudaSuccess) {
+    cudaGetLastError();
+    return SCONE_ERR_CUDA;
+  }
+  return SCONE_OK;
+}
+
+extern "C" int scone_decode_destroy(scone_decode* st) {
+  if (!st) return SCONE_OK;
+  if (st->hist || st->hist_len) {
+    DeviceGuard g(st->table ? st->table->device : 0);
+    cudaDeviceSynchronize();
+    if (st->hist) cudaFree(st->hist);
+    if (st->hist_len) cudaFree(st->hist_len);
+  }
+  delete st;
+  return SCONE_OK;
+}

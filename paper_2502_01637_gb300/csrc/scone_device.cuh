@@ -1,0 +1,317 @@
+// Device-side building blocks of the SCONE embedding path (sm_103a).
+//
+// The f-gram dictionary (Sec. 2, "a hash dictionary that maps f-grams to
+// matrix indices") is an open-addressing table with linear probing over
+// 32-byte buckets. Every bucket is one DRAM sector and is read with one
+// 256-bit load.
+//
+// Key: an injective packing of the n-gram. Token fields of b bits
+// (b = ceil(log2 vocab)) hold the newest token at bit 0, the one before it
+// at bit b, and so on, so the key of length n+1 extends the key of length n
+// by one field; the length n sits in a 4-bit field at the top of the key.
+// n >= 2, so a valid key is never all ones, which marks an empty slot.
+//
+//   FMT16: key of 96 bits (K*b <= 92), 16-byte slot = {key bits 0..63,
+//          key bits 64..95 | row << 32}; two slots per bucket.
+//   FMT32: key of 224 bits (K*b <= 220), 32-byte slot = {key 0..63,
+//          64..127, 128..191, key 192..223 | row << 32}; one slot per bucket.
+//
+// The row word of an empty slot is 0xFFFFFFFF (row -1).
+
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "scone.h"
+
+namespace scone {
+
+constexpr int kBucketBytes = 32;
+constexpr int FMT16 = 0;
+constexpr int FMT32 = 1;
+constexpr uint32_t kEmptyRow = 0xFFFFFFFFu;
+constexpr uint64_t kHashSeed = 0x6A09E667F3BCC908ull;  // frac(sqrt 2), first 64 bits
+
+template <int FMT>
+struct Fmt;
+template <>
+struct Fmt<FMT16> {
+  static constexpr int kWords = 2;        // 64-bit key words (96 bits used)
+  static constexpr int kSlotsPerBucket = 2;
+  static constexpr int kLenShift = 28;    // length field in bits 92..95 (word 1, bits 28..31)
+};
+template <>
+struct Fmt<FMT32> {
+  static constexpr int kWords = 4;        // 224 bits used
+  static constexpr int kSlotsPerBucket = 1;
+  static constexpr int kLenShift = 28;    // bits 220..223 (word 3, bits 28..31)
+};
+
+// What a kernel needs to know about a table (passed by value).
+struct TableView {
+  const uint8_t* slots;      // bucket q at slots + 32 q
+  uint64_t n_buckets;
+  int64_t probe_limit;       // buckets one lookup may read
+  int64_t n_fgrams;
+  const uint16_t* F;         // device-accessible address of F (HBM or host-mapped)
+  const uint16_t* T;
+  int* status;               // sticky first device-detected error
+  int32_t K;
+  int32_t bits;
+  int32_t vocab;
+  int32_t d;
+};
+
+template <int NW>
+struct KeyBits {
+  uint64_t w[NW];
+};
+
+struct Bucket {
+  uint64_t a, b, c, e;
+};
+
+__device__ __forceinline__ uint64_t fmix64(uint64_t z) {
+  // SplitMix64 / MurmurHash3 finalizer (Steele, Lea, Flood 2014)
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Inserts field value v (< 2^b) at bit offset off.
+template <int NW>
+__device__ __forceinline__ void put_field(KeyBits<NW>& k, int off, uint32_t v, int b) {
+#pragma unroll
+  for (int q = 0; q < NW; ++q) {
+    const int rel = off - 64 * q;
+    if (rel >= 0 && rel < 64) {
+      k.w[q] |= (uint64_t)v << rel;
+    } else if (rel < 0 && rel > -b) {
+      k.w[q] |= (uint64_t)v >> (-rel);
+    }
+  }
+}
+
+template <int FMT>
+__device__ __forceinline__ void put_len(KeyBits<Fmt<FMT>::kWords>& k, int n) {
+  k.w[Fmt<FMT>::kWords - 1] |= (uint64_t)n << Fmt<FMT>::kLenShift;
+}
+
+template <int FMT>
+__device__ __forceinline__ uint64_t key_hash(const KeyBits<Fmt<FMT>::kWords>& k) {
+  uint64_t h = kHashSeed;
+#pragma unroll
+  for (int q = Fmt<FMT>::kWords - 1; q >= 0; --q) h = fmix64(k.w[q] ^ h);
+  return h;
+}
+
+// Lemire's multiply-shift range reduction: maps h uniformly onto [0, n).
+__device__ __forceinline__ uint64_t fastrange(uint64_t h, uint64_t n) { return __umul64hi(h, n); }
+
+// One 256-bit read-only load of a bucket.
+__device__ __forceinline__ Bucket ld_bucket(const uint8_t* p) {
+  Bucket r;
+  asm("ld.global.nc.v4.u64 {%0, %1, %2, %3}, [%4];"
+      : "=l"(r.a), "=l"(r.b), "=l"(r.c), "=l"(r.e)
+      : "l"(p));
+  return r;
+}
+
+// >= 0: the key's row. -1: definitive miss (an empty slot ends the probe run).
+// -2: bucket full of other keys, continue with the next bucket.
+template <int FMT>
+__device__ __forceinline__ int32_t check_bucket(const Bucket& v,
+                                                const KeyBits<Fmt<FMT>::kWords>& k) {
+  if constexpr (FMT == FMT16) {
+    if (v.a == k.w[0] && (uint32_t)v.b == (uint32_t)k.w[1]) return (int32_t)(v.b >> 32);
+    if ((uint32_t)(v.b >> 32) == kEmptyRow) return -1;
+    if (v.c == k.w[0] && (uint32_t)v.e == (uint32_t)k.w[1]) return (int32_t)(v.e >> 32);
+    if ((uint32_t)(v.e >> 32) == kEmptyRow) return -1;
+    return -2;
+  } else {
+    if (v.a == k.w[0] && v.b == k.w[1] && v.c == k.w[2] && (uint32_t)v.e == (uint32_t)k.w[3])
+      return (int32_t)(v.e >> 32);
+    if ((uint32_t)(v.e >> 32) == kEmptyRow) return -1;
+    return -2;
+  }
+}
+
+__device__ __forceinline__ void record_error(int* status, int code) {
+  if (*reinterpret_cast<volatile int*>(status) == 0) atomicCAS(status, 0, code);
+}
+
+__device__ __forceinline__ bool valid_token(int32_t x, int32_t vocab) {
+  return (uint32_t)x < (uint32_t)vocab;
+}
+
+// Algorithm 1's selection for one position: the longest n in [2, min(K, i+1)]
+// whose window (tok[p-n+1 .. p]) is an f-gram. All candidate lengths are
+// hashed in registers and their home buckets loaded together (K-1 loads in
+// flight), then resolved longest first; a full bucket continues the linear
+// probe. Returns the row (or -1) and sets *len (n, 1 for the token fallback,
+// 0 for an error position) and *err.
+template <int FMT, int KT>
+__device__ __forceinline__ int32_t match_position(const TableView& t,
+                                                  const int32_t* __restrict__ tok, int64_t p,
+                                                  int32_t i, int32_t tok_p, int* len, int* err) {
+  constexpr int NW = Fmt<FMT>::kWords;
+  if (!valid_token(tok_p, t.vocab)) {
+    *err = SCONE_ERR_TOKEN_RANGE;
+    *len = 0;
+    return -1;
+  }
+  int nmax = t.K < i + 1 ? t.K : i + 1;
+  int32_t w[KT];
+  w[0] = tok_p;
+#pragma unroll
+  for (int j = 1; j < KT; ++j) w[j] = (j < nmax) ? __ldg(tok + p - j) : 0;
+  // a window is usable only if all its tokens are valid
+  int nvalid = 1;
+#pragma unroll
+  for (int j = 1; j < KT; ++j)
+    if (nvalid == j && j < nmax && valid_token(w[j], t.vocab)) nvalid = j + 1;
+  nmax = nvalid;
+
+  KeyBits<NW> acc;
+#pragma unroll
+  for (int q = 0; q < NW; ++q) acc.w[q] = 0;
+  acc.w[0] = (uint32_t)w[0];
+  KeyBits<NW> keys[KT - 1];
+  uint64_t home[KT - 1];
+  Bucket first[KT - 1];
+#pragma unroll
+  for (int n = 2; n <= KT; ++n) {
+    put_field<NW>(acc, (n - 1) * t.bits, (uint32_t)w[n - 1], t.bits);
+    keys[n - 2] = acc;
+    put_len<FMT>(keys[n - 2], n);
+    if (n <= nmax) {
+      home[n - 2] = fastrange(key_hash<FMT>(keys[n - 2]), t.n_buckets);
+      first[n - 2] = ld_bucket(t.slots + home[n - 2] * kBucketBytes);
+    }
+  }
+#pragma unroll
+  for (int n = KT; n >= 2; --n) {
+    if (n > nmax) continue;
+    int32_t r = check_bucket<FMT>(first[n - 2], keys[n - 2]);
+    uint64_t q = home[n - 2];
+    int64_t reads = 1;
+    while (r == -2) {
+      if (reads >= t.probe_limit) {
+        *err = SCONE_ERR_PROBE_LIMIT;
+        *len = 0;
+        return -1;
+      }
+      q = (q + 1 == t.n_buckets) ? 0 : q + 1;
+      r = check_bucket<FMT>(ld_bucket(t.slots + q * kBucketBytes), keys[n - 2]);
+      ++reads;
+    }
+    if (r >= 0) {
+      *len = n;
+      return r;
+    }
+  }
+  *len = 1;
+  return -1;
+}
+
+// ------------------------------------------------------------- row copies
+template <typename E>
+__device__ __forceinline__ E ld_row(const E* p) {
+  return __ldg(p);
+}
+template <>
+__device__ __forceinline__ uint4 ld_row<uint4>(const uint4* p) {
+  uint4 v;
+  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+      : "l"(p));
+  return v;
+}
+
+template <typename E>
+__device__ __forceinline__ void st_out(E* p, const E& v) {
+  __stcs(p, v);
+}
+
+template <typename E>
+__device__ __forceinline__ E zero_of() {
+  return E{};
+}
+template <>
+__device__ __forceinline__ uint4 zero_of<uint4>() {
+  return make_uint4(0, 0, 0, 0);
+}
+template <>
+__device__ __forceinline__ uint2 zero_of<uint2>() {
+  return make_uint2(0, 0);
+}
+
+constexpr int kLoadsInFlight = 16;
+
+// A warp copies nrows rows of epr elements of type E: row r from src[r]
+// (NULL writes zeros) to dst + r * epr, rows contiguous in dst. The warp
+// walks the nrows * epr elements in order, lane l taking every 32nd one, and
+// keeps U loads per lane outstanding before the matching streaming stores.
+// (row, column) of a lane's element advance incrementally, so any row width
+// works without a division.
+template <typename E, int U>
+__device__ __forceinline__ void warp_copy_rows(const E* const* src, E* __restrict__ dst,
+                                               int nrows, int epr, int lane) {
+  const int64_t total = (int64_t)nrows * epr;
+  int r = 0, col = lane;
+  while (col >= epr) {
+    col -= epr;
+    ++r;
+  }
+  for (int64_t base = 0; base < total; base += 32 * U) {
+    E v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      v[u] = zero_of<E>();
+      if (r < nrows) {
+        const E* s = src[r];
+        if (s != nullptr) v[u] = ld_row<E>(s + col);
+      }
+      col += 32;
+      while (col >= epr) {
+        col -= epr;
+        ++r;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t c = base + 32 * u + lane;
+      if (c < total) st_out<E>(dst + c, v[u]);
+    }
+  }
+}
+
+// Row copy for a width chosen at run time: 16-byte chunks when W == 16,
+// otherwise the widest of 8, 4 or 2 bytes that the row size and all three
+// base addresses allow (width_bytes).
+template <int W>
+__device__ __forceinline__ void warp_copy_rows_w(const void* const* src, void* dst, int nrows,
+                                                 int row_bytes, int width_bytes, int lane) {
+  if constexpr (W == 16) {
+    warp_copy_rows<uint4, kLoadsInFlight>(reinterpret_cast<const uint4* const*>(src),
+                                          reinterpret_cast<uint4*>(dst), nrows, row_bytes >> 4,
+                                          lane);
+  } else {
+    if (width_bytes == 8) {
+      warp_copy_rows<uint2, kLoadsInFlight>(reinterpret_cast<const uint2* const*>(src),
+                                            reinterpret_cast<uint2*>(dst), nrows, row_bytes >> 3,
+                                            lane);
+    } else if (width_bytes == 4) {
+      warp_copy_rows<unsigned int, kLoadsInFlight>(
+          reinterpret_cast<const unsigned int* const*>(src), reinterpret_cast<unsigned int*>(dst),
+          nrows, row_bytes >> 2, lane);
+    } else {
+      warp_copy_rows<unsigned short, kLoadsInFlight>(
+          reinterpret_cast<const unsigned short* const*>(src),
+          reinterpret_cast<unsigned short*>(dst), nrows, row_bytes >> 1, lane);
+    }
+  }
+}
+
+}  // namespace scone

@@ -1,0 +1,240 @@
+// Prefill path: match, gather and the fused embed (Algorithm 1, inference
+// branch, Sec. 3), plus the launch helpers.
+//
+// Work split: one warp per tile of 32 consecutive positions of the flattened
+// [B x L] batch. Each lane matches one position (all K-1 candidate lengths
+// probed at once, longest hit kept), the 32 selected row addresses go to
+// shared memory, and the warp then streams the 32 rows to the contiguous
+// output block with 16-byte loads, 16 in flight per lane, and streaming
+// (evict-first) stores. Blocks are 8 warps; the grid is capped at the number
+// of blocks that are resident at once and walks the tiles grid-stride.
+
+#include <map>
+#include <mutex>
+#include <utility>
+
+#include "scone_host.h"
+
+namespace scone {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+
+int sm_count() {
+  int dev = 0, sms = 1;
+  cudaGetDevice(&dev);
+  static std::mutex mu;
+  static std::map<int, int> cache;
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = cache.find(dev);
+  if (it != cache.end()) return it->second;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cache[dev] = sms;
+  return sms;
+}
+
+int blocks_per_sm(const void* fn, int threads, size_t smem) {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int> cache;
+  std::lock_guard<std::mutex> lk(mu);
+  const auto key = std::make_pair(fn, dev * 4096 + threads);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  int n = 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, smem) != cudaSuccess || n < 1) {
+    cudaGetLastError();
+    n = 1;
+  }
+  cache[key] = n;
+  return n;
+}
+
+namespace {
+
+int grid_size(const void* fn, int64_t blocks_needed) {
+  const int64_t cap = (int64_t)sm_count() * blocks_per_sm(fn, kThreads, 0);
+  int64_t g = blocks_needed < cap ? blocks_needed : cap;
+  return g < 1 ? 1 : (int)g;
+}
+
+// Widest copy unit (16, 8, 4 or 2 bytes) that the row size and every base
+// address allow.
+int copy_width(const TableView& t, const void* out) {
+  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)(t.d * 2);
+  if (t.n_fgrams > 0) a |= (uintptr_t)t.F;
+  if ((a & 15) == 0) return 16;
+  if ((a & 7) == 0) return 8;
+  if ((a & 3) == 0) return 4;
+  return 2;
+}
+
+__device__ __forceinline__ int32_t pos_in_seq(int64_t p, int32_t L) { return (int32_t)(p % L); }
+
+template <int FMT, int KT>
+__global__ void __launch_bounds__(kThreads)
+    match_kernel(const TableView t, const int32_t* __restrict__ tok, int64_t n_tok, int32_t L,
+                 int32_t* __restrict__ row_out, uint8_t* __restrict__ len_out) {
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < n_tok;
+       p += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t x = __ldg(tok + p);
+    int len = 0, err = 0;
+    const int32_t r = match_position<FMT, KT>(t, tok, p, pos_in_seq(p, L), x, &len, &err);
+    if (err) record_error(t.status, err);
+    row_out[p] = r;
+    if (len_out) len_out[p] = (uint8_t)len;
+  }
+}
+
+template <int FMT, int KT, int W>
+__global__ void __launch_bounds__(kThreads)
+    embed_kernel(const TableView t, const int32_t* __restrict__ tok, int64_t n_tok, int32_t L,
+                 uint8_t* __restrict__ out, int32_t* __restrict__ row_out,
+                 uint8_t* __restrict__ len_out, int width) {
+  __shared__ const void* src_s[kWarps][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int row_bytes = t.d * 2;
+  const int64_t n_tiles = (n_tok + 31) >> 5;
+  for (int64_t tile = (int64_t)blockIdx.x * kWarps + warp; tile < n_tiles;
+       tile += (int64_t)gridDim.x * kWarps) {
+    const int64_t p = (tile << 5) + lane;
+    const void* src = nullptr;
+    if (p < n_tok) {
+      const int32_t x = __ldg(tok + p);
+      int len = 0, err = 0;
+      const int32_t r = match_position<FMT, KT>(t, tok, p, pos_in_seq(p, L), x, &len, &err);
+      if (err) {
+        record_error(t.status, err);
+      } else {
+        src = r >= 0 ? static_cast<const void*>(t.F + (int64_t)r * t.d)
+                     : static_cast<const void*>(t.T + (int64_t)x * t.d);
+      }
+      if (row_out) row_out[p] = r;
+      if (len_out) len_out[p] = (uint8_t)len;
+    }
+    src_s[warp][lane] = src;
+    __syncwarp();
+    const int nrows = (int)(n_tok - (tile << 5) < 32 ? n_tok - (tile << 5) : 32);
+    warp_copy_rows_w<W>(src_s[warp], out + (tile << 5) * (int64_t)row_bytes, nrows, row_bytes,
+                        width, lane);
+    __syncwarp();
+  }
+}
+
+template <int W>
+__global__ void __launch_bounds__(kThreads)
+    gather_kernel(const TableView t, const int32_t* __restrict__ tok,
+                  const int32_t* __restrict__ row, int64_t n_tok, uint8_t* __restrict__ out,
+                  int width) {
+  __shared__ const void* src_s[kWarps][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int row_bytes = t.d * 2;
+  const int64_t n_tiles = (n_tok + 31) >> 5;
+  for (int64_t tile = (int64_t)blockIdx.x * kWarps + warp; tile < n_tiles;
+       tile += (int64_t)gridDim.x * kWarps) {
+    const int64_t p = (tile << 5) + lane;
+    const void* src = nullptr;
+    if (p < n_tok) {
+      const int32_t r = __ldg(row + p);
+      if (r >= 0) {
+        if (r < t.n_fgrams) src = t.F + (int64_t)r * t.d;
+        else record_error(t.status, SCONE_ERR_INVALID_ARG);
+      } else {
+        const int32_t x = __ldg(tok + p);
+        if (valid_token(x, t.vocab)) src = t.T + (int64_t)x * t.d;
+        else record_error(t.status, SCONE_ERR_TOKEN_RANGE);
+      }
+    }
+    src_s[warp][lane] = src;
+    __syncwarp();
+    const int nrows = (int)(n_tok - (tile << 5) < 32 ? n_tok - (tile << 5) : 32);
+    warp_copy_rows_w<W>(src_s[warp], out + (tile << 5) * (int64_t)row_bytes, nrows, row_bytes,
+                        width, lane);
+    __syncwarp();
+  }
+}
+
+using MatchFn = void (*)(TableView, const int32_t*, int64_t, int32_t, int32_t*, uint8_t*);
+using EmbedFn = void (*)(TableView, const int32_t*, int64_t, int32_t, uint8_t*, int32_t*,
+                         uint8_t*, int);
+
+// K <= 3 -> unrolled for 3, K <= 5 -> 5, else 8. The 32-byte key format only
+// arises for K*b > 92, so it is instantiated for the two larger unrolls.
+MatchFn pick_match(int fmt, int K) {
+  if (fmt == FMT16) {
+    if (K <= 3) return match_kernel<FMT16, 3>;
+    if (K <= 5) return match_kernel<FMT16, 5>;
+    return match_kernel<FMT16, 8>;
+  }
+  if (K <= 5) return match_kernel<FMT32, 5>;
+  return match_kernel<FMT32, 8>;
+}
+
+template <int W>
+EmbedFn pick_embed_w(int fmt, int K) {
+  if (fmt == FMT16) {
+    if (K <= 3) return embed_kernel<FMT16, 3, W>;
+    if (K <= 5) return embed_kernel<FMT16, 5, W>;
+    return embed_kernel<FMT16, 8, W>;
+  }
+  if (K <= 5) return embed_kernel<FMT32, 5, W>;
+  return embed_kernel<FMT32, 8, W>;
+}
+
+EmbedFn pick_embed(int fmt, int K, int width) {
+  return width == 16 ? pick_embed_w<16>(fmt, K) : pick_embed_w<0>(fmt, K);
+}
+
+bool misaligned(const void* p, uintptr_t a) { return ((uintptr_t)p & (a - 1)) != 0; }
+
+}  // namespace
+
+}  // namespace scone
+
+using namespace scone;
+
+extern "C" int scone_match(const scone_table* tb, const int32_t* tok, int32_t B, int32_t L,
+                           int32_t* row, uint8_t* len, void* stream) {
+  if (!tb || B < 0 || L < 0) return SCONE_ERR_INVALID_ARG;
+  const int64_t n = (int64_t)B * L;
+  if (n == 0) return SCONE_OK;
+  if (!tok || !row || misaligned(tok, 4) || misaligned(row, 4)) return SCONE_ERR_INVALID_ARG;
+  DeviceGuard g(tb->device);
+  const MatchFn fn = pick_match(tb->fmt, tb->view.K);
+  const int grid = grid_size((const void*)fn, (n + kThreads - 1) / kThreads);
+  fn<<<grid, kThreads, 0, (cudaStream_t)stream>>>(tb->view, tok, n, L, row, len);
+  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}
+
+extern "C" int scone_embed_gather(const scone_table* tb, const int32_t* tok, const int32_t* row,
+                                  int64_t n_tok, scone_bf16* out, void* stream) {
+  if (!tb || n_tok < 0) return SCONE_ERR_INVALID_ARG;
+  if (n_tok == 0) return SCONE_OK;
+  if (!tok || !row || !out || misaligned(tok, 4) || misaligned(row, 4) || misaligned(out, 2))
+    return SCONE_ERR_INVALID_ARG;
+  DeviceGuard g(tb->device);
+  const int width = copy_width(tb->view, out);
+  const auto fn = width == 16 ? gather_kernel<16> : gather_kernel<0>;
+  const int grid = grid_size((const void*)fn, ((n_tok + 31) / 32 + kWarps - 1) / kWarps);
+  fn<<<grid, kThreads, 0, (cudaStream_t)stream>>>(tb->view, tok, row, n_tok,
+                                                  reinterpret_cast<uint8_t*>(out), width);
+  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}
+
+extern "C" int scone_embed(const scone_table* tb, const int32_t* tok, int32_t B, int32_t L,
+                           scone_bf16* out, int32_t* row, uint8_t* len, void* stream) {
+  if (!tb || B < 0 || L < 0) return SCONE_ERR_INVALID_ARG;
+  const int64_t n = (int64_t)B * L;
+  if (n == 0) return SCONE_OK;
+  if (!tok || !out || misaligned(tok, 4) || misaligned(out, 2) || (row && misaligned(row, 4)))
+    return SCONE_ERR_INVALID_ARG;
+  DeviceGuard g(tb->device);
+  const int width = copy_width(tb->view, out);
+  const EmbedFn fn = pick_embed(tb->fmt, tb->view.K, width);
+  const int grid = grid_size((const void*)fn, ((n + 31) / 32 + kWarps - 1) / kWarps);
+  fn<<<grid, kThreads, 0, (cudaStream_t)stream>>>(tb->view, tok, n, L,
+                                                  reinterpret_cast<uint8_t*>(out), row, len,
+                                                  width);
+  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}

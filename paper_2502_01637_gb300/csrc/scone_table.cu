@@ -1,0 +1,367 @@
+// f-gram table build, lifetime and status (C ABI).
+//
+// Build (Sec. 2: "a hash dictionary that maps f-grams to matrix indices"):
+//   1. the slot array is set to all ones (every row word = empty);
+//   2. one thread per f-gram claims a slot with a 32-bit atomicCAS on the row
+//      word, walking the linear-probe sequence from its home bucket. When a
+//      CAS finds another row there, the thread compares the two f-grams in
+//      the device copy of the input list: equal means a duplicate, otherwise
+//      it moves on. The list is immutable during the build, so no thread
+//      ever waits on another;
+//   3. one thread per slot writes the packed key of the row it holds.
+// Slots are claimed in probe order and never released, so every key sits
+// after an unbroken run of occupied slots from its home bucket: the
+// invariant linear-probe lookups rely on.
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "scone_device.cuh"
+#include "scone_host.h"
+
+namespace scone {
+
+namespace {
+
+struct BuildFlags {
+  int duplicate;
+  int full;
+  int max_probe;
+};
+
+template <int FMT>
+__device__ __forceinline__ KeyBits<Fmt<FMT>::kWords> key_of_listed(const int32_t* ftok,
+                                                                    const uint8_t* flen,
+                                                                    int64_t r, int K, int bits) {
+  constexpr int NW = Fmt<FMT>::kWords;
+  KeyBits<NW> k;
+#pragma unroll
+  for (int q = 0; q < NW; ++q) k.w[q] = 0;
+  const int n = flen[r];
+  const int32_t* g = ftok + r * K;
+  k.w[0] = (uint32_t)g[n - 1];
+  for (int j = 1; j < n; ++j) put_field<NW>(k, j * bits, (uint32_t)g[n - 1 - j], bits);
+  put_len<FMT>(k, n);
+  return k;
+}
+
+__device__ __forceinline__ bool same_fgram(const int32_t* ftok, const uint8_t* flen, int64_t a,
+                                           int64_t b, int K) {
+  if (flen[a] != flen[b]) return false;
+  for (int j = 0; j < flen[a]; ++j)
+    if (ftok[a * K + j] != ftok[b * K + j]) return false;
+  return true;
+}
+
+template <int FMT>
+__global__ void insert_kernel(uint8_t* slots, uint64_t n_buckets, const int32_t* ftok,
+                              const uint8_t* flen, int64_t n, int K, int bits, BuildFlags* flags) {
+  constexpr int SPB = Fmt<FMT>::kSlotsPerBucket;
+  constexpr int SLOT = kBucketBytes / SPB;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n;
+       r += (int64_t)gridDim.x * blockDim.x) {
+    const auto k = key_of_listed<FMT>(ftok, flen, r, K, bits);
+    uint64_t q = fastrange(key_hash<FMT>(k), n_buckets);
+    bool done = false;
+    for (uint64_t probe = 0; probe < n_buckets && !done; ++probe) {
+#pragma unroll
+      for (int s = 0; s < SPB && !done; ++s) {
+        // the row word is the upper half of the slot's last 8 bytes
+        unsigned int* rowp =
+            reinterpret_cast<unsigned int*>(slots + q * kBucketBytes + s * SLOT + SLOT - 4);
+        const unsigned int old = atomicCAS(rowp, kEmptyRow, (unsigned int)r);
+        if (old == kEmptyRow) {
+          atomicMax(&flags->max_probe, (int)(probe + 1 < 0x7FFFFFFF ? probe + 1 : 0x7FFFFFFF));
+          done = true;
+        } else if (same_fgram(ftok, flen, (int64_t)old, r, K)) {
+          atomicExch(&flags->duplicate, 1);
+          done = true;
+        }
+      }
+      q = (q + 1 == n_buckets) ? 0 : q + 1;
+    }
+    if (!done) atomicExch(&flags->full, 1);
+  }
+}
+
+template <int FMT>
+__global__ void fill_keys_kernel(uint8_t* slots, uint64_t n_slots, const int32_t* ftok,
+                                 const uint8_t* flen, int K, int bits) {
+  constexpr int SLOT = kBucketBytes / Fmt<FMT>::kSlotsPerBucket;
+  constexpr int NW = Fmt<FMT>::kWords;
+  for (uint64_t s = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; s < n_slots;
+       s += (uint64_t)gridDim.x * blockDim.x) {
+    uint64_t* w = reinterpret_cast<uint64_t*>(slots + s * SLOT);
+    const uint32_t row = (uint32_t)(w[NW - 1] >> 32);
+    if (row == kEmptyRow) continue;
+    const auto k = key_of_listed<FMT>(ftok, flen, (int64_t)row, K, bits);
+#pragma unroll
+    for (int q = 0; q < NW - 1; ++q) w[q] = k.w[q];
+    w[NW - 1] = (uint64_t)(uint32_t)k.w[NW - 1] | ((uint64_t)row << 32);
+  }
+}
+
+int grid_for(int64_t n, int threads) {
+  int dev = 0, sms = 1;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t g = (n + threads - 1) / threads;
+  const int64_t cap = (int64_t)sms * 32;
+  if (g > cap) g = cap;
+  return g < 1 ? 1 : (int)g;
+}
+
+int bits_for_vocab(int32_t vocab) {
+  int b = 0;
+  while (b < 31 && ((int64_t)1 << b) < (int64_t)vocab) ++b;
+  return b < 1 ? 1 : b;
+}
+
+bool is_device_accessible(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+}  // namespace
+
+}  // namespace scone
+
+using namespace scone;
+
+extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_len,
+                                 int64_t n_fgrams, int32_t K, int32_t vocab, int32_t d,
+                                 const scone_bf16* F, int32_t F_location, const scone_bf16* T,
+                                 float load_factor, void* stream, scone_table** out) {
+  if (!out) return SCONE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (n_fgrams < 0 || n_fgrams > 0x7FFFFFFELL || K < 2 || K > 8 || vocab < 1 || d < 1 || !T)
+    return SCONE_ERR_INVALID_ARG;
+  if (n_fgrams > 0 && (!fgram_tok || !fgram_len || !F)) return SCONE_ERR_INVALID_ARG;
+  if (F_location != SCONE_ROWS_DEVICE && F_location != SCONE_ROWS_HOST_MAPPED)
+    return SCONE_ERR_INVALID_ARG;
+  if (load_factor == 0.0f) load_factor = 0.5f;
+  if (!(load_factor > 0.0f && load_factor <= 0.95f)) return SCONE_ERR_INVALID_ARG;
+  const int bits = bits_for_vocab(vocab);
+  const int key_bits = K * bits + 4;
+  int fmt;
+  if (K * bits <= 92) {
+    fmt = FMT16;
+  } else if (K * bits <= 220) {
+    fmt = FMT32;
+  } else {
+    return SCONE_ERR_UNSUPPORTED;
+  }
+  // host validation of the list: lengths in [2, K], tokens in [0, vocab)
+  for (int64_t r = 0; r < n_fgrams; ++r) {
+    const int n = fgram_len[r];
+    if (n < 2 || n > K) return SCONE_ERR_INVALID_ARG;
+    for (int j = 0; j < n; ++j)
+      if (fgram_tok[r * K + j] < 0 || fgram_tok[r * K + j] >= vocab) return SCONE_ERR_INVALID_ARG;
+  }
+  if (!is_device_accessible(T)) return SCONE_ERR_INVALID_ARG;
+  const uint16_t* F_dev = reinterpret_cast<const uint16_t*>(F);
+  if (n_fgrams > 0) {
+    if (F_location == SCONE_ROWS_DEVICE) {
+      if (!is_device_accessible(F)) return SCONE_ERR_INVALID_ARG;
+    } else {
+      void* dp = nullptr;
+      if (cudaHostGetDevicePointer(&dp, const_cast<scone_bf16*>(F), 0) != cudaSuccess || !dp) {
+        cudaGetLastError();
+        return SCONE_ERR_INVALID_ARG;
+      }
+      F_dev = reinterpret_cast<const uint16_t*>(dp);
+    }
+  }
+
+  const int spb = fmt == FMT16 ? 2 : 1;
+  int64_t n_slots = (int64_t)std::ceil((double)n_fgrams / (double)load_factor);
+  if (n_slots < n_fgrams + 1) n_slots = n_fgrams + 1;
+  if (n_slots < 2) n_slots = 2;
+  const int64_t n_buckets = (n_slots + spb - 1) / spb;
+  n_slots = n_buckets * spb;
+
+  scone_table* t = new (std::nothrow) scone_table();
+  if (!t) return SCONE_ERR_NOMEM;
+  cudaGetDevice(&t->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  if (cudaMalloc(&t->slots, (size_t)n_buckets * kBucketBytes) != cudaSuccess ||
+      cudaMalloc(&t->status, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    scone_table_destroy(t);
+    return SCONE_ERR_NOMEM;
+  }
+  int rc = SCONE_OK;
+  int32_t* d_tok = nullptr;
+  uint8_t* d_len = nullptr;
+  BuildFlags* d_flags = nullptr;
+  BuildFlags flags = {0, 0, 0};
+  do {
+    if (cudaMemsetAsync(t->slots, 0xFF, (size_t)n_buckets * kBucketBytes, s) != cudaSuccess ||
+        cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess) {
+      rc = SCONE_ERR_CUDA;
+      break;
+    }
+    if (n_fgrams > 0) {
+      if (cudaMalloc(&d_tok, (size_t)n_fgrams * K * sizeof(int32_t)) != cudaSuccess ||
+          cudaMalloc(&d_len, (size_t)n_fgrams) != cudaSuccess ||
+          cudaMalloc(&d_flags, sizeof(BuildFlags)) != cudaSuccess) {
+        rc = SCONE_ERR_NOMEM;
+        break;
+      }
+      if (cudaMemcpyAsync(d_tok, fgram_tok, (size_t)n_fgrams * K * sizeof(int32_t),
+                          cudaMemcpyHostToDevice, s) != cudaSuccess ||
+          cudaMemcpyAsync(d_len, fgram_len, (size_t)n_fgrams, cudaMemcpyHostToDevice, s) !=
+              cudaSuccess ||
+          cudaMemsetAsync(d_flags, 0, sizeof(BuildFlags), s) != cudaSuccess) {
+        rc = SCONE_ERR_CUDA;
+        break;
+      }
+      const int th = 256;
+      if (fmt == FMT16) {
+        insert_kernel<FMT16><<<grid_for(n_fgrams, th), th, 0, s>>>(
+            t->slots, (uint64_t)n_buckets, d_tok, d_len, n_fgrams, K, bits, d_flags);
+        fill_keys_kernel<FMT16><<<grid_for(n_slots, th), th, 0, s>>>(
+            t->slots, (uint64_t)n_slots, d_tok, d_len, K, bits);
+      } else {
+        insert_kernel<FMT32><<<grid_for(n_fgrams, th), th, 0, s>>>(
+            t->slots, (uint64_t)n_buckets, d_tok, d_len, n_fgrams, K, bits, d_flags);
+        fill_keys_kernel<FMT32><<<grid_for(n_slots, th), th, 0, s>>>(
+            t->slots, (uint64_t)n_slots, d_tok, d_len, K, bits);
+      }
+      if (cudaGetLastError() != cudaSuccess ||
+          cudaMemcpyAsync(&flags, d_flags, sizeof(BuildFlags), cudaMemcpyDeviceToHost, s) !=
+              cudaSuccess) {
+        rc = SCONE_ERR_CUDA;
+        break;
+      }
+    }
+    if (cudaStreamSynchronize(s) != cudaSuccess) {
+      rc = SCONE_ERR_CUDA;
+      break;
+    }
+    if (flags.duplicate) rc = SCONE_ERR_DUPLICATE_FGRAM;
+    else if (flags.full) rc = SCONE_ERR_TABLE_FULL;
+  } while (0);
+  if (d_tok) cudaFree(d_tok);
+  if (d_len) cudaFree(d_len);
+  if (d_flags) cudaFree(d_flags);
+  if (rc != SCONE_OK) {
+    cudaGetLastError();
+    scone_table_destroy(t);
+    return rc;
+  }
+
+  t->fmt = fmt;
+  TableView& v = t->view;
+  v.slots = t->slots;
+  v.n_buckets = (uint64_t)n_buckets;
+  v.probe_limit = n_buckets;
+  v.n_fgrams = n_fgrams;
+  v.F = F_dev;
+  v.T = reinterpret_cast<const uint16_t*>(T);
+  v.status = t->status;
+  v.K = K;
+  v.bits = bits;
+  v.vocab = vocab;
+  v.d = d;
+  scone_table_info& in = t->info;
+  in.n_fgrams = n_fgrams;
+  in.n_slots = n_slots;
+  in.n_buckets = n_buckets;
+  in.slot_bytes = kBucketBytes / spb;
+  in.key_bits = key_bits;
+  in.bits_per_token = bits;
+  in.K = K;
+  in.vocab = vocab;
+  in.d = d;
+  in.F_location = F_location;
+  in.max_insert_probe = flags.max_probe;
+  in.table_bytes = n_buckets * kBucketBytes;
+  in.F_bytes = n_fgrams * (int64_t)d * 2;
+  in.T_bytes = (int64_t)vocab * d * 2;
+  *out = t;
+  return SCONE_OK;
+}
+
+extern "C" int scone_table_destroy(scone_table* t) {
+  if (!t) return SCONE_OK;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (prev != t->device) cudaSetDevice(t->device);
+  if (t->slots || t->status) cudaDeviceSynchronize();
+  if (t->slots) cudaFree(t->slots);
+  if (t->status) cudaFree(t->status);
+  if (prev >= 0 && prev != t->device) cudaSetDevice(prev);
+  delete t;
+  return SCONE_OK;
+}
+
+extern "C" int scone_table_get_info(const scone_table* t, scone_table_info* info) {
+  if (!t || !info) return SCONE_ERR_INVALID_ARG;
+  *info = t->info;
+  return SCONE_OK;
+}
+
+extern "C" int scone_table_set_probe_limit(scone_table* t, int64_t max_buckets) {
+  if (!t || max_buckets < 1) return SCONE_ERR_INVALID_ARG;
+  t->view.probe_limit =
+      max_buckets > (int64_t)t->view.n_buckets ? (int64_t)t->view.n_buckets : max_buckets;
+  return SCONE_OK;
+}
+
+extern "C" int scone_status(const scone_table* t, void* stream) {
+  if (!t) return SCONE_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  int code = 0;
+  if (cudaMemcpyAsync(&code, t->status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return SCONE_ERR_CUDA;
+  }
+  return code;
+}
+
+extern "C" int scone_host_alloc(int64_t bytes, void** out) {
+  if (!out) return SCONE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (bytes < 1) return SCONE_ERR_INVALID_ARG;
+  void* p = nullptr;
+  if (cudaHostAlloc(&p, (size_t)bytes, cudaHostAllocMapped | cudaHostAllocPortable) !=
+          cudaSuccess ||
+      !p) {
+    cudaGetLastError();
+    return SCONE_ERR_NOMEM;
+  }
+  *out = p;
+  return SCONE_OK;
+}
+
+extern "C" int scone_host_free(void* p) {
+  if (!p) return SCONE_OK;
+  cudaDeviceSynchronize();
+  return cudaFreeHost(p) == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}
+
+extern "C" const char* scone_strerror(int code) {
+  switch (code) {
+    case SCONE_OK: return "ok";
+    case SCONE_ERR_INVALID_ARG: return "invalid argument";
+    case SCONE_ERR_TOKEN_RANGE: return "token id outside [0, vocab)";
+    case SCONE_ERR_DUPLICATE_FGRAM: return "duplicate f-gram in the list";
+    case SCONE_ERR_TABLE_FULL: return "hash table full";
+    case SCONE_ERR_PROBE_LIMIT: return "lookup exceeded the probe limit";
+    case SCONE_ERR_UNSUPPORTED: return "key does not fit (K * ceil(log2 vocab) > 220)";
+    case SCONE_ERR_CUDA: return "CUDA runtime error";
+    case SCONE_ERR_NOMEM: return "out of memory";
+    default: return "unknown error";
+  }
+}
+
+extern "C" int scone_version(void) { return (1 << 16) | 0; }

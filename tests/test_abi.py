@@ -1,0 +1,106 @@
+"""The C ABI library loads and exports what include/scone.h declares (CPU).
+
+Also checks the host-side argument validation, which returns before any
+CUDA call, so it runs without a GPU.
+"""
+
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+
+import paper_2502_01637_gb300 as scone
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "scone.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(scone_[a-z_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported():
+    lib = scone.load_library()
+    names = declared_functions()
+    assert len(names) >= 14
+    for n in names:
+        assert hasattr(lib, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", scone.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (scone_[a-z_]+)", out))
+    assert set(names) <= exported, set(names) - exported
+    assert set(scone.EXPORTS) == set(names)
+
+
+def test_strerror_and_version():
+    assert scone.scone_strerror(0) == "ok"
+    assert "duplicate" in scone.scone_strerror(scone.SCONE_ERR_DUPLICATE_FGRAM)
+    assert scone.scone_strerror(-99) == "unknown error"
+    assert scone.scone_version() >> 16 == 1
+
+
+def _build_rc(fgram_tok, fgram_len, K, vocab, d=8, T=0x1000, F=0x2000, lf=0.0, loc=0):
+    lib = scone.load_library()
+    ft = np.ascontiguousarray(fgram_tok, dtype=np.int32).reshape(-1)
+    fl = np.ascontiguousarray(fgram_len, dtype=np.uint8).reshape(-1)
+    h = ctypes.c_void_p()
+    return lib.scone_table_build(ft.ctypes.data if fl.size else None,
+                                 fl.ctypes.data if fl.size else None, fl.size, K, vocab, d, F, loc,
+                                 T, lf, None, ctypes.byref(h))
+
+
+def test_host_validation_returns_before_device_work():
+    ok_tok = np.array([[1, 2, -1]], np.int32)
+    ok_len = np.array([2], np.uint8)
+    inv = scone.SCONE_ERR_INVALID_ARG
+    assert _build_rc(ok_tok, ok_len, 1, 10) == inv          # K < 2
+    assert _build_rc(ok_tok, ok_len, 9, 10) == inv          # K > 8
+    assert _build_rc(ok_tok, ok_len, 3, 0) == inv           # empty vocab
+    assert _build_rc(ok_tok, ok_len, 3, 10, d=0) == inv     # d < 1
+    assert _build_rc(ok_tok, ok_len, 3, 10, T=0) == inv     # no T
+    assert _build_rc(ok_tok, ok_len, 3, 10, F=0) == inv     # no F with f-grams
+    assert _build_rc(ok_tok, ok_len, 3, 10, lf=0.99) == inv  # load factor too high
+    assert _build_rc(ok_tok, ok_len, 3, 10, lf=-1.0) == inv
+    assert _build_rc(ok_tok, ok_len, 3, 10, loc=7) == inv   # unknown F location
+    assert _build_rc(ok_tok, np.array([1], np.uint8), 3, 10) == inv   # 1-gram
+    assert _build_rc(ok_tok, np.array([4], np.uint8), 3, 10) == inv   # longer than K
+    assert _build_rc(np.array([[1, 10, -1]], np.int32), ok_len, 3, 10) == inv  # token range
+    assert _build_rc(np.array([[-1, 2, -1]], np.int32), ok_len, 3, 10) == inv
+    # key does not fit: K=8 tokens of 30 bits
+    assert _build_rc(np.zeros((1, 8), np.int32), ok_len, 8, 1 << 30) == scone.SCONE_ERR_UNSUPPORTED
+    lib = scone.load_library()
+    assert lib.scone_table_build(None, None, 0, 3, 10, 8, None, 0, 0x1000, 0.0, None,
+                                 None) == inv               # no out pointer
+
+
+def test_null_handles_rejected():
+    lib = scone.load_library()
+    inv = scone.SCONE_ERR_INVALID_ARG
+    assert lib.scone_match(None, None, 1, 1, None, None, None) == inv
+    assert lib.scone_embed(None, None, 1, 1, None, None, None, None) == inv
+    assert lib.scone_embed_gather(None, None, None, 1, None, None) == inv
+    assert lib.scone_decode_step(None, None, None, None, None, None) == inv
+    assert lib.scone_decode_create(None, 1, None, None, None) == inv
+    assert lib.scone_status(None, None) == inv
+    assert lib.scone_table_destroy(None) == 0
+    assert lib.scone_decode_destroy(None) == 0
+    assert lib.scone_table_get_info(None, None) == inv
+    assert lib.scone_table_set_probe_limit(None, 1) == inv
+
+
+def test_key_format_boundaries():
+    """FMT16 up to K*b = 92, FMT32 up to 220 (K*b + 4 length bits)."""
+    # bits per token = ceil(log2 vocab): vocab 2^18 -> 18 bits; K=5 -> 90 <= 92 fits the
+    # 16-byte slot; vocab 2^18+1 -> 19 bits -> 95 > 92 needs the 32-byte slot; both are
+    # accepted by the host checks (they fail later only because T is not device memory).
+    for vocab in (1 << 18, (1 << 18) + 1):
+        rc = _build_rc(np.zeros((1, 5), np.int32), np.array([2], np.uint8), 5, vocab)
+        assert rc == scone.SCONE_ERR_INVALID_ARG     # T=0x1000 is not device memory
+    rc = _build_rc(np.zeros((1, 8), np.int32), np.array([2], np.uint8), 8, 1 << 27)
+    assert rc == scone.SCONE_ERR_INVALID_ARG         # 8*27 = 216 <= 220: format fits
+    rc = _build_rc(np.zeros((1, 8), np.int32), np.array([2], np.uint8), 8, (1 << 27) + 1)
+    assert rc == scone.SCONE_ERR_UNSUPPORTED         # 8*28 = 224 > 220

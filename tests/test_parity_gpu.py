@@ -1,0 +1,285 @@
+"""CUDA path vs the oracle, element by element, on seeded inputs (GPU).
+
+Bit-exact throughout: row ids and lengths are integers and the outputs are
+copies of stored bf16 rows, so the tolerance is zero.
+"""
+
+import itertools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+import paper_2502_01637_gb300 as scone
+from gpu_cases import DEV, SmallCase, dev_rows, run_embed
+
+pytestmark = pytest.mark.gpu
+
+TINY = synth.WORKLOADS["tiny"]
+
+
+def assert_parity(case: SmallCase, out, row, ln):
+    o_out, o_row, o_len, _ = case.expected()
+    n = case.tok.size
+    assert np.array_equal(ln, o_len.reshape(n)), "match lengths differ"
+    assert np.array_equal(row, o_row.reshape(n).astype(np.int32)), "row ids differ"
+    assert np.array_equal(out, o_out.reshape(n, -1)), "output bytes differ"
+
+
+@pytest.mark.parametrize("mode", ["fused", "match+gather", "fused_noaux"])
+def test_tiny_full(mode):
+    case = SmallCase(TINY)
+    table = case.build()
+    out, row, ln = run_embed(table, case.tok, TINY.d, mode)
+    assert_parity(case, out, row, ln)
+    assert scone.scone_status(table) == 0
+    info = table.info()
+    assert info["n_fgrams"] == TINY.n_fgrams and info["slot_bytes"] == 16
+    assert info["n_slots"] >= 2 * TINY.n_fgrams
+    # every length occurs, so every branch of the selection ran
+    assert set(np.unique(ln)) == {1, 2, 3}
+
+
+@pytest.mark.parametrize("B,L", [(3, 77), (1, 1), (1, 31), (2, 33), (5, 2), (7, 129)])
+def test_ragged_shapes(B, L):
+    w = TINY.scaled("tiny_ragged", B=B, L=L, quotas=((2, 20000), (3, 15000)))
+    case = SmallCase(w)
+    table = case.build()
+    for mode in ("fused", "match+gather"):
+        out, row, ln = run_embed(table, case.tok, w.d, mode)
+        assert_parity(case, out, row, ln)
+
+
+def test_empty_batches():
+    case = SmallCase(TINY.scaled("tiny_empty", B=1, L=8, quotas=((2, 100), (3, 50))))
+    table = case.build()
+    for B, L in ((0, 5), (3, 0), (0, 0)):
+        t = torch.empty((B, L), dtype=torch.int32, device=DEV)
+        out = torch.empty((0, TINY.d), dtype=torch.int16, device=DEV)
+        scone.scone_embed(table, t, out)
+        scone.scone_match(table, t, torch.empty(0, dtype=torch.int32, device=DEV))
+    assert scone.scone_status(table) == 0
+
+
+@pytest.mark.parametrize("name,K,vocab,d,quotas,inject", [
+    ("k2", 2, 32000, 256, ((2, 8000),), 0.0),
+    ("k4_d512", 4, 50000, 512, ((2, 6000), (3, 6000), (4, 6000)), 0.02),
+    ("k5_stress", 5, 100000, 1536, ((2, 20000), (3, 20000), (4, 10000), (5, 10000)), 0.05 / 6),
+    ("k5_fmt32", 5, 300000, 128, ((2, 5000), (3, 5000), (4, 5000), (5, 5000)), 0.05),
+    ("k8_fmt32", 8, 1 << 20, 64, tuple((n, 2000) for n in range(2, 9)), 0.05),
+    ("k7_fmt16", 7, 8192, 64, tuple((n, 2000) for n in range(2, 8)), 0.05),
+    ("k3_d1024", 3, 100000, 1024, ((2, 6000), (3, 4000)), 0.0),
+    ("k3_d4096", 3, 100000, 4096, ((2, 600), (3, 400)), 0.0),
+])
+def test_key_formats_and_widths(name, K, vocab, d, quotas, inject):
+    w = synth.Workload(name, 40 + K, vocab, 1.05, 3, 700, quotas, K, d, inject_p=inject,
+                       n_phrases=512 if inject else 0, phrase_len=(K, K + 2))
+    case = SmallCase(w)
+    table = case.build()
+    info = table.info()
+    bits = int(np.ceil(np.log2(vocab)))
+    assert info["bits_per_token"] == bits
+    assert info["slot_bytes"] == (16 if K * bits <= 92 else 32)
+    out, row, ln = run_embed(table, case.tok, d)
+    assert_parity(case, out, row, ln)
+    assert (ln >= 2).any()
+    if K in (2, 4, 5):
+        assert (ln == K).any(), "longest length never matched"
+
+
+@pytest.mark.parametrize("d,offset", [(100, 0), (6, 0), (3, 0), (256, 1), (8, 2)])
+def test_generic_copy_widths(d, offset):
+    """Rows or outputs not 16-byte aligned take the 8, 4 or 2 byte copy."""
+    w = TINY.scaled(f"tiny_d{d}", B=2, L=150, d=d, quotas=((2, 4000), (3, 3000)))
+    case = SmallCase(w)
+    table = case.build()
+    for mode in ("fused", "match+gather"):
+        out, row, ln = run_embed(table, case.tok, d, mode, out_offset=offset)
+        assert_parity(case, out, row, ln)
+
+
+@pytest.mark.parametrize("lf", [0.25, 0.5, 0.8, 0.95])
+def test_load_factors(lf):
+    w = TINY.scaled("tiny_lf", B=2, L=512)
+    case = SmallCase(w)
+    table = case.build(load_factor=lf)
+    info = table.info()
+    assert info["n_slots"] >= int(np.ceil(w.n_fgrams / lf))
+    out, row, ln = run_embed(table, case.tok, w.d)
+    assert_parity(case, out, row, ln)
+
+
+def test_permuted_list_same_output():
+    w = TINY.scaled("tiny_perm", B=2, L=300, quotas=((2, 5000), (3, 5000)))
+    case = SmallCase(w)
+    out, row, ln = run_embed(case.build(), case.tok, w.d)
+    perm = np.random.default_rng(9).permutation(w.n_fgrams)
+    case2 = SmallCase(w, fgrams=(case.fg_tok[perm], case.fg_len[perm]), tok=case.tok)
+    case2.F = case.F[perm]
+    out2, row2, ln2 = run_embed(case2.build(), case.tok, w.d)
+    assert np.array_equal(out, out2) and np.array_equal(ln, ln2)
+    assert np.array_equal(np.where(row2 >= 0, perm[np.maximum(row2, 0)], -1), row)
+
+
+def test_empty_fgram_set_is_token_embedding():
+    rng = np.random.default_rng(2)
+    V, d = 1000, 64
+    tok = rng.integers(0, V, size=(4, 100)).astype(np.int32)
+    T = rng.integers(0, 2**16, size=(V, d), dtype=np.uint16)
+    Td = dev_rows(T)
+    table = scone.scone_table_build(np.zeros((0, 3), np.int32), np.zeros(0, np.uint8), 3, V, d,
+                                    None, Td)
+    out, row, ln = run_embed(table, tok, d)
+    ref = torch.nn.functional.embedding(torch.from_numpy(tok.astype(np.int64)).to(DEV), Td)
+    assert np.array_equal(out, ref.cpu().numpy().view(np.uint16).reshape(-1, d))
+    assert (row == -1).all() and (ln == 1).all()
+
+
+def test_invalid_tokens_zero_rows_and_status():
+    w = TINY.scaled("tiny_bad", B=2, L=64, quotas=((2, 3000), (3, 2000)))
+    tok = synth.query_tokens(w)
+    tok[0, 5] = -1
+    tok[0, 17] = w.vocab
+    tok[1, 0] = 2**31 - 1
+    tok[1, 40] = -7
+    case = SmallCase(w, tok=tok)
+    table = case.build()
+    for mode in ("fused", "match+gather"):
+        out, row, ln = run_embed(table, case.tok, w.d, mode)
+        o_out, o_row, o_len, rc = case.expected()
+        assert rc == oracle.ERR_TOKEN_RANGE
+        assert_parity(case, out, row, ln)
+        assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+        assert scone.scone_status(table) == 0       # read clears it
+
+
+def test_duplicate_fgrams_rejected():
+    ft = np.array([[1, 2, -1], [3, 4, 5], [1, 2, 9]], np.int32)
+    fl = np.array([2, 3, 2], np.uint8)
+    T = dev_rows(np.zeros((10, 8), np.uint16))
+    F = dev_rows(np.zeros((3, 8), np.uint16))
+    with pytest.raises(scone.SconeError) as e:
+        scone.scone_table_build(ft, fl, 3, 10, 8, F, T)
+    assert e.value.code == scone.SCONE_ERR_DUPLICATE_FGRAM
+    # the padding after the length is ignored: this list has no duplicate
+    fl2 = np.array([2, 3, 3], np.uint8)
+    ft2 = np.array([[1, 2, 7], [3, 4, 5], [1, 2, 9]], np.int32)
+    scone.scone_table_build(ft2, fl2, 3, 10, 8, F, T).close()
+
+
+def test_probe_limit_reports_and_never_hangs():
+    """A cap of one bucket at load 0.95: long probe runs become error
+    positions (zero row, len 0, sticky status); all others still match."""
+    w = TINY.scaled("tiny_probe", B=4, L=512)
+    case = SmallCase(w)
+    table = case.build(load_factor=0.95)
+    assert table.info()["max_insert_probe"] > 1
+    scone.scone_table_set_probe_limit(table, 1)
+    out, row, ln = run_embed(table, case.tok, w.d)
+    o_out, o_row, o_len, _ = case.expected()
+    err = ln == 0
+    assert err.any() and not err.all()
+    assert (row[err] == -1).all() and (out[err] == 0).all()
+    ok = ~err
+    assert np.array_equal(ln[ok], o_len.reshape(-1)[ok])
+    assert np.array_equal(out[ok], o_out.reshape(-1, w.d)[ok])
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_PROBE_LIMIT
+    scone.scone_table_set_probe_limit(table, 1 << 40)   # back to the whole table
+    out, row, ln = run_embed(table, case.tok, w.d)
+    assert_parity(case, out, row, ln)
+    assert scone.scone_status(table) == 0
+
+
+def test_host_mapped_F():
+    w = TINY.scaled("tiny_host", B=3, L=400)
+    case = SmallCase(w)
+    buf = scone.scone_host_alloc(case.F.nbytes)
+    buf.numpy()[:] = case.F.reshape(-1)
+    table = case.build(F_location=scone.SCONE_ROWS_HOST_MAPPED, F=buf.ptr)
+    assert table.info()["F_location"] == scone.SCONE_ROWS_HOST_MAPPED
+    for mode in ("fused", "match+gather"):
+        out, row, ln = run_embed(table, case.tok, w.d, mode)
+        assert_parity(case, out, row, ln)
+    table.close()
+    buf.free()
+
+
+# ------------------------------------------------------------------ decode
+def _decode_case(K, S, steps, vocab=2000, d=96, seed=0):
+    rng = np.random.default_rng(seed)
+    H = K - 1
+    full = (rng.zipf(1.3, size=(S, H + steps)) % vocab).astype(np.int32)
+    # f-grams: windows of the sequences themselves (so long matches occur) + random ones
+    fg = set()
+    for s in range(S):
+        for p in range(full.shape[1]):
+            n = int(rng.integers(2, K + 1))
+            if p + n <= full.shape[1] and rng.random() < 0.4:
+                fg.add(tuple(full[s, p:p + n].tolist()))
+    for _ in range(500):
+        n = int(rng.integers(2, K + 1))
+        fg.add(tuple(rng.integers(0, vocab, size=n).tolist()))
+    fg = sorted(fg)
+    ft = np.full((len(fg), K), -1, np.int32)
+    fl = np.array([len(g) for g in fg], np.uint8)
+    for r, g in enumerate(fg):
+        ft[r, :len(g)] = g
+    hl = rng.integers(0, H + 1, size=S).astype(np.int32)
+    hl[:3] = [0, H, min(1, H)]
+    hist = rng.integers(0, vocab, size=(S, H)).astype(np.int32)   # ignored entries: valid ids
+    for s in range(S):
+        if hl[s]:
+            hist[s, H - hl[s]:] = full[s, H - hl[s]:H]
+    new = np.ascontiguousarray(full[:, H:].T)
+    F = rng.integers(0, 2**16, size=(len(fg), d), dtype=np.uint16)
+    T = rng.integers(0, 2**16, size=(vocab, d), dtype=np.uint16)
+    return ft, fl, hist, hl, new, F, T
+
+
+@pytest.mark.parametrize("K,S,vocab", [(3, 100, 2000), (5, 70, 2000), (2, 33, 2000),
+                                       (8, 40, 2000), (6, 40, 1 << 20)])
+def test_decode_steps_match_oracle(K, S, vocab):
+    steps, d = 12, 96
+    ft, fl, hist, hl, new, F, T = _decode_case(K, S, steps, vocab, d, seed=K)
+    new[3, 5] = -4            # an invalid token mid-stream
+    new[7, 0] = vocab
+    o = oracle.Oracle(ft, fl, K, vocab)
+    o_out, o_row, o_len, rc = o.decode(hist, hl, new, F, T)
+    assert rc == oracle.ERR_TOKEN_RANGE
+    table = scone.scone_table_build(ft, fl, K, vocab, d, dev_rows(F), dev_rows(T))
+    st = scone.scone_decode_create(table, hist, hl)
+    new_d = torch.from_numpy(new).to(DEV)
+    out = torch.empty((S, d), dtype=torch.int16, device=DEV)
+    row = torch.empty(S, dtype=torch.int32, device=DEV)
+    ln = torch.empty(S, dtype=torch.uint8, device=DEV)
+    for k in range(steps):
+        scone.scone_decode_step(st, new_d[k], out, row, ln)
+        assert np.array_equal(ln.cpu().numpy(), o_len[k]), k
+        assert np.array_equal(row.cpu().numpy(), o_row[k].astype(np.int32)), k
+        assert np.array_equal(out.cpu().numpy().view(np.uint16), o_out[k]), k
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+    h2, hl2 = scone.scone_decode_get_history(st)
+    H = K - 1
+    assert (hl2 == np.minimum(hl + steps, H)).all()
+    if H:
+        assert np.array_equal(h2[:, H - min(H, steps):], new.T[:, steps - min(H, steps):])
+    assert set(np.unique(o_len)) >= {0, 1, 2}
+
+
+def test_decode_equals_prefill_on_device():
+    K, S, steps, vocab, d = 3, 64, 20, 2000, 64
+    ft, fl, hist, hl, new, F, T = _decode_case(K, S, steps, vocab, d, seed=11)
+    hl[:] = 0
+    table = scone.scone_table_build(ft, fl, K, vocab, d, dev_rows(F), dev_rows(T))
+    st = scone.scone_decode_create(table, hist, hl)
+    new_d = torch.from_numpy(new).to(DEV)
+    outs = []
+    out = torch.empty((S, d), dtype=torch.int16, device=DEV)
+    for k in range(steps):
+        scone.scone_decode_step(st, new_d[k], out)
+        outs.append(out.clone())
+    dec = torch.stack(outs, 1).cpu().numpy().view(np.uint16)     # [S, steps, d]
+    pre, _, _ = run_embed(table, np.ascontiguousarray(new.T), d)
+    assert np.array_equal(dec.reshape(-1, d), pre)
