@@ -7,7 +7,7 @@ One step is one pass of the whole path (match + gather, fused in one launch)
 over one batch of the workload's seeded synthetic tokens; the default
 workload is the 1B-model prefill configuration (32 x 2048 tokens, 1e6
 f-grams, K = 3, d = 2048, Zipf(1.1) over a 100k vocabulary). Steps rotate
-over 4 distinct batches and L2 is flushed (a 256 MB write) between timed
+over 4 distinct batches and L2 is flushed (256 MB written, then read) between timed
 steps; each step is timed with CUDA events on its stream. Prints one JSON
 line (see the keys below). ``--impl reference`` times the CPU oracle (the
 plain statement of Algorithm 1) on the host cores instead.
@@ -37,8 +37,28 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "embedded tokens/s at 1 GB300; achieved GB/s vs HBM or host-link roofline"
+
+
+def workload(name):
+    import synth
+
+    if name == "prefill_profile":
+        # the prefill law at a size an ncu capture handles (about 1.5 GB on the device)
+        return synth.WORKLOADS["prefill_1b"].scaled("prefill_profile", B=16,
+                                                    quotas=((2, 120000), (3, 80000)))
+    return synth.WORKLOADS[name]
+
+
 N_BATCHES = 4
 FLUSH_BYTES = 256 << 20
+
+
+def flush_l2(buf):
+    """Writes then reads a buffer twice the size of L2: the previous step's
+    lines are gone and the write-backs of the flush itself happen here, not
+    inside the next timed kernel."""
+    buf.zero_()
+    buf.sum()
 
 
 # ------------------------------------------------------------------ clocks
@@ -186,7 +206,7 @@ def bench_prefill(args, world, rank, local):
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    w = synth.WORKLOADS[args.workload]
+    w = workload(args.workload)
     n_tok = w.B * w.L
     t0 = time.time()
     fg_tok, fg_len, used = synth.fgram_set(w)
@@ -201,6 +221,9 @@ def bench_prefill(args, world, rank, local):
     synth.rows_gpu(synth.T_seed(w), w.d, 0, w.vocab, T.data_ptr(), stream.cuda_stream)
     table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, F, T,
                                     load_factor=w.load_factor)
+    scone.scone_table_set_copy_mode(table, {"auto": scone.SCONE_COPY_AUTO,
+                                            "registers": scone.SCONE_COPY_REGISTERS,
+                                            "bulk": scone.SCONE_COPY_BULK}[args.copy])
     info = table.info()
     setup_s = time.time() - t0
     batches = [torch.from_numpy(b).to(dev) for b in batches_np]
@@ -218,7 +241,7 @@ def bench_prefill(args, world, rank, local):
         scone.scone_embed(table, batches[k % N_BATCHES], out)
 
     for k in range(args.warmup):
-        flush.zero_()
+        flush_l2(flush)
         step(k)
     torch.cuda.synchronize()
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -229,7 +252,7 @@ def bench_prefill(args, world, rank, local):
     wall0 = time.perf_counter()
     with clocks:
         for k in range(args.steps):
-            flush.zero_()
+            flush_l2(flush)
             ev[k][0].record(stream)
             step(k)
             ev[k][1].record(stream)
@@ -253,7 +276,7 @@ def bench_prefill(args, world, rank, local):
     barrier(world)
     e2e_t = []
     for k in range(e2e_steps):
-        flush.zero_()
+        flush_l2(flush)
         torch.cuda.synchronize()
         t1 = time.perf_counter()
         dev_tok.copy_(host_tok[k % N_BATCHES], non_blocking=True)
@@ -285,9 +308,10 @@ def bench_prefill(args, world, rank, local):
                          f"Zipf({w.zipf_s}), F in HBM, load factor {w.load_factor}"),
             "global_batch_tokens": world * n_tok,
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-            "l2": f"flushed between timed steps ({FLUSH_BYTES >> 20} MB write); "
+            "l2": f"flushed between timed steps ({FLUSH_BYTES >> 20} MB write + read back); "
                   f"steps rotate over {N_BATCHES} batches",
             "timing": "CUDA events around each step's launch on its stream",
+            "copy": args.copy,
         },
         "roofline": {
             "bound": "hbm",
@@ -298,7 +322,8 @@ def bench_prefill(args, world, rank, local):
             "traffic": profiled_traffic(w.name),
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
             "algorithmic_bytes_per_launch": bytes_launch,
-            "kernel": "embed_kernel (fused match + gather)",
+            "kernel": "embed_bulk_kernel (fused match + TMA bulk gather)" if args.copy == "bulk"
+                      else "embed_kernel (fused match + gather)",
         },
         "e2e": {
             "value": world * n_tok / (e2e_ms * 1e-3),
@@ -356,7 +381,7 @@ def bench_reference(args, world, rank):
     import synth
     import oracle
 
-    w = synth.WORKLOADS[args.workload]
+    w = workload(args.workload)
     fg_tok, fg_len, _ = synth.fgram_set(w)
     tok = synth.query_tokens(w, range(0, 8))
     o = oracle.Oracle(fg_tok, fg_len, w.K, w.vocab)
@@ -393,8 +418,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="scone", choices=["scone", "reference"])
     ap.add_argument("--workload", default="prefill_1b",
-                    choices=["tiny", "prefill_1b", "large_hbm", "stress_k5"])
+                    choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
+                    help="row copy method of the fused kernel (results are identical)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     world, rank, local = dist_setup()

@@ -128,6 +128,17 @@ int scone_table_get_info(const scone_table* table, scone_table_info* info);
  */
 int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
 
+/* How scone_embed moves rows (a tuning knob; results are identical). */
+enum scone_copy_mode {
+  SCONE_COPY_AUTO = 0,       /* the library picks per call */
+  SCONE_COPY_REGISTERS = 1,  /* 16-byte loads and streaming stores through registers */
+  SCONE_COPY_BULK = 2        /* cp.async.bulk (TMA) through a shared-memory ring; needs rows of a
+                                multiple of 16 bytes, 16-byte aligned F, T and out, and F in
+                                device memory, else scone_embed returns SCONE_ERR_UNSUPPORTED */
+};
+
+int scone_table_set_copy_mode(scone_table* table, int32_t mode);
+
 /*
  * scone_match — the selection step of Algorithm 1 (Sec. 3): for each
  * position, the length of the longest f-gram ending there and its row of F.

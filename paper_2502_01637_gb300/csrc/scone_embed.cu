@@ -1,13 +1,14 @@
 // Prefill path: match, gather and the fused embed (Algorithm 1, inference
 // branch, Sec. 3), plus the launch helpers.
 //
-// Work split: one warp per tile of 32 consecutive positions of the flattened
-// [B x L] batch. Each lane matches one position (all K-1 candidate lengths
-// probed at once, longest hit kept), the 32 selected row addresses go to
-// shared memory, and the warp then streams the 32 rows to the contiguous
-// output block with 16-byte loads, 16 in flight per lane, and streaming
-// (evict-first) stores. Blocks are 8 warps; the grid is capped at the number
-// of blocks that are resident at once and walks the tiles grid-stride.
+// Work split: the grid is persistent (as many 8-warp blocks as are resident
+// at once, all SMs equally loaded) and the flattened [B x L] positions are
+// split evenly over all its warps, so every warp moves the same number of
+// rows (+-1). A warp walks its range in tiles of up to 32 positions: each
+// lane matches one position (all K-1 candidate lengths probed at once,
+// longest hit kept), the selected row addresses go to shared memory, and the
+// warp then streams the rows to the contiguous output block with 16-byte
+// loads, 16 in flight per lane, and streaming (evict-first) stores.
 
 #include <map>
 #include <mutex>
@@ -59,6 +60,13 @@ int grid_size(const void* fn, int64_t blocks_needed) {
   return g < 1 ? 1 : (int)g;
 }
 
+// Copy kernels: every resident block, unless the batch is so small that
+// warps would get fewer than kMinRowsPerWarp rows each.
+constexpr int64_t kMinRowsPerWarp = 8;
+int copy_grid(const void* fn, int64_t n_tok) {
+  return grid_size(fn, (n_tok + kWarps * kMinRowsPerWarp - 1) / (kWarps * kMinRowsPerWarp));
+}
+
 // Widest copy unit (16, 8, 4 or 2 bytes) that the row size and every base
 // address allow.
 int copy_width(const TableView& t, const void* out) {
@@ -87,6 +95,13 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// Positions [lo, hi) of warp w out of nw, an even split of n.
+__device__ __forceinline__ void warp_range(int64_t n, int64_t w, int64_t nw, int64_t* lo,
+                                           int64_t* hi) {
+  *lo = n * w / nw;
+  *hi = n * (w + 1) / nw;
+}
+
 template <int FMT, int KT, int W>
 __global__ void __launch_bounds__(kThreads)
     embed_kernel(const TableView t, const int32_t* __restrict__ tok, int64_t n_tok, int32_t L,
@@ -95,12 +110,13 @@ __global__ void __launch_bounds__(kThreads)
   __shared__ const void* src_s[kWarps][32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int row_bytes = t.d * 2;
-  const int64_t n_tiles = (n_tok + 31) >> 5;
-  for (int64_t tile = (int64_t)blockIdx.x * kWarps + warp; tile < n_tiles;
-       tile += (int64_t)gridDim.x * kWarps) {
-    const int64_t p = (tile << 5) + lane;
+  int64_t lo, hi;
+  warp_range(n_tok, (int64_t)blockIdx.x * kWarps + warp, (int64_t)gridDim.x * kWarps, &lo, &hi);
+  for (int64_t base = lo; base < hi; base += 32) {
+    const int nrows = (int)(hi - base < 32 ? hi - base : 32);
+    const int64_t p = base + lane;
     const void* src = nullptr;
-    if (p < n_tok) {
+    if (lane < nrows) {
       const int32_t x = __ldg(tok + p);
       int len = 0, err = 0;
       const int32_t r = match_position<FMT, KT>(t, tok, p, pos_in_seq(p, L), x, &len, &err);
@@ -115,9 +131,8 @@ __global__ void __launch_bounds__(kThreads)
     }
     src_s[warp][lane] = src;
     __syncwarp();
-    const int nrows = (int)(n_tok - (tile << 5) < 32 ? n_tok - (tile << 5) : 32);
-    warp_copy_rows_w<W>(src_s[warp], out + (tile << 5) * (int64_t)row_bytes, nrows, row_bytes,
-                        width, lane);
+    warp_copy_rows_w<W>(src_s[warp], out + base * (int64_t)row_bytes, nrows, row_bytes, width,
+                        lane);
     __syncwarp();
   }
 }
@@ -130,12 +145,13 @@ __global__ void __launch_bounds__(kThreads)
   __shared__ const void* src_s[kWarps][32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int row_bytes = t.d * 2;
-  const int64_t n_tiles = (n_tok + 31) >> 5;
-  for (int64_t tile = (int64_t)blockIdx.x * kWarps + warp; tile < n_tiles;
-       tile += (int64_t)gridDim.x * kWarps) {
-    const int64_t p = (tile << 5) + lane;
+  int64_t lo, hi;
+  warp_range(n_tok, (int64_t)blockIdx.x * kWarps + warp, (int64_t)gridDim.x * kWarps, &lo, &hi);
+  for (int64_t base = lo; base < hi; base += 32) {
+    const int nrows = (int)(hi - base < 32 ? hi - base : 32);
+    const int64_t p = base + lane;
     const void* src = nullptr;
-    if (p < n_tok) {
+    if (lane < nrows) {
       const int32_t r = __ldg(row + p);
       if (r >= 0) {
         if (r < t.n_fgrams) src = t.F + (int64_t)r * t.d;
@@ -148,9 +164,8 @@ __global__ void __launch_bounds__(kThreads)
     }
     src_s[warp][lane] = src;
     __syncwarp();
-    const int nrows = (int)(n_tok - (tile << 5) < 32 ? n_tok - (tile << 5) : 32);
-    warp_copy_rows_w<W>(src_s[warp], out + (tile << 5) * (int64_t)row_bytes, nrows, row_bytes,
-                        width, lane);
+    warp_copy_rows_w<W>(src_s[warp], out + base * (int64_t)row_bytes, nrows, row_bytes, width,
+                        lane);
     __syncwarp();
   }
 }
@@ -216,7 +231,7 @@ extern "C" int scone_embed_gather(const scone_table* tb, const int32_t* tok, con
   DeviceGuard g(tb->device);
   const int width = copy_width(tb->view, out);
   const auto fn = width == 16 ? gather_kernel<16> : gather_kernel<0>;
-  const int grid = grid_size((const void*)fn, ((n_tok + 31) / 32 + kWarps - 1) / kWarps);
+  const int grid = copy_grid((const void*)fn, n_tok);
   fn<<<grid, kThreads, 0, (cudaStream_t)stream>>>(tb->view, tok, row, n_tok,
                                                   reinterpret_cast<uint8_t*>(out), width);
   return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
@@ -230,9 +245,15 @@ extern "C" int scone_embed(const scone_table* tb, const int32_t* tok, int32_t B,
   if (!tok || !out || misaligned(tok, 4) || misaligned(out, 2) || (row && misaligned(row, 4)))
     return SCONE_ERR_INVALID_ARG;
   DeviceGuard g(tb->device);
+  const bool bulk_ok = bulk_eligible(tb, out);
+  if (tb->copy_mode == SCONE_COPY_BULK) {
+    if (!bulk_ok) return SCONE_ERR_UNSUPPORTED;
+    return launch_embed_bulk(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
+                             (cudaStream_t)stream);
+  }
   const int width = copy_width(tb->view, out);
   const EmbedFn fn = pick_embed(tb->fmt, tb->view.K, width);
-  const int grid = grid_size((const void*)fn, ((n + 31) / 32 + kWarps - 1) / kWarps);
+  const int grid = copy_grid((const void*)fn, n);
   fn<<<grid, kThreads, 0, (cudaStream_t)stream>>>(tb->view, tok, n, L,
                                                   reinterpret_cast<uint8_t*>(out), row, len,
                                                   width);

@@ -12,6 +12,8 @@ struct scone_table {
   int fmt = scone::FMT16;
   uint8_t* slots = nullptr;  // n_buckets * 32 bytes
   int* status = nullptr;     // sticky device error word
+  uint8_t* zero_row = nullptr;  // d * 2 zero bytes: the source of error positions (bulk copies)
+  int copy_mode = SCONE_COPY_AUTO;
   scone::TableView view{};
   scone_table_info info{};
 };
@@ -37,6 +39,11 @@ struct DeviceGuard {
     if (prev >= 0 && prev != want) cudaSetDevice(prev);
   }
 };
+
+// Bulk (TMA) fused embed: eligibility for a call and launch.
+bool bulk_eligible(const scone_table* tb, const void* out);
+int launch_embed_bulk(const scone_table* tb, const int32_t* tok, int64_t n, int32_t L,
+                      uint8_t* out, int32_t* row, uint8_t* len, cudaStream_t stream);
 
 // Resident blocks per SM for a kernel at a block size (cached per function).
 int blocks_per_sm(const void* fn, int threads, size_t smem);

@@ -191,7 +191,8 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   cudaGetDevice(&t->device);
   cudaStream_t s = (cudaStream_t)stream;
   if (cudaMalloc(&t->slots, (size_t)n_buckets * kBucketBytes) != cudaSuccess ||
-      cudaMalloc(&t->status, sizeof(int)) != cudaSuccess) {
+      cudaMalloc(&t->status, sizeof(int)) != cudaSuccess ||
+      cudaMalloc(&t->zero_row, (size_t)d * 2) != cudaSuccess) {
     cudaGetLastError();
     scone_table_destroy(t);
     return SCONE_ERR_NOMEM;
@@ -203,7 +204,8 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   BuildFlags flags = {0, 0, 0};
   do {
     if (cudaMemsetAsync(t->slots, 0xFF, (size_t)n_buckets * kBucketBytes, s) != cudaSuccess ||
-        cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess) {
+        cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess ||
+        cudaMemsetAsync(t->zero_row, 0, (size_t)d * 2, s) != cudaSuccess) {
       rc = SCONE_ERR_CUDA;
       break;
     }
@@ -294,9 +296,10 @@ extern "C" int scone_table_destroy(scone_table* t) {
   int prev = -1;
   cudaGetDevice(&prev);
   if (prev != t->device) cudaSetDevice(t->device);
-  if (t->slots || t->status) cudaDeviceSynchronize();
+  if (t->slots || t->status || t->zero_row) cudaDeviceSynchronize();
   if (t->slots) cudaFree(t->slots);
   if (t->status) cudaFree(t->status);
+  if (t->zero_row) cudaFree(t->zero_row);
   if (prev >= 0 && prev != t->device) cudaSetDevice(prev);
   delete t;
   return SCONE_OK;
@@ -312,6 +315,12 @@ extern "C" int scone_table_set_probe_limit(scone_table* t, int64_t max_buckets) 
   if (!t || max_buckets < 1) return SCONE_ERR_INVALID_ARG;
   t->view.probe_limit =
       max_buckets > (int64_t)t->view.n_buckets ? (int64_t)t->view.n_buckets : max_buckets;
+  return SCONE_OK;
+}
+
+extern "C" int scone_table_set_copy_mode(scone_table* t, int32_t mode) {
+  if (!t || mode < SCONE_COPY_AUTO || mode > SCONE_COPY_BULK) return SCONE_ERR_INVALID_ARG;
+  t->copy_mode = mode;
   return SCONE_OK;
 }
 

@@ -283,3 +283,51 @@ def test_decode_equals_prefill_on_device():
     dec = torch.stack(outs, 1).cpu().numpy().view(np.uint16)     # [S, steps, d]
     pre, _, _ = run_embed(table, np.ascontiguousarray(new.T), d)
     assert np.array_equal(dec.reshape(-1, d), pre)
+
+
+# ---------------------------------------------------- bulk (TMA) row copies
+@pytest.mark.parametrize("name,K,vocab,d,B,L,quotas", [
+    ("bulk_tiny", 3, 32000, 256, 4, 512, ((2, 60000), (3, 40000))),
+    ("bulk_d2048_ragged", 3, 100000, 2048, 3, 1001, ((2, 30000), (3, 20000))),
+    ("bulk_k5_d1536", 5, 100000, 1536, 2, 900, ((2, 9000), (3, 9000), (4, 4000), (5, 4000))),
+    ("bulk_d4096", 3, 100000, 4096, 2, 333, ((2, 3000), (3, 2000))),
+    ("bulk_one_row", 3, 1000, 2048, 1, 1, ((2, 10), (3, 10))),
+])
+def test_bulk_copy_parity(name, K, vocab, d, B, L, quotas):
+    w = synth.Workload(name, 60 + K, vocab, 1.1, B, L, quotas, K, d)
+    case = SmallCase(w)
+    table = case.build()
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_BULK)
+    out, row, ln = run_embed(table, case.tok, d)
+    assert_parity(case, out, row, ln)
+    assert scone.scone_status(table) == 0
+
+
+def test_bulk_copy_error_positions_get_zero_rows():
+    w = TINY.scaled("bulk_bad", B=3, L=300, quotas=((2, 3000), (3, 2000)))
+    tok = synth.query_tokens(w)
+    tok[0, 3] = -1
+    tok[2, 299] = w.vocab + 5
+    case = SmallCase(w, tok=tok)
+    table = case.build()
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_BULK)
+    out, row, ln = run_embed(table, case.tok, w.d)
+    assert_parity(case, out, row, ln)
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+
+
+def test_bulk_copy_refuses_ineligible_calls():
+    w = TINY.scaled("bulk_inel", B=1, L=64, quotas=((2, 300), (3, 200)))
+    case = SmallCase(w)
+    table = case.build()
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_BULK)
+    t = torch.from_numpy(case.tok).to(DEV)
+    buf = torch.empty(w.B * w.L * w.d + 1, dtype=torch.int16, device=DEV)
+    with pytest.raises(scone.SconeError) as e:
+        scone.scone_embed(table, t, buf[1:])          # output not 16-byte aligned
+    assert e.value.code == scone.SCONE_ERR_UNSUPPORTED
+    with pytest.raises(scone.SconeError):
+        scone.scone_table_set_copy_mode(table, 7)
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_REGISTERS)
+    out, row, ln = run_embed(table, case.tok, w.d, out_offset=1)
+    assert_parity(case, out, row, ln)
