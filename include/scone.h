@@ -101,6 +101,39 @@ int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_len, int64_
 /* Frees the slot array and status word (after a device synchronize). NULL is a no-op. */
 int scone_table_destroy(scone_table* table);
 
+/*
+ * scone_table_rebuild_noalloc — puts a new f-gram list (and its rows F) into
+ * a table made by scone_table_build, without allocating any memory. The
+ * paper has no counterpart: it is for callers that cannot allocate at the
+ * moment they swap lists, e.g. a serving process whose device memory is
+ * owned by another allocator (cudaMalloc would fail or fragment it), or a
+ * latency-bound thread that must not pay for cudaMalloc / cudaFree, which can
+ * synchronize the whole device.
+ *
+ * It reuses the table's own slot array, so the new list must fit it: at most
+ * 0.95 * n_slots f-grams (see scone_table_get_info). K, vocab, d, T and the F
+ * location stay those of the original build. The build kernels' scratch (a
+ * device copy of the list plus three flags) lives in one file-scope device
+ * array of SCONE_REBUILD_SCRATCH_BYTES, which every GPU that loads the library
+ * holds until the process exits; a list needs 64 + n_fgrams * (4 K + 1)
+ * bytes of it, rounded up to 256, and a larger list is rejected with
+ * SCONE_ERR_INVALID_ARG before any device work. The first call on a device
+ * looks the array's address up (once per device); make that first call
+ * before any stream capture begins.
+ *
+ * All calls share that array and it keeps the last call's contents; the
+ * flags are cleared by each call. Calls whose device work overlaps (other
+ * streams, other threads) race on it, and so do lookups on this table from
+ * other streams during the call. Synchronous: it synchronizes `stream`.
+ * Errors: INVALID_ARG (table NULL, list too large for the table or the
+ * scratch, bad list or F), DUPLICATE_FGRAM or TABLE_FULL (the table is then
+ * left empty: every position falls back to T), CUDA.
+ */
+#define SCONE_REBUILD_SCRATCH_BYTES (16u << 20)
+int scone_table_rebuild_noalloc(scone_table* table, const int32_t* fgram_tok,
+                                const uint8_t* fgram_len, int64_t n_fgrams, const scone_bf16* F,
+                                void* stream);
+
 /* Host-side description of a built table (sizes are in bytes). */
 typedef struct scone_table_info {
   int64_t n_fgrams;

@@ -37,7 +37,8 @@ SCONE_COPY_AUTO = 0
 SCONE_COPY_REGISTERS = 1
 SCONE_COPY_BULK = 2
 
-EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_get_info",
+EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noalloc",
+           "scone_table_get_info",
            "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
@@ -78,6 +79,7 @@ def load_library():
     lib.scone_table_build.argtypes = [_vp, _vp, _i64, _i32, _i32, _i32, _vp, _i32, _vp,
                                       ctypes.c_float, _vp, ctypes.POINTER(_vp)]
     lib.scone_table_destroy.argtypes = [_vp]
+    lib.scone_table_rebuild_noalloc.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_table_get_info.argtypes = [_vp, ctypes.POINTER(scone_table_info)]
     lib.scone_table_set_probe_limit.argtypes = [_vp, _i64]
     lib.scone_table_set_copy_mode.argtypes = [_vp, _i32]
@@ -182,6 +184,29 @@ def scone_table_build(fgram_tok: np.ndarray, fgram_len: np.ndarray, K: int, voca
 
 def scone_table_destroy(table: Table) -> None:
     table.close()
+
+
+def scone_table_rebuild_noalloc(table: Table, fgram_tok: np.ndarray, fgram_len: np.ndarray, F,
+                                stream=None) -> None:
+    """Swaps a new f-gram list (and its rows F) into an existing table without
+    allocating: for callers that may not call cudaMalloc at that point (device
+    memory owned by another allocator, or threads that must not pay for
+    allocation and the device-wide synchronization cudaFree can cause). The
+    list must fit the table (at most 0.95 of its slots) and the library's
+    fixed device scratch (SCONE_REBUILD_SCRATCH_BYTES); calls that overlap on
+    the GPU race on that scratch. Synchronizes the stream.
+    """
+    K = table.info()["K"]
+    ft = np.ascontiguousarray(fgram_tok, dtype=np.int32).reshape(-1)
+    fl = np.ascontiguousarray(fgram_len, dtype=np.uint8).reshape(-1)
+    n = fl.shape[0]
+    if ft.shape[0] != n * K:
+        raise ValueError("fgram_tok must be [n_fgrams, K]")
+    rc = load_library().scone_table_rebuild_noalloc(table.handle, _ptr(ft) if n else None,
+                                                    _ptr(fl) if n else None, n, _ptr(F),
+                                                    _stream(stream))
+    table._keep = (F, table._keep[1] if table._keep else None)
+    _check(rc, "scone_table_rebuild_noalloc")
 
 
 def scone_table_get_info(table: Table) -> dict:

@@ -16,6 +16,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <new>
 
 #include "scone_device.cuh"
@@ -374,3 +375,143 @@ extern "C" const char* scone_strerror(int code) {
 }
 
 extern "C" int scone_version(void) { return (1 << 16) | 0; }
+
+// ------------------------------------------------------------------------
+// Rebuild without allocating (scone_table_rebuild_noalloc).
+//
+// For callers that cannot allocate when they swap in a new f-gram list: the
+// table's slot array, status word and zero row are reused as they are, and
+// the build kernels' per-call scratch (device copy of the list, build
+// flags) lives in the file-scope array below instead of cudaMalloc'd
+// buffers. Host code never uses the array's name as an address: the device
+// address is looked up with cudaGetSymbolAddress once per device, with that
+// device current, on the first call there.
+
+static __device__ __align__(256) uint8_t g_rebuild_scratch[SCONE_REBUILD_SCRATCH_BYTES];
+
+namespace scone {
+namespace {
+
+constexpr int kMaxScratchDevices = 64;
+std::mutex g_scratch_mu;
+uint8_t* g_scratch_addr[kMaxScratchDevices];  // zero-initialized: not looked up yet
+
+int rebuild_scratch(int dev, uint8_t** out) {
+  if (dev < 0 || dev >= kMaxScratchDevices) return SCONE_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_rebuild_scratch) != cudaSuccess || !p) {
+      cudaGetLastError();
+      return SCONE_ERR_CUDA;
+    }
+    g_scratch_addr[dev] = static_cast<uint8_t*>(p);
+  }
+  *out = g_scratch_addr[dev];
+  return SCONE_OK;
+}
+
+constexpr int64_t round256(int64_t x) { return (x + 255) / 256 * 256; }
+
+}  // namespace
+}  // namespace scone
+
+extern "C" int scone_table_rebuild_noalloc(scone_table* t, const int32_t* fgram_tok,
+                                           const uint8_t* fgram_len, int64_t n_fgrams,
+                                           const scone_bf16* F, void* stream) {
+  if (!t || n_fgrams < 0) return SCONE_ERR_INVALID_ARG;
+  if (n_fgrams > 0 && (!fgram_tok || !fgram_len || !F)) return SCONE_ERR_INVALID_ARG;
+  const int K = t->view.K, vocab = t->view.vocab, d = t->view.d;
+  // the new list must fit the existing slot array at load factor <= 0.95
+  if ((double)n_fgrams > 0.95 * (double)t->info.n_slots) return SCONE_ERR_INVALID_ARG;
+  // scratch layout: [flags: 64 B][fgram_len: n B][fgram_tok: n * K * 4 B], 256-aligned parts
+  const int64_t off_len = 256;
+  const int64_t off_tok = off_len + round256(n_fgrams);
+  const int64_t need = off_tok + round256(n_fgrams * K * 4);
+  if (n_fgrams > 0 && need > (int64_t)SCONE_REBUILD_SCRATCH_BYTES) return SCONE_ERR_INVALID_ARG;
+  for (int64_t r = 0; r < n_fgrams; ++r) {
+    const int n = fgram_len[r];
+    if (n < 2 || n > K) return SCONE_ERR_INVALID_ARG;
+    for (int j = 0; j < n; ++j)
+      if (fgram_tok[r * K + j] < 0 || fgram_tok[r * K + j] >= vocab) return SCONE_ERR_INVALID_ARG;
+  }
+  DeviceGuard g(t->device);
+  const uint16_t* F_dev = reinterpret_cast<const uint16_t*>(F);
+  if (n_fgrams > 0) {
+    if (t->info.F_location == SCONE_ROWS_DEVICE) {
+      if (!is_device_accessible(F)) return SCONE_ERR_INVALID_ARG;
+    } else {
+      void* dp = nullptr;
+      if (cudaHostGetDevicePointer(&dp, const_cast<scone_bf16*>(F), 0) != cudaSuccess || !dp) {
+        cudaGetLastError();
+        return SCONE_ERR_INVALID_ARG;
+      }
+      F_dev = reinterpret_cast<const uint16_t*>(dp);
+    }
+  }
+  uint8_t* scratch = nullptr;
+  int rc = rebuild_scratch(t->device, &scratch);
+  if (rc != SCONE_OK) return rc;
+  BuildFlags* d_flags = reinterpret_cast<BuildFlags*>(scratch);
+  uint8_t* d_len = scratch + off_len;
+  int32_t* d_tok = reinterpret_cast<int32_t*>(scratch + off_tok);
+  const uint64_t n_buckets = (uint64_t)t->info.n_buckets;
+  const uint64_t n_slots = (uint64_t)t->info.n_slots;
+  cudaStream_t s = (cudaStream_t)stream;
+  BuildFlags flags = {0, 0, 0};
+  // the array keeps the previous call's contents: the flags must start at zero
+  if (cudaMemsetAsync(t->slots, 0xFF, (size_t)n_buckets * kBucketBytes, s) != cudaSuccess ||
+      cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess ||
+      cudaMemsetAsync(d_flags, 0, sizeof(BuildFlags), s) != cudaSuccess) {
+    cudaGetLastError();
+    return SCONE_ERR_CUDA;
+  }
+  if (n_fgrams > 0) {
+    if (cudaMemcpyAsync(d_tok, fgram_tok, (size_t)n_fgrams * K * sizeof(int32_t),
+                        cudaMemcpyHostToDevice, s) != cudaSuccess ||
+        cudaMemcpyAsync(d_len, fgram_len, (size_t)n_fgrams, cudaMemcpyHostToDevice, s) !=
+            cudaSuccess) {
+      cudaGetLastError();
+      return SCONE_ERR_CUDA;
+    }
+    const int th = 256;
+    if (t->fmt == FMT16) {
+      insert_kernel<FMT16><<<grid_for(n_fgrams, th), th, 0, s>>>(
+          t->slots, n_buckets, d_tok, d_len, n_fgrams, K, t->view.bits, d_flags);
+      fill_keys_kernel<FMT16><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
+          t->slots, n_slots, d_tok, d_len, K, t->view.bits);
+    } else {
+      insert_kernel<FMT32><<<grid_for(n_fgrams, th), th, 0, s>>>(
+          t->slots, n_buckets, d_tok, d_len, n_fgrams, K, t->view.bits, d_flags);
+      fill_keys_kernel<FMT32><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
+          t->slots, n_slots, d_tok, d_len, K, t->view.bits);
+    }
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemcpyAsync(&flags, d_flags, sizeof(BuildFlags), cudaMemcpyDeviceToHost, s) !=
+            cudaSuccess) {
+      cudaGetLastError();
+      return SCONE_ERR_CUDA;
+    }
+  }
+  if (cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return SCONE_ERR_CUDA;
+  }
+  rc = flags.duplicate ? SCONE_ERR_DUPLICATE_FGRAM : (flags.full ? SCONE_ERR_TABLE_FULL : SCONE_OK);
+  if (rc != SCONE_OK) {
+    // leave a valid, empty table: every position falls back to T
+    if (cudaMemsetAsync(t->slots, 0xFF, (size_t)n_buckets * kBucketBytes, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess) {
+      cudaGetLastError();
+      return SCONE_ERR_CUDA;
+    }
+    n_fgrams = 0;
+    flags.max_probe = 0;
+  }
+  t->view.n_fgrams = n_fgrams;
+  t->view.F = n_fgrams > 0 ? F_dev : t->view.F;
+  t->info.n_fgrams = n_fgrams;
+  t->info.max_insert_probe = flags.max_probe;
+  t->info.F_bytes = n_fgrams * (int64_t)d * 2;
+  return rc;
+}
