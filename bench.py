@@ -46,6 +46,10 @@ def workload(name):
         # the prefill law at a size an ncu capture handles (about 1.5 GB on the device)
         return synth.WORKLOADS["prefill_1b"].scaled("prefill_profile", B=16,
                                                     quotas=((2, 120000), (3, 80000)))
+    if name == "decode_profile":
+        # the offloaded-decode law with 2e6 f-grams (8 GB of host rows) for ncu captures
+        return synth.WORKLOADS["offload_decode"].scaled(
+            "decode_profile", quotas=((2, 1_200_000), (3, 800_000)))
     return synth.WORKLOADS[name]
 
 
@@ -224,13 +228,15 @@ def bench_prefill(args, world, rank, local):
     scone.scone_table_set_copy_mode(table, {"auto": scone.SCONE_COPY_AUTO,
                                             "registers": scone.SCONE_COPY_REGISTERS,
                                             "bulk": scone.SCONE_COPY_BULK}[args.copy])
+    if args.prefetch >= 0:
+        scone.scone_table_set_prefetch_rows(table, args.prefetch)
     info = table.info()
     setup_s = time.time() - t0
     batches = [torch.from_numpy(b).to(dev) for b in batches_np]
     out = torch.empty((n_tok, w.d), dtype=torch.int16, device=dev)
     row = torch.empty(n_tok, dtype=torch.int32, device=dev)
     ln = torch.empty(n_tok, dtype=torch.uint8, device=dev)
-    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
 
     # match statistics of the workload (diagnostic; untimed)
     scone.scone_match(table, batches[0], row, ln)
@@ -312,6 +318,7 @@ def bench_prefill(args, world, rank, local):
                   f"steps rotate over {N_BATCHES} batches",
             "timing": "CUDA events around each step's launch on its stream",
             "copy": args.copy,
+            "prefetch_rows": args.prefetch if args.prefetch >= 0 else "default",
         },
         "roofline": {
             "bound": "hbm",
@@ -375,6 +382,157 @@ def cpu_baseline(w, fg_tok, fg_len, tok, F, T, budget_s: float = 10.0):
                       f"({toks} tokens, {dt:.1f} s, map build untimed)"}
 
 
+# ------------------------------------------------------- offloaded decode
+def host_link_bandwidth(dev, table, F_rows: int, d: int):
+    """Host -> device bandwidth, measured two ways; the larger is the roofline.
+
+    copy: pinned cudaMemcpyAsync of 1 GiB, best of 10.
+    zero_copy: the library's gather kernel streaming consecutive rows of the
+    host-mapped F (device loads over the host link), 1 GiB, best of 10.
+    """
+    import torch
+
+    import paper_2502_01637_gb300 as scone
+
+    nb = 1 << 30
+    src = torch.empty(nb, dtype=torch.uint8).pin_memory()
+    dst = torch.empty(nb, dtype=torch.uint8, device=dev)
+    best_copy = 0.0
+    for _ in range(10):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        dst.copy_(src, non_blocking=True)
+        b.record()
+        b.synchronize()
+        best_copy = max(best_copy, nb / (a.elapsed_time(b) * 1e-3) / 1e9)
+    del dst
+    n = min(F_rows, nb // (2 * d))
+    row = torch.arange(n, dtype=torch.int32, device=dev)
+    tok = torch.zeros(n, dtype=torch.int32, device=dev)
+    out = torch.empty((n, d), dtype=torch.int16, device=dev)
+    best_zc = 0.0
+    for _ in range(10):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        scone.scone_embed_gather(table, tok, row, out)
+        b.record()
+        b.synchronize()
+        best_zc = max(best_zc, n * 2 * d / (a.elapsed_time(b) * 1e-3) / 1e9)
+    scone.scone_status(table)
+    return {"copy_gbs": best_copy, "zero_copy_gbs": best_zc, "peak_gbs": max(best_copy, best_zc)}
+
+
+def bench_decode(args, world, rank, local):
+    import torch
+
+    import synth
+    import paper_2502_01637_gb300 as scone
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = workload(args.workload)
+    t0 = time.time()
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    stream = torch.cuda.current_stream()
+    buf = scone.scone_host_alloc(w.n_fgrams * w.d * 2)
+    synth.rows_gpu(synth.F_seed(w), w.d, 0, w.n_fgrams, buf.ptr, stream.cuda_stream)
+    T = torch.empty((w.vocab, w.d), dtype=torch.int16, device=dev)
+    synth.rows_gpu(synth.T_seed(w), w.d, 0, w.vocab, T.data_ptr(), stream.cuda_stream)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, buf.ptr, T,
+                                    F_location=scone.SCONE_ROWS_HOST_MAPPED)
+    setup_s = time.time() - t0
+    link = host_link_bandwidth(dev, table, w.n_fgrams, w.d)
+    hist, hl, new = synth.decode_inputs(w)
+    S, steps = w.dec_S, w.dec_steps
+    new_d = torch.from_numpy(new).to(dev)
+    out = torch.empty((S, w.d), dtype=torch.int16, device=dev)
+    lens = torch.empty((steps, S), dtype=torch.uint8, device=dev)
+    # one eager pass: match lengths of every step (host bytes = matched rows)
+    st = scone.scone_decode_create(table, hist, hl)
+    for k in range(steps):
+        scone.scone_decode_step(st, new_d[k], out, None, lens[k])
+    scone.scone_status(table)
+    ln = lens.cpu().numpy()
+    matched = int((ln >= 2).sum())
+    hist_counts = np.bincount(ln.reshape(-1), minlength=w.K + 1)
+    st.close()
+    # timed: the 256-step loop captured once in a CUDA graph, replayed
+    st = scone.scone_decode_create(table, hist, hl)
+    for k in range(3):
+        scone.scone_decode_step(st, new_d[k], out)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for k in range(steps):
+            scone.scone_decode_step(st, new_d[k], out)
+    replays = max(1, args.steps // steps)
+    for _ in range(max(1, args.warmup // steps) + 1):
+        g.replay()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(replays)]
+    clocks = ClockSampler(local)
+    torch.cuda.synchronize()
+    with clocks:
+        for r in range(replays):
+            ev[r][0].record()
+            g.replay()
+            ev[r][1].record()
+        torch.cuda.synchronize()
+    scone.scone_status(table)
+    per_replay = [a.elapsed_time(b) for a, b in ev]
+    ms_step = statistics.mean(per_replay) / steps
+    host_bytes_step = matched / steps * 2 * w.d
+    hbm_bytes_step = (S * (4 + 32 * (w.K - 1)) + (S - matched / steps) * 2 * w.d + S * 2 * w.d)
+    achieved = host_bytes_step / (ms_step * 1e-3) / 1e9
+    res = {
+        "metric": METRIC,
+        "value": S / (ms_step * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": replays * steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded Zipf histories, tokens and f-gram set)",
+        "config": {
+            "workload": (f"{w.name}: {S} live sequences x {steps} decode steps, "
+                         f"{w.n_fgrams} f-grams (n=2..{w.K}), d={w.d}, vocab {w.vocab}, "
+                         f"F ({w.n_fgrams * w.d * 2 / 1e9:.1f} GB) host-pinned, device-mapped"),
+            "timing": f"{steps} steps captured in one CUDA graph, {replays} replays, "
+                      "CUDA events per replay",
+            "l2": "working set per replay (~%d MB of rows) exceeds L2" %
+                  (steps * S * 2 * w.d * 2 >> 20),
+        },
+        "roofline": {
+            "bound": "host-link",
+            "achieved": achieved,
+            "peak": link["peak_gbs"],
+            "unit": "GB/s",
+            "frac": achieved / link["peak_gbs"],
+            "traffic": None,
+            "peak_source": "measured in this run: max(pinned 1 GiB H2D copy, zero-copy "
+                           "streaming read by the gather kernel)",
+            "host_link": link,
+            "host_bytes_per_step": host_bytes_step,
+            "hbm_bytes_per_step": hbm_bytes_step,
+            "kernel": "decode_kernel (one warp per sequence)",
+        },
+        "gpu_launches": replays * steps,
+        "clocks": clocks.summary(),
+        "match_len_hist": {str(i): int(c) for i, c in enumerate(hist_counts)},
+        "match_rate": matched / (S * steps),
+        "setup_s": setup_s,
+    }
+    st.close()
+    table.close()
+    buf.free()
+    return res
+
+
 # ----------------------------------------------------------- reference arm
 def bench_reference(args, world, rank):
     """The CPU oracle on the host cores, same workload and metric."""
@@ -418,10 +576,13 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="scone", choices=["scone", "reference"])
     ap.add_argument("--workload", default="prefill_1b",
-                    choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile"])
+                    choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
+                             "offload_decode", "decode_profile"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
+    ap.add_argument("--prefetch", type=int, default=-1,
+                    help="L2 prefetch distance in rows (-1: library default)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     world, rank, local = dist_setup()
@@ -434,7 +595,10 @@ def main():
     if rank == 0:
         __graft_entry__.build()
     barrier(world)
-    res = bench_prefill(args, world, rank, local)
+    if args.workload in ("offload_decode", "decode_profile"):
+        res = bench_decode(args, world, rank, local)
+    else:
+        res = bench_prefill(args, world, rank, local)
     if rank == 0:
         print(json.dumps(res), flush=True)
     if world > 1:

@@ -173,6 +173,15 @@ enum scone_copy_mode {
 int scone_table_set_copy_mode(scone_table* table, int32_t mode);
 
 /*
+ * Tuning: how many rows ahead of its register copies each warp of
+ * scone_embed keeps in flight as L2 prefetches (cp.async.bulk.prefetch.L2);
+ * 0..64, 0 disables (the default: distances 2..16 measured no gain on GB300).
+ * Results are identical. For F in host-mapped memory only 0 is accepted
+ * (SCONE_ERR_UNSUPPORTED otherwise).
+ */
+int scone_table_set_prefetch_rows(scone_table* table, int32_t rows);
+
+/*
  * scone_match — the selection step of Algorithm 1 (Sec. 3): for each
  * position, the length of the longest f-gram ending there and its row of F.
  * Probes lengths 2..min(K, i+1), i.e. at most K-1 lookups per token, the

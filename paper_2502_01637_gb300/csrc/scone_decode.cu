@@ -9,6 +9,14 @@
 // the lanes shift the new token into the history, and the warp copies the
 // selected row (F over the host link in the offloaded tier, or T from HBM)
 // with every lane's loads issued at once.
+//
+// Steps are launched with programmatic dependent launch: each step lets the
+// next one be scheduled at once (griddepcontrol.launch_dependents) and every
+// step waits on the device (griddepcontrol.wait) until the previous grid has
+// completed and its writes (the history ring) are visible. The launch
+// latency between consecutive steps overlaps the running step; the data
+// dependency is kept in full. Without a preceding programmatic launch the
+// wait returns at once.
 
 #include <new>
 
@@ -49,6 +57,8 @@ __global__ void __launch_bounds__(kDecThreads)
   __shared__ const void* src_s[kDecWarps][1];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int row_bytes = t.d * 2;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;");
   for (int64_t s = (int64_t)blockIdx.x * kDecWarps + warp; s < S;
        s += (int64_t)gridDim.x * kDecWarps) {
     const int32_t x = __ldg(new_tok + s);
@@ -180,11 +190,24 @@ extern "C" int scone_decode_step(scone_decode* st, const int32_t* new_tok, scone
   const int64_t need = (st->S + kDecWarps - 1) / kDecWarps;
   const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)fn, kDecThreads, 0);
   const int grid = (int)(need < cap ? need : cap);
-  fn<<<grid, kDecThreads, 0, (cudaStream_t)stream>>>(tb->view, st->hist, st->hist_len, new_tok,
-                                                     st->S, st->H,
-                                                     reinterpret_cast<uint8_t*>(out), row, len,
-                                                     width);
-  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kDecThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = (cudaStream_t)stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, fn, tb->view, st->hist, st->hist_len, new_tok,
+                                           st->S, st->H, reinterpret_cast<uint8_t*>(out), row,
+                                           len, width);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return SCONE_ERR_CUDA;
+  }
+  return SCONE_OK;
 }
 
 extern "C" int scone_decode_get_history(const scone_decode* st, int32_t* hist,

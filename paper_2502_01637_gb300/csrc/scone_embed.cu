@@ -8,7 +8,9 @@
 // lane matches one position (all K-1 candidate lengths probed at once,
 // longest hit kept), the selected row addresses go to shared memory, and the
 // warp then streams the rows to the contiguous output block with 16-byte
-// loads, 16 in flight per lane, and streaming (evict-first) stores.
+// loads, 16 in flight per lane, and streaming (evict-first) stores. On
+// request (scone_table_set_prefetch_rows) it also keeps the next rows of its
+// range in flight as bulk L2 prefetches, which hold no registers.
 
 #include <map>
 #include <mutex>
@@ -132,7 +134,7 @@ __global__ void __launch_bounds__(kThreads)
     src_s[warp][lane] = src;
     __syncwarp();
     warp_copy_rows_w<W>(src_s[warp], out + base * (int64_t)row_bytes, nrows, row_bytes, width,
-                        lane);
+                        lane, t.prefetch_rows);
     __syncwarp();
   }
 }

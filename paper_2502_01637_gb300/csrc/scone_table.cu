@@ -24,6 +24,9 @@
 
 namespace scone {
 
+// L2 prefetch distance (rows) of the fused embed for tables with F in HBM.
+constexpr int32_t kDefaultPrefetchRows = 0;
+
 namespace {
 
 struct BuildFlags {
@@ -269,6 +272,7 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   v.F = F_dev;
   v.T = reinterpret_cast<const uint16_t*>(T);
   v.status = t->status;
+  v.prefetch_rows = F_location == SCONE_ROWS_DEVICE ? kDefaultPrefetchRows : 0;
   v.K = K;
   v.bits = bits;
   v.vocab = vocab;
@@ -316,6 +320,13 @@ extern "C" int scone_table_set_probe_limit(scone_table* t, int64_t max_buckets) 
   if (!t || max_buckets < 1) return SCONE_ERR_INVALID_ARG;
   t->view.probe_limit =
       max_buckets > (int64_t)t->view.n_buckets ? (int64_t)t->view.n_buckets : max_buckets;
+  return SCONE_OK;
+}
+
+extern "C" int scone_table_set_prefetch_rows(scone_table* t, int32_t rows) {
+  if (!t || rows < 0 || rows > 64) return SCONE_ERR_INVALID_ARG;
+  if (rows > 0 && t->info.F_location != SCONE_ROWS_DEVICE) return SCONE_ERR_UNSUPPORTED;
+  t->view.prefetch_rows = rows;
   return SCONE_OK;
 }
 

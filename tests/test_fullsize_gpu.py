@@ -1,0 +1,141 @@
+"""Parity at the workloads' full sizes, in the launch configuration the
+benchmark times (GPU).
+
+Every position of the full batch runs through the CUDA path. The oracle
+answers a sample of positions one by one (row id, length, output bytes from
+the host-side row generator); at every position the output must equal the
+row the kernel selected (F[row] or T[token], gathered by torch on the
+device), and the selection must obey the length bounds of Algorithm 1.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+import paper_2502_01637_gb300 as scone
+from gpu_cases import DEV, gpu_rows
+
+pytestmark = pytest.mark.gpu
+
+
+def sample_positions(B, L, K, n_random, seed):
+    rng = np.random.default_rng(seed)
+    starts = np.arange(B, dtype=np.int64) * L
+    pos = [rng.choice(B * L, size=min(n_random, B * L), replace=False),
+           starts, starts + 1, starts + K - 1, starts + L - 1,    # sequence edges
+           np.arange(min(B * L, 300)),                            # the first tiles
+           np.arange(max(0, B * L - 300), B * L)]                 # the ragged end
+    return np.unique(np.concatenate(pos))
+
+
+def check_sampled(w, tok, row, ln, out, pos):
+    o = oracle.Oracle(*synth.fgram_set(w)[:2], w.K, w.vocab)
+    o_row, o_len, rc = o.select_at(tok, pos)
+    assert rc == 0
+    assert np.array_equal(ln[pos], o_len), "lengths differ from the oracle"
+    assert np.array_equal(row[pos], o_row.astype(np.int32)), "rows differ from the oracle"
+    flat_tok = tok.reshape(-1)[pos]
+    exp = np.empty((pos.shape[0], w.d), np.uint16)
+    hit = o_row >= 0
+    exp[hit] = synth.rows_cpu(synth.F_seed(w), w.d, o_row[hit])
+    exp[~hit] = synth.rows_cpu(synth.T_seed(w), w.d, flat_tok[~hit])
+    got = out[torch.from_numpy(pos).to(DEV)].cpu().numpy().view(np.uint16)
+    assert np.array_equal(got, exp), "output bytes differ from the oracle's rows"
+
+
+def check_all_positions(w, tok_d, row_d, ln_d, out, F, T):
+    n = tok_d.numel()
+    r64 = row_d.to(torch.int64)
+    sel = torch.where(r64 >= 0, r64, 0)
+    expect_f = F.index_select(0, sel)
+    expect_t = T.index_select(0, tok_d.reshape(-1).to(torch.int64))
+    exp = torch.where((r64 >= 0)[:, None], expect_f, expect_t)
+    assert torch.equal(out, exp), "some output row is not the row the kernel selected"
+    i = torch.arange(n, device=DEV) % tok_d.shape[-1]
+    ln = ln_d.to(torch.int64)
+    assert bool(((r64 >= 0) == (ln >= 2)).all())
+    assert bool((ln >= 1).all()) and bool((ln <= torch.clamp(i + 1, max=w.K)).all())
+    return torch.bincount(ln, minlength=w.K + 1).cpu().numpy()
+
+
+@pytest.mark.parametrize("name", ["prefill_1b", "large_hbm", "stress_k5"])
+def test_fullsize_prefill(name):
+    w = synth.WORKLOADS[name]
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    tok = synth.query_tokens(w)
+    F = gpu_rows(synth.F_seed(w), w.n_fgrams, w.d)
+    T = gpu_rows(synth.T_seed(w), w.vocab, w.d)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, F, T,
+                                    load_factor=w.load_factor)
+    tok_d = torch.from_numpy(tok).to(DEV)
+    n = tok.size
+    out = torch.empty((n, w.d), dtype=torch.int16, device=DEV)
+    row_d = torch.empty(n, dtype=torch.int32, device=DEV)
+    ln_d = torch.empty(n, dtype=torch.uint8, device=DEV)
+    scone.scone_embed(table, tok_d, out, row_d, ln_d)          # AUTO, as the benchmark runs
+    assert scone.scone_status(table) == 0
+    hist = check_all_positions(w, tok_d, row_d, ln_d, out, F, T)
+    assert (hist[1:] > 0).all(), f"some length never occurs: {hist}"
+    # the same launch without the optional outputs writes the same rows
+    out2 = torch.empty_like(out)
+    scone.scone_embed(table, tok_d, out2)
+    assert torch.equal(out, out2)
+    pos = sample_positions(w.B, w.L, w.K, 6000, seed=len(name))
+    check_sampled(w, tok, row_d.cpu().numpy(), ln_d.cpu().numpy(), out, pos)
+    table.close()
+
+
+def test_fullsize_offload_decode():
+    """2e7 f-grams, F (82 GB) in host-pinned mapped memory; 512 sequences x 256
+    steps. Rows and lengths of every step are checked against the oracle (decode
+    is Algorithm 1 on prefix + new tokens); output bytes on a sample."""
+    w = synth.WORKLOADS["offload_decode"]
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    nbytes = w.n_fgrams * w.d * 2
+    try:
+        buf = scone.scone_host_alloc(nbytes)
+    except scone.SconeError as e:
+        pytest.fail(f"host-pinned allocation of {nbytes / 1e9:.1f} GB failed: {e}")
+    stream = torch.cuda.current_stream().cuda_stream
+    synth.rows_gpu(synth.F_seed(w), w.d, 0, w.n_fgrams, buf.ptr, stream)
+    T = gpu_rows(synth.T_seed(w), w.vocab, w.d)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, buf.ptr, T,
+                                    F_location=scone.SCONE_ROWS_HOST_MAPPED)
+    hist, hl, new = synth.decode_inputs(w)
+    st = scone.scone_decode_create(table, hist, hl)
+    S, steps = w.dec_S, w.dec_steps
+    new_d = torch.from_numpy(new).to(DEV)
+    rows = torch.empty((steps, S), dtype=torch.int32, device=DEV)
+    lens = torch.empty((steps, S), dtype=torch.uint8, device=DEV)
+    keep = np.random.default_rng(5).choice(S, 16, replace=False)
+    keep_d = torch.from_numpy(keep).to(DEV)
+    kept = torch.empty((steps, keep.shape[0], w.d), dtype=torch.int16, device=DEV)
+    out = torch.empty((S, w.d), dtype=torch.int16, device=DEV)
+    for k in range(steps):
+        scone.scone_decode_step(st, new_d[k], out, rows[k], lens[k])
+        kept[k] = out.index_select(0, keep_d)
+    assert scone.scone_status(table) == 0
+    rows, lens = rows.cpu().numpy(), lens.cpu().numpy()
+    # oracle: Algorithm 1 over prefix ++ new tokens, positions after the prefix
+    H = w.K - 1
+    seq = np.concatenate([hist, new.T], axis=1)               # [S, H + steps]; hl == H here
+    assert (hl == H).all()
+    o = oracle.Oracle(fg_tok, fg_len, w.K, w.vocab)
+    pos = (np.arange(S)[:, None] * (H + steps) + H + np.arange(steps)[None, :]).reshape(-1)
+    o_row, o_len, rc = o.select_at(seq, pos)
+    assert rc == 0
+    assert np.array_equal(lens.T.reshape(-1), o_len)
+    assert np.array_equal(rows.T.reshape(-1), o_row.astype(np.int32))
+    assert (o_len == 3).any() and (o_len == 1).any()
+    r = rows[:, keep]                                          # [steps, 16]
+    t = new[:, keep]
+    exp = np.empty((steps, keep.shape[0], w.d), np.uint16)
+    hit = r >= 0
+    exp[hit] = synth.rows_cpu(synth.F_seed(w), w.d, r[hit])
+    exp[~hit] = synth.rows_cpu(synth.T_seed(w), w.d, t[~hit])
+    assert np.array_equal(kept.cpu().numpy().view(np.uint16), exp)
+    st.close()
+    table.close()
+    buf.free()
