@@ -173,15 +173,6 @@ enum scone_copy_mode {
 int scone_table_set_copy_mode(scone_table* table, int32_t mode);
 
 /*
- * Tuning: how many rows ahead of its register copies each warp of
- * scone_embed keeps in flight as L2 prefetches (cp.async.bulk.prefetch.L2);
- * 0..64, 0 disables (the default: distances 2..16 measured no gain on GB300).
- * Results are identical. For F in host-mapped memory only 0 is accepted
- * (SCONE_ERR_UNSUPPORTED otherwise).
- */
-int scone_table_set_prefetch_rows(scone_table* table, int32_t rows);
-
-/*
  * scone_match — the selection step of Algorithm 1 (Sec. 3): for each
  * position, the length of the longest f-gram ending there and its row of F.
  * Probes lengths 2..min(K, i+1), i.e. at most K-1 lookups per token, the
@@ -248,10 +239,15 @@ int scone_status(const scone_table* table, void* stream);
 
 /*
  * Host memory for the offloaded tier: pinned and mapped into the device
- * address space (cudaHostAlloc with cudaHostAllocMapped | cudaHostAllocPortable),
- * so kernels read it over the host link. Use it for F with
- * SCONE_ROWS_HOST_MAPPED. Synchronous. Errors: INVALID_ARG (bytes < 1 or
- * out NULL), NOMEM (the pinned allocation failed; *out is NULL).
+ * address space, so kernels read it over the host link. Use it for F with
+ * SCONE_ROWS_HOST_MAPPED. Where the OS offers transparent huge pages the
+ * buffer is a huge-page-aligned anonymous mapping advised MADV_HUGEPAGE,
+ * touched, then registered (cudaHostRegister, Mapped | Portable): scattered
+ * row reads over tens of GB then need far fewer GPU address translations
+ * (measured on GB300: 2x the random-row read rate of cudaHostAlloc memory at
+ * 82 GB). Otherwise it is cudaHostAlloc(Mapped | Portable). The contents
+ * start as zeros only in the first case. Synchronous. Errors: INVALID_ARG
+ * (bytes < 1 or out NULL), NOMEM (no pinned allocation succeeded; *out is NULL).
  */
 int scone_host_alloc(int64_t bytes, void** out);
 

@@ -39,8 +39,7 @@ SCONE_COPY_BULK = 2
 
 EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noalloc",
            "scone_table_get_info",
-           "scone_table_set_probe_limit", "scone_table_set_copy_mode",
-           "scone_table_set_prefetch_rows", "scone_match", "scone_embed_gather", "scone_embed",
+           "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
            "scone_strerror", "scone_version")
@@ -84,7 +83,6 @@ def load_library():
     lib.scone_table_get_info.argtypes = [_vp, ctypes.POINTER(scone_table_info)]
     lib.scone_table_set_probe_limit.argtypes = [_vp, _i64]
     lib.scone_table_set_copy_mode.argtypes = [_vp, _i32]
-    lib.scone_table_set_prefetch_rows.argtypes = [_vp, _i32]
     lib.scone_match.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp]
     lib.scone_embed_gather.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_embed.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]
@@ -226,11 +224,6 @@ def scone_table_set_probe_limit(table: Table, max_buckets: int) -> None:
 def scone_table_set_copy_mode(table: Table, mode: int) -> None:
     _check(load_library().scone_table_set_copy_mode(table.handle, mode),
            "scone_table_set_copy_mode")
-
-
-def scone_table_set_prefetch_rows(table: Table, rows: int) -> None:
-    _check(load_library().scone_table_set_prefetch_rows(table.handle, rows),
-           "scone_table_set_prefetch_rows")
 
 
 def _bl(tok):

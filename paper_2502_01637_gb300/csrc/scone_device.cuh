@@ -57,7 +57,6 @@ struct TableView {
   const uint16_t* F;         // device-accessible address of F (HBM or host-mapped)
   const uint16_t* T;
   int* status;               // sticky first device-detected error
-  int32_t prefetch_rows;     // L2 prefetch distance of the fused copy (0: off)
   int32_t K;
   int32_t bits;
   int32_t vocab;
@@ -250,43 +249,22 @@ __device__ __forceinline__ uint2 zero_of<uint2>() {
 
 constexpr int kLoadsInFlight = 16;
 
-// Asks L2 to fetch bytes at p (16-byte aligned, a multiple of 16 bytes) from
-// DRAM without waiting and without holding registers or shared memory.
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
-
 // A warp copies nrows rows of epr elements of type E: row r from src[r]
 // (NULL writes zeros) to dst + r * epr, rows contiguous in dst. The warp
 // walks the nrows * epr elements in order, lane l taking every 32nd one, and
 // keeps U loads per lane outstanding before the matching streaming stores.
 // (row, column) of a lane's element advance incrementally, so any row width
-// works without a division. With pf_rows > 0 the warp also keeps the next
-// pf_rows rows beyond the ones being loaded in flight as L2 prefetches
-// (whole rows, so E must be uint4-sized chunks of a 16-byte multiple row).
+// works without a division.
 template <typename E, int U>
 __device__ __forceinline__ void warp_copy_rows(const E* const* src, E* __restrict__ dst,
-                                               int nrows, int epr, int lane, int pf_rows = 0) {
+                                               int nrows, int epr, int lane) {
   const int64_t total = (int64_t)nrows * epr;
-  const int rows_per_iter = (32 * U + epr - 1) / epr + 1;
-  int pf = rows_per_iter;   // rows [0, pf) need no prefetch: they are loaded at once
   int r = 0, col = lane;
   while (col >= epr) {
     col -= epr;
     ++r;
   }
   for (int64_t base = 0; base < total; base += 32 * U) {
-    if (pf_rows > 0) {
-      const int r0 = __shfl_sync(0xFFFFFFFFu, r, 0);
-      int want = r0 + rows_per_iter + pf_rows;
-      if (want > nrows) want = nrows;
-      const int n = want - pf < 32 ? want - pf : 32;
-      if (lane < n) {
-        const E* s = src[pf + lane];
-        if (s != nullptr) prefetch_l2(s, (uint32_t)(epr * sizeof(E)));
-      }
-      if (n > 0) pf += n;
-    }
     E v[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -309,17 +287,15 @@ __device__ __forceinline__ void warp_copy_rows(const E* const* src, E* __restric
   }
 }
 
-// Row copy for a width chosen at run time: 16-byte chunks when W == 16,
-// otherwise the widest of 8, 4 or 2 bytes that the row size and all three
-// base addresses allow (width_bytes).
-template <int W>
+// Row copy for a width chosen at run time: 16-byte chunks when W == 16
+// (U of them in flight per lane), otherwise the widest of 8, 4 or 2 bytes
+// that the row size and all three base addresses allow (width_bytes).
+template <int W, int U = kLoadsInFlight>
 __device__ __forceinline__ void warp_copy_rows_w(const void* const* src, void* dst, int nrows,
-                                                 int row_bytes, int width_bytes, int lane,
-                                                 int pf_rows = 0) {
+                                                 int row_bytes, int width_bytes, int lane) {
   if constexpr (W == 16) {
-    warp_copy_rows<uint4, kLoadsInFlight>(reinterpret_cast<const uint4* const*>(src),
-                                          reinterpret_cast<uint4*>(dst), nrows, row_bytes >> 4,
-                                          lane, pf_rows);
+    warp_copy_rows<uint4, U>(reinterpret_cast<const uint4* const*>(src),
+                             reinterpret_cast<uint4*>(dst), nrows, row_bytes >> 4, lane);
   } else {
     if (width_bytes == 8) {
       warp_copy_rows<uint2, kLoadsInFlight>(reinterpret_cast<const uint2* const*>(src),

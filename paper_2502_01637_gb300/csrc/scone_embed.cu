@@ -8,9 +8,14 @@
 // lane matches one position (all K-1 candidate lengths probed at once,
 // longest hit kept), the selected row addresses go to shared memory, and the
 // warp then streams the rows to the contiguous output block with 16-byte
-// loads, 16 in flight per lane, and streaming (evict-first) stores. On
-// request (scone_table_set_prefetch_rows) it also keeps the next rows of its
-// range in flight as bulk L2 prefetches, which hold no registers.
+// loads and streaming (evict-first) stores.
+//
+// Occupancy: the match of a tile is a chain of dependent loads during which
+// its warp moves no rows, so the kernel wants many resident warps; the copy
+// wants many loads in flight per warp. For K <= 3 the best measured split is
+// 8 loads in flight per lane with 3 blocks (24 warps) per SM (80 registers,
+// no spills); for the longer unrolls 16 loads in flight with 2 blocks
+// (K <= 5) or 1 block (K <= 8), where the keys need more registers.
 
 #include <map>
 #include <mutex>
@@ -104,8 +109,14 @@ __device__ __forceinline__ void warp_range(int64_t n, int64_t w, int64_t nw, int
   *hi = n * (w + 1) / nw;
 }
 
+template <int KT>
+struct EmbedTuning {
+  static constexpr int kLoads = KT <= 3 ? 8 : 16;
+  static constexpr int kMinBlocks = KT <= 3 ? 3 : (KT <= 5 ? 2 : 1);
+};
+
 template <int FMT, int KT, int W>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, EmbedTuning<KT>::kMinBlocks)
     embed_kernel(const TableView t, const int32_t* __restrict__ tok, int64_t n_tok, int32_t L,
                  uint8_t* __restrict__ out, int32_t* __restrict__ row_out,
                  uint8_t* __restrict__ len_out, int width) {
@@ -133,8 +144,8 @@ __global__ void __launch_bounds__(kThreads)
     }
     src_s[warp][lane] = src;
     __syncwarp();
-    warp_copy_rows_w<W>(src_s[warp], out + base * (int64_t)row_bytes, nrows, row_bytes, width,
-                        lane, t.prefetch_rows);
+    warp_copy_rows_w<W, EmbedTuning<KT>::kLoads>(src_s[warp], out + base * (int64_t)row_bytes,
+                                                 nrows, row_bytes, width, lane);
     __syncwarp();
   }
 }

@@ -13,19 +13,22 @@
 // after an unbroken run of occupied slots from its home bucket: the
 // invariant linear-probe lookups rely on.
 
+#include <sys/mman.h>
+#include <unistd.h>
+
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <map>
 #include <mutex>
 #include <new>
+#include <thread>
+#include <vector>
 
 #include "scone_device.cuh"
 #include "scone_host.h"
 
 namespace scone {
-
-// L2 prefetch distance (rows) of the fused embed for tables with F in HBM.
-constexpr int32_t kDefaultPrefetchRows = 0;
 
 namespace {
 
@@ -272,7 +275,6 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   v.F = F_dev;
   v.T = reinterpret_cast<const uint16_t*>(T);
   v.status = t->status;
-  v.prefetch_rows = F_location == SCONE_ROWS_DEVICE ? kDefaultPrefetchRows : 0;
   v.K = K;
   v.bits = bits;
   v.vocab = vocab;
@@ -323,13 +325,6 @@ extern "C" int scone_table_set_probe_limit(scone_table* t, int64_t max_buckets) 
   return SCONE_OK;
 }
 
-extern "C" int scone_table_set_prefetch_rows(scone_table* t, int32_t rows) {
-  if (!t || rows < 0 || rows > 64) return SCONE_ERR_INVALID_ARG;
-  if (rows > 0 && t->info.F_location != SCONE_ROWS_DEVICE) return SCONE_ERR_UNSUPPORTED;
-  t->view.prefetch_rows = rows;
-  return SCONE_OK;
-}
-
 extern "C" int scone_table_set_copy_mode(scone_table* t, int32_t mode) {
   if (!t || mode < SCONE_COPY_AUTO || mode > SCONE_COPY_BULK) return SCONE_ERR_INVALID_ARG;
   t->copy_mode = mode;
@@ -349,10 +344,85 @@ extern "C" int scone_status(const scone_table* t, void* stream) {
   return code;
 }
 
+// ------------------------------------------------------------------------
+// Host memory for an offloaded F.
+//
+// The offloaded tier reads scattered rows of F over the host link. Over tens
+// of GB, GPU address translation of host pages, not the link, limits random
+// row reads: on GB300 (64 KB base pages) random 4 KB rows over 82 GB of
+// cudaHostAlloc memory read at about a third of the link's sequential rate,
+// and at twice that when the same memory is backed by transparent huge pages.
+// So the buffer is an anonymous mapping aligned to the huge-page size,
+// advised MADV_HUGEPAGE, touched in parallel, then pinned and mapped with
+// cudaHostRegister; if any step fails it falls back to cudaHostAlloc.
+
+namespace scone {
+namespace {
+
+struct HostMapping {
+  void* base;   // what mmap returned
+  size_t len;   // what was mapped
+};
+
+std::mutex g_host_mu;
+std::map<void*, HostMapping> g_host_maps;   // registered buffers by user address
+
+size_t huge_page_bytes() {
+  size_t h = 2u << 20;
+  if (FILE* f = std::fopen("/sys/kernel/mm/transparent_hugepage/hpage_pmd_size", "r")) {
+    unsigned long long v = 0;
+    if (std::fscanf(f, "%llu", &v) == 1 && v >= 4096 && (v & (v - 1)) == 0) h = (size_t)v;
+    std::fclose(f);
+  }
+  return h;
+}
+
+void* map_huge(size_t bytes, HostMapping* m) {
+  const size_t huge = huge_page_bytes();
+  const size_t plen = (bytes + huge - 1) / huge * huge;
+  const size_t len = plen + huge;
+  void* base = mmap(nullptr, len, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
+  if (base == MAP_FAILED) return nullptr;
+  uint8_t* p = reinterpret_cast<uint8_t*>(((uintptr_t)base + huge - 1) / huge * huge);
+  madvise(p, plen, MADV_HUGEPAGE);
+  // first touch, one write per base page, spread over the host cores
+  const size_t page = (size_t)sysconf(_SC_PAGESIZE) > 0 ? (size_t)sysconf(_SC_PAGESIZE) : 4096;
+  unsigned nt = std::thread::hardware_concurrency();
+  nt = nt < 1 ? 1 : (nt > 32 ? 32 : nt);
+  const size_t chunk = (plen / nt + huge - 1) / huge * huge;
+  std::vector<std::thread> pool;
+  for (unsigned t = 0; t < nt; ++t) {
+    const size_t a = t * chunk, b = a + chunk < plen ? a + chunk : plen;
+    if (a >= b) break;
+    pool.emplace_back([=] {
+      for (size_t o = a; o < b; o += page) p[o] = 0;
+    });
+  }
+  for (auto& th : pool) th.join();
+  m->base = base;
+  m->len = len;
+  return p;
+}
+
+}  // namespace
+}  // namespace scone
+
 extern "C" int scone_host_alloc(int64_t bytes, void** out) {
   if (!out) return SCONE_ERR_INVALID_ARG;
   *out = nullptr;
   if (bytes < 1) return SCONE_ERR_INVALID_ARG;
+  HostMapping m{nullptr, 0};
+  if (void* p = map_huge((size_t)bytes, &m)) {
+    if (cudaHostRegister(p, (size_t)bytes, cudaHostRegisterMapped | cudaHostRegisterPortable) ==
+        cudaSuccess) {
+      std::lock_guard<std::mutex> lk(g_host_mu);
+      g_host_maps[p] = m;
+      *out = p;
+      return SCONE_OK;
+    }
+    cudaGetLastError();
+    munmap(m.base, m.len);
+  }
   void* p = nullptr;
   if (cudaHostAlloc(&p, (size_t)bytes, cudaHostAllocMapped | cudaHostAllocPortable) !=
           cudaSuccess ||
@@ -367,6 +437,20 @@ extern "C" int scone_host_alloc(int64_t bytes, void** out) {
 extern "C" int scone_host_free(void* p) {
   if (!p) return SCONE_OK;
   cudaDeviceSynchronize();
+  HostMapping m{nullptr, 0};
+  {
+    std::lock_guard<std::mutex> lk(g_host_mu);
+    auto it = g_host_maps.find(p);
+    if (it != g_host_maps.end()) {
+      m = it->second;
+      g_host_maps.erase(it);
+    }
+  }
+  if (m.base) {
+    const bool ok = cudaHostUnregister(p) == cudaSuccess;
+    munmap(m.base, m.len);
+    return ok ? SCONE_OK : SCONE_ERR_CUDA;
+  }
   return cudaFreeHost(p) == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
 }
 

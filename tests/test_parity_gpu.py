@@ -331,33 +331,3 @@ def test_bulk_copy_refuses_ineligible_calls():
     scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_REGISTERS)
     out, row, ln = run_embed(table, case.tok, w.d, out_offset=1)
     assert_parity(case, out, row, ln)
-
-
-# ------------------------------------------------------ L2 prefetch distance
-@pytest.mark.parametrize("pf", [0, 1, 3, 8, 64])
-def test_prefetch_distance_does_not_change_results(pf):
-    w = synth.Workload("pf_case", 70, 100000, 1.1, 3, 1000, ((2, 30000), (3, 20000)), 3, 2048)
-    case = SmallCase(w)
-    table = case.build()
-    scone.scone_table_set_prefetch_rows(table, pf)
-    out, row, ln = run_embed(table, case.tok, w.d)
-    assert_parity(case, out, row, ln)
-
-
-def test_prefetch_knob_limits():
-    w = TINY.scaled("pf_limits", B=1, L=64, quotas=((2, 300), (3, 200)))
-    case = SmallCase(w)
-    table = case.build()
-    with pytest.raises(scone.SconeError):
-        scone.scone_table_set_prefetch_rows(table, 65)
-    with pytest.raises(scone.SconeError):
-        scone.scone_table_set_prefetch_rows(table, -1)
-    buf = scone.scone_host_alloc(case.F.nbytes)
-    buf.numpy()[:] = case.F.reshape(-1)
-    host_table = case.build(F_location=scone.SCONE_ROWS_HOST_MAPPED, F=buf.ptr)
-    with pytest.raises(scone.SconeError) as e:
-        scone.scone_table_set_prefetch_rows(host_table, 4)
-    assert e.value.code == scone.SCONE_ERR_UNSUPPORTED
-    scone.scone_table_set_prefetch_rows(host_table, 0)
-    host_table.close()
-    buf.free()
