@@ -381,7 +381,7 @@ def cpu_baseline(w, fg_tok, fg_len, tok, F, T, budget_s: float = 10.0):
 
 
 # ------------------------------------------------------- offloaded decode
-def host_link_bandwidth(dev, table, F_rows: int, d: int):
+def host_link_bandwidth(dev, table, F_rows: int, d: int, zero_copy: bool = True):
     """Host -> device bandwidth, measured two ways; the larger is the roofline.
 
     copy: pinned cudaMemcpyAsync of 1 GiB, best of 10.
@@ -397,7 +397,7 @@ def host_link_bandwidth(dev, table, F_rows: int, d: int):
     nb = 1 << 30
     src = torch.empty(nb, dtype=torch.uint8).pin_memory()
     dst = torch.empty(nb, dtype=torch.uint8, device=dev)
-    best_copy = 0.0
+    best_copy = best_d2h = 0.0
     for _ in range(10):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record()
@@ -405,7 +405,16 @@ def host_link_bandwidth(dev, table, F_rows: int, d: int):
         b.record()
         b.synchronize()
         best_copy = max(best_copy, nb / (a.elapsed_time(b) * 1e-3) / 1e9)
+    for _ in range(10):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        src.copy_(dst, non_blocking=True)
+        b.record()
+        b.synchronize()
+        best_d2h = max(best_d2h, nb / (a.elapsed_time(b) * 1e-3) / 1e9)
     del dst
+    if not zero_copy:
+        return {"copy_gbs": best_copy, "d2h_copy_gbs": best_d2h, "peak_gbs": best_copy}
     n = min(F_rows, nb // (2 * d))
     tok = torch.zeros(n, dtype=torch.int32, device=dev)
     out = torch.empty((n, d), dtype=torch.int16, device=dev)
@@ -426,7 +435,8 @@ def host_link_bandwidth(dev, table, F_rows: int, d: int):
     best_rand = gather_rate(torch.from_numpy(rnd).to(dev))
     scone.scone_status(table)
     return {"copy_gbs": best_copy, "zero_copy_gbs": best_zc,
-            "zero_copy_random_gbs": best_rand, "peak_gbs": max(best_copy, best_zc)}
+            "zero_copy_random_gbs": best_rand, "peak_gbs": max(best_copy, best_zc),
+            "d2h_copy_gbs": best_d2h}
 
 
 def bench_decode(args, world, rank, local):
@@ -540,6 +550,96 @@ def bench_decode(args, world, rank, local):
     return res
 
 
+# --------------------------------------------------- training-time pre-scan
+def bench_prescan(args, world, rank, local):
+    """scone_match over a corpus in host memory: tokens read and (row, len)
+    tags written through host-mapped addresses by the match kernel."""
+    import torch
+
+    import synth
+    import paper_2502_01637_gb300 as scone
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = workload(args.workload)
+    n = w.B * w.L
+    t0 = time.time()
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    F = torch.zeros((w.n_fgrams, w.d), dtype=torch.int16, device=dev)
+    T = torch.zeros((w.vocab, w.d), dtype=torch.int16, device=dev)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, F, T,
+                                    load_factor=w.load_factor)
+    corpus = scone.scone_host_alloc(n * 4)
+    tags_len = scone.scone_host_alloc(n)
+    tags_row = scone.scone_host_alloc(n * 4)
+    synth.query_tokens(w, out=corpus.numpy(np.int32)[:n].reshape(w.B, w.L))
+    setup_s = time.time() - t0
+    link = host_link_bandwidth(dev, table, w.n_fgrams, w.d, zero_copy=False)
+    lib = scone.load_library()
+    stream = torch.cuda.current_stream()
+
+    def step():
+        rc = lib.scone_match(table.handle, corpus.ptr, w.B, w.L, tags_row.ptr, tags_len.ptr,
+                             stream.cuda_stream)
+        assert rc == 0
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    with clocks:
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+    scone.scone_status(table)
+    ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    h2d = 4 * n / (ms * 1e-3) / 1e9
+    d2h = 5 * n / (ms * 1e-3) / 1e9
+    lens = np.bincount(tags_len.numpy(np.uint8)[:n], minlength=w.K + 1)
+    res = {
+        "metric": METRIC,
+        "value": n / (ms * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int32",
+        "data": "synthetic corpus (seeded Zipf sequences) and f-gram set",
+        "config": {"workload": (f"{w.name}: pre-scan of {w.B} x {w.L} = {n} corpus tokens in "
+                                f"host memory, {w.n_fgrams} f-grams (n=2..{w.K}); tags row "
+                                "(int32) and len (uint8) written to host memory"),
+                   "timing": "CUDA events around each full-corpus scone_match"},
+        "roofline": {
+            "bound": "host-link",
+            "achieved": h2d,
+            "peak": link["copy_gbs"],
+            "unit": "GB/s",
+            "frac": max(h2d / link["copy_gbs"], d2h / link["d2h_copy_gbs"]),
+            "traffic": None,
+            "d2h_achieved": d2h,
+            "host_link": link,
+            "kernel": "match_kernel (host-mapped tokens and tags)",
+        },
+        "gpu_launches": args.steps,
+        "clocks": clocks.summary(),
+        "match_len_hist": {str(i): int(c) for i, c in enumerate(lens)},
+        "setup_s": setup_s,
+    }
+    table.close()
+    corpus.free()
+    tags_len.free()
+    tags_row.free()
+    return res
+
+
 # ----------------------------------------------------------- reference arm
 def bench_reference(args, world, rank):
     """The CPU oracle on the host cores, same workload and metric."""
@@ -584,7 +684,7 @@ def main():
     ap.add_argument("--impl", default="scone", choices=["scone", "reference"])
     ap.add_argument("--workload", default="prefill_1b",
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
-                             "offload_decode", "decode_profile"])
+                             "offload_decode", "decode_profile", "prescan"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
@@ -602,6 +702,8 @@ def main():
     barrier(world)
     if args.workload in ("offload_decode", "decode_profile"):
         res = bench_decode(args, world, rank, local)
+    elif args.workload == "prescan":
+        res = bench_prescan(args, world, rank, local)
     else:
         res = bench_prefill(args, world, rank, local)
     if rank == 0:

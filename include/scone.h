@@ -178,9 +178,14 @@ int scone_table_set_copy_mode(scone_table* table, int32_t mode);
  * Probes lengths 2..min(K, i+1), i.e. at most K-1 lookups per token, the
  * bound Sec. 4.3 states ("up to four queries per token" for K = 5). Async.
  *
- *  tok  device int32 [B * L]; row device int32 [B * L] (F row, or -1 when T
- *  is used or on error); len device uint8 [B * L] or NULL (n in 2..K for an
- *  f-gram, 1 for the token fallback, 0 for an error position).
+ *  tok  int32 [B * L]; row int32 [B * L] (F row, or -1 when T is used or on
+ *  error); len uint8 [B * L] or NULL (n in 2..K for an f-gram, 1 for the
+ *  token fallback, 0 for an error position). All three are device-accessible
+ *  addresses: device memory, or host memory from scone_host_alloc, which the
+ *  kernel then reads and writes over the host link. The latter is the
+ *  training-time pre-scan of Appendix F (tag every corpus token with its
+ *  longest matching length): a corpus too large for HBM is tagged in place.
+ *  B * L may exceed 2^31.
  */
 int scone_match(const scone_table* table, const int32_t* tok, int32_t B, int32_t L,
                 int32_t* row, uint8_t* len, void* stream);

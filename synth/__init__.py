@@ -16,6 +16,7 @@ prefill_1b         1e5    1.1   32x2048 1e6 (60/40)  3    2048  device
 large_hbm          1e5    1.1   64x4096 1e7 (60/40)  3    2048  device
 offload_decode     1e5    1.1   512 seq x 256 steps  2e7  3     2048  host-mapped
 stress_k5          1e5    1.05  16x8192 5e6 n=2..5   5    1536  device
+prescan            1e5    1.1   2^19x2048 1e7 (60/40) 3   8     (tokens in host memory)
 =================  =====  ====  ======  ===========  ===  ====  ==============
 
 f-gram sets are the first distinct n-grams of a separate Zipf source stream of
@@ -66,6 +67,9 @@ def _load():
     lib.synth_stream_seed.restype = u64
     lib.synth_zipf_tokens.argtypes = [u64, i32, dbl, i64, dbl, _i32p, _i32p, i32, i32, _i32p]
     lib.synth_zipf_tokens.restype = ctypes.c_int
+    lib.synth_query_batch.argtypes = [u64, ctypes.c_uint32, ctypes.c_uint32, u64, i64, i64, i32,
+                                      dbl, dbl, _i32p, _i32p, i32, i32, _i32p, i32]
+    lib.synth_query_batch.restype = ctypes.c_int
     lib.synth_phrase_pool.argtypes = [u64, i32, dbl, i32, i32, i32, _i32p, _i32p]
     lib.synth_phrase_pool.restype = ctypes.c_int
     lib.synth_fgram_set.argtypes = [u64, i32, dbl, i32, _i64p, dbl, _i32p, _i32p, i32, i32, i64,
@@ -140,6 +144,10 @@ WORKLOADS: Dict[str, Workload] = {
     "stress_k5": Workload("stress_k5", 5, 100000, 1.05, 16, 8192,
                           ((2, 1_666_666), (3, 1_666_666), (4, 833_334), (5, 833_334)), 5, 1536,
                           inject_p=0.05 / 6, n_phrases=4096),
+    # training-time pre-scan (tag every corpus token with its match length and row):
+    # 2^19 training sequences of 2048 tokens (1.07e9 tokens) in host memory
+    "prescan": Workload("prescan", 6, 100000, 1.1, 1 << 19, 2048,
+                        _split(10_000_000, {2: 0.6, 3: 0.4}), 3, 8, location="host_mapped"),
 }
 
 
@@ -180,12 +188,26 @@ def zipf_tokens(w: Workload, seed: int, n: int, inject: bool = True) -> np.ndarr
     return out
 
 
-def query_tokens(w: Workload, seqs: Optional[range] = None) -> np.ndarray:
-    """Query batch [B, L] int32; sequence b is sub-stream b of the query stream."""
+def query_tokens(w: Workload, seqs: Optional[range] = None, out: Optional[np.ndarray] = None,
+                 threads: int = 0) -> np.ndarray:
+    """Query batch [B, L] int32; sequence b is sub-stream b of the query stream.
+
+    ``seqs`` must be a contiguous range; ``out`` may be a preallocated [len, L]
+    int32 array (for instance a view of host-mapped memory).
+    """
     seqs = range(w.B) if seqs is None else seqs
-    out = np.empty((len(seqs), w.L), np.int32)
-    for k, b in enumerate(seqs):
-        out[k] = zipf_tokens(w, stream_seed(w, S_QUERY, b), w.L)
+    assert seqs.step == 1
+    if out is None:
+        out = np.empty((len(seqs), w.L), np.int32)
+    assert out.shape == (len(seqs), w.L) and out.dtype == np.int32 and out.flags["C_CONTIGUOUS"]
+    pt, pl = phrase_pool(w)
+    n_ph = 0 if pt is None else pt.shape[0]
+    stride = 0 if pt is None else pt.shape[1]
+    threads = threads or min(16, os.cpu_count() or 1)
+    rc = _load().synth_query_batch(MASTER_SEED, w.wid, S_QUERY, seqs.start, len(seqs), w.L,
+                                   w.vocab, w.zipf_s, w.inject_p if n_ph else 0.0, _p(pt, _i32p),
+                                   _p(pl, _i32p), n_ph, stride, _p(out, _i32p), threads)
+    assert rc == 0
     return out
 
 

@@ -194,6 +194,36 @@ int synth_zipf_tokens(uint64_t seed, int32_t vocab, double s, int64_t n, double 
   return 0;
 }
 
+// B query sequences of L tokens: sequence k uses the stream seed
+// synth_stream_seed(master, workload_id, stream_id, first_sub + k), exactly
+// as synth_zipf_tokens called once per sequence; sequences are split over
+// `threads` threads. out is [B * L].
+int synth_query_batch(uint64_t master, uint32_t workload_id, uint32_t stream_id,
+                      uint64_t first_sub, int64_t B, int64_t L, int32_t vocab, double s,
+                      double inject_p, const int32_t* ph_tok, const int32_t* ph_len,
+                      int32_t n_ph, int32_t ph_stride, int32_t* out, int32_t threads) {
+  if (vocab <= 0 || B < 0 || L < 0 || s <= 0.0 || (B * L > 0 && !out)) return -1;
+  if (threads < 1) threads = 1;
+  const Zipf z(vocab, s);
+  std::vector<std::thread> pool;
+  const int64_t per = (B + threads - 1) / threads;
+  for (int32_t t = 0; t < threads; ++t) {
+    const int64_t a = t * per, b = std::min<int64_t>(B, a + per);
+    if (a >= b) break;
+    pool.emplace_back([=, &z] {
+      for (int64_t k = a; k < b; ++k) {
+        const uint64_t base = mix64(master ^ (((uint64_t)workload_id << 32) | stream_id));
+        const uint64_t seed = mix64(base ^ mix64(first_sub + (uint64_t)k + kGamma));
+        Stream st(z, seed, inject_p, ph_tok, ph_len, n_ph, ph_stride);
+        int32_t* o = out + k * L;
+        for (int64_t i = 0; i < L; ++i) o[i] = st.next();
+      }
+    });
+  }
+  for (auto& th : pool) th.join();
+  return 0;
+}
+
 // Pool of n_ph phrases with lengths uniform in [min_len, max_len] and Zipf(s)
 // tokens; tok_out is [n_ph * max_len] (row-padded with -1).
 int synth_phrase_pool(uint64_t seed, int32_t vocab, double s, int32_t n_ph, int32_t min_len,

@@ -139,3 +139,41 @@ def test_fullsize_offload_decode():
     st.close()
     table.close()
     buf.free()
+
+
+def test_prescan_host_mapped_corpus():
+    """The training-time pre-scan (Appendix F): scone_match reads a corpus
+    held in host memory and writes its tags (row, len) to host memory. Tags
+    equal those of the same launch on device copies; sampled positions equal
+    the oracle."""
+    w = synth.WORKLOADS["prescan"].scaled("prescan_test", B=4096)   # 8.4M tokens
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    n = w.B * w.L
+    F = torch.zeros((w.n_fgrams, w.d), dtype=torch.int16, device=DEV)
+    T = torch.zeros((w.vocab, w.d), dtype=torch.int16, device=DEV)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, F, T)
+    corpus = scone.scone_host_alloc(n * 4)
+    tags_len = scone.scone_host_alloc(n)
+    tags_row = scone.scone_host_alloc(n * 4)
+    tok = synth.query_tokens(w, out=corpus.numpy(np.int32)[:n].reshape(w.B, w.L))
+    lib = scone.load_library()
+    stream = torch.cuda.current_stream().cuda_stream
+    assert lib.scone_match(table.handle, corpus.ptr, w.B, w.L, tags_row.ptr, tags_len.ptr,
+                           stream) == scone.SCONE_OK
+    assert scone.scone_status(table) == 0
+    h_len = tags_len.numpy(np.uint8)[:n].copy()
+    h_row = tags_row.numpy(np.int32)[:n].copy()
+    tok_d = torch.from_numpy(tok).to(DEV)
+    row_d = torch.empty(n, dtype=torch.int32, device=DEV)
+    ln_d = torch.empty(n, dtype=torch.uint8, device=DEV)
+    scone.scone_match(table, tok_d, row_d, ln_d)
+    assert np.array_equal(h_len, ln_d.cpu().numpy()) and np.array_equal(h_row, row_d.cpu().numpy())
+    o = oracle.Oracle(fg_tok, fg_len, w.K, w.vocab)
+    pos = sample_positions(w.B, w.L, w.K, 20000, seed=17)
+    o_row, o_len, rc = o.select_at(tok, pos)
+    assert rc == 0
+    assert np.array_equal(h_len[pos], o_len) and np.array_equal(h_row[pos], o_row.astype(np.int32))
+    assert (np.bincount(h_len, minlength=4)[1:] > 0).all()
+    table.close()
+    for b in (corpus, tags_len, tags_row):
+        b.free()

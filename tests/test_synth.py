@@ -79,3 +79,12 @@ def test_decode_inputs_shapes():
     hist, hl, new = synth.decode_inputs(w)
     assert hist.shape == (8, 2) and (hl == 2).all() and new.shape == (5, 8)
     assert (hist >= 0).all() and (new >= 0).all() and (new < w.vocab).all()
+
+
+def test_query_batch_equals_per_sequence_streams():
+    for name in ("tiny", "stress_k5"):
+        w = synth.WORKLOADS[name].scaled(name + "_qb", B=5, L=300)
+        batch = synth.query_tokens(w, range(3, 8), threads=3)
+        for k, b in enumerate(range(3, 8)):
+            one = synth.zipf_tokens(w, synth.stream_seed(w, synth.S_QUERY, b), w.L)
+            assert np.array_equal(batch[k], one)
