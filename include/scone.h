@@ -12,10 +12,11 @@
  *
  * F is stored as "a dense embedding matrix paired with a hash dictionary
  * that maps f-grams to matrix indices" (Sec. 2, "Efficient Indexing for
- * Large Embedding Layers"). Here the dictionary is a GPU open-addressing
- * table built once by scone_table_build; the dense matrix stays caller-owned
- * in HBM or in host-pinned, device-mapped memory (the paper's off-accelerator
- * tier, Sec. 4.3).
+ * Large Embedding Layers"). Here the dictionary is a GPU bucketized cuckoo
+ * hash table (two candidate buckets of two slots per key, both read in one
+ * round trip) built once by scone_table_build; the dense matrix stays
+ * caller-owned in HBM or in host-pinned, device-mapped memory (the paper's
+ * off-accelerator tier, Sec. 4.3).
  *
  * Conventions shared by every call
  *  - Pointers are plain addresses; "device" means a CUDA device address
@@ -84,13 +85,15 @@ enum scone_rows_location {
  *             May be NULL only when n_fgrams = 0.
  *  T          device [vocab * d] bf16 token embeddings (Sec. 2: T stays on the
  *             accelerator).
- *  load_factor  target fill of the slot array, in (0, 0.95]; 0 selects 0.5.
+ *  load_factor  target fill of the slot array, in (0, 0.85]; 0 selects 0.5.
  *  stream     used for the build kernels; the call synchronizes it.
  *  out        receives the table.
  *
  * The table borrows F and T (they must outlive it) and owns only its slot
- * array (16 or 32 bytes per slot, 32-byte buckets) and a status word. Errors:
- * INVALID_ARG (bad list, length, token or pointer), DUPLICATE_FGRAM,
+ * array (16- or 32-byte slots, two per bucket), a status word and a zero row.
+ * Insertion may retry with new hash seeds; TABLE_FULL means eight seeds
+ * failed (not expected below load factor 0.85). Errors: INVALID_ARG (bad
+ * list, length, token or pointer), DUPLICATE_FGRAM, TABLE_FULL,
  * UNSUPPORTED (key does not fit: K*ceil(log2 vocab) > 220), NOMEM, CUDA.
  */
 int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_len, int64_t n_fgrams,
@@ -111,7 +114,7 @@ int scone_table_destroy(scone_table* table);
  * synchronize the whole device.
  *
  * It reuses the table's own slot array, so the new list must fit it: at most
- * 0.95 * n_slots f-grams (see scone_table_get_info). K, vocab, d, T and the F
+ * 0.85 * n_slots f-grams (see scone_table_get_info). K, vocab, d, T and the F
  * location stay those of the original build. The build kernels' scratch (a
  * device copy of the list plus three flags) lives in one file-scope device
  * array of SCONE_REBUILD_SCRATCH_BYTES, which every GPU that loads the library
@@ -146,7 +149,7 @@ typedef struct scone_table_info {
   int32_t vocab;
   int32_t d;
   int32_t F_location;
-  int32_t max_insert_probe;  /* most buckets any f-gram insert read */
+  int32_t max_insert_probe;  /* most cuckoo evictions any f-gram insert needed */
   int64_t table_bytes;       /* slot array */
   int64_t F_bytes;           /* n_fgrams * d * 2 (borrowed) */
   int64_t T_bytes;           /* vocab * d * 2 (borrowed) */
@@ -155,9 +158,10 @@ typedef struct scone_table_info {
 int scone_table_get_info(const scone_table* table, scone_table_info* info);
 
 /*
- * Diagnostic: caps the buckets one lookup may read (default: all of them).
- * A lookup that reaches the cap records SCONE_ERR_PROBE_LIMIT and treats the
- * position as an error position. max_buckets >= 1.
+ * Diagnostic: caps the buckets one lookup may read. A lookup normally reads
+ * both candidate buckets (2, the default); with 1 it reads only the first,
+ * and a key not found there makes the position an error position with
+ * SCONE_ERR_PROBE_LIMIT recorded. max_buckets >= 1 (values above 2 act as 2).
  */
 int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
 
@@ -176,7 +180,8 @@ int scone_table_set_copy_mode(scone_table* table, int32_t mode);
  * scone_match — the selection step of Algorithm 1 (Sec. 3): for each
  * position, the length of the longest f-gram ending there and its row of F.
  * Probes lengths 2..min(K, i+1), i.e. at most K-1 lookups per token, the
- * bound Sec. 4.3 states ("up to four queries per token" for K = 5). Async.
+ * bound Sec. 4.3 states ("up to four queries per token" for K = 5); each
+ * lookup reads its two candidate buckets at once. Async.
  *
  *  tok  int32 [B * L]; row int32 [B * L] (F row, or -1 when T is used or on
  *  error); len uint8 [B * L] or NULL (n in 2..K for an f-gram, 1 for the

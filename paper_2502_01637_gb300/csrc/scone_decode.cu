@@ -4,8 +4,9 @@
 // Algorithm 1 only needs the last K-1 tokens before a position, so the state
 // keeps, per sequence, a device ring of its last K-1 tokens (right-aligned,
 // oldest first) and how many of them are known. One warp serves one
-// sequence: lane j probes the window of length j + 2 ending at the new token
-// (a full linear-probe lookup each), a warp ballot keeps the longest hit,
+// sequence: lane j looks up the window of length j + 2 ending at the new
+// token (both cuckoo buckets in one round trip), a warp ballot keeps the
+// longest hit,
 // the lanes shift the new token into the history, and the warp copies the
 // selected row (F over the host link in the offloaded tier, or T from HBM)
 // with every lane's loads issued at once.
@@ -28,24 +29,6 @@ constexpr int kDecThreads = 128;
 constexpr int kDecWarps = kDecThreads / 32;
 
 namespace {
-
-template <int FMT>
-__device__ __forceinline__ int32_t lookup(const TableView& t, const KeyBits<Fmt<FMT>::kWords>& k,
-                                          int* err) {
-  uint64_t q = fastrange(key_hash<FMT>(k), t.n_buckets);
-  int32_t r = check_bucket<FMT>(ld_bucket(t.slots + q * kBucketBytes), k);
-  int64_t reads = 1;
-  while (r == -2) {
-    if (reads >= t.probe_limit) {
-      *err = SCONE_ERR_PROBE_LIMIT;
-      return -1;
-    }
-    q = (q + 1 == t.n_buckets) ? 0 : q + 1;
-    r = check_bucket<FMT>(ld_bucket(t.slots + q * kBucketBytes), k);
-    ++reads;
-  }
-  return r;
-}
 
 template <int FMT, int W>
 __global__ void __launch_bounds__(kDecThreads)
@@ -80,7 +63,7 @@ __global__ void __launch_bounds__(kDecThreads)
         put_field<NW>(k, m * t.bits, (uint32_t)y, t.bits);
       }
       put_len<FMT>(k, n);
-      if (ok) r_lane = lookup<FMT>(t, k, &err);
+      if (ok) r_lane = cuckoo_lookup<FMT>(t, k, &err);
     }
     const unsigned hits = __ballot_sync(0xFFFFFFFFu, r_lane >= 0);
     const unsigned errs = __ballot_sync(0xFFFFFFFFu, err != 0);

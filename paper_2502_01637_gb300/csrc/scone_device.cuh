@@ -1,9 +1,16 @@
 // Device-side building blocks of the SCONE embedding path (sm_103a).
 //
 // The f-gram dictionary (Sec. 2, "a hash dictionary that maps f-grams to
-// matrix indices") is an open-addressing table with linear probing over
-// 32-byte buckets. Every bucket is one DRAM sector and is read with one
-// 256-bit load.
+// matrix indices") is a bucketized cuckoo hash table: every key lives in one
+// of two buckets chosen by two hashes of the key, and a bucket holds two
+// slots (cuckoo hashing: Pagh and Rodler 2001; parallel GPU insertion:
+// Alcantara et al. 2009). The build fills a key's first bucket before its
+// second and never empties a slot, so a key can sit in its second bucket
+// only if its first bucket is full. A lookup therefore reads the first
+// bucket and stops there unless that bucket is full without holding the
+// key; then it reads the second. Every lookup ends after at most two round
+// trips (about 1.3 sectors on average at load factor 0.5), where linear
+// probing has a long tail of dependent reads.
 //
 // Key: an injective packing of the n-gram. Token fields of b bits
 // (b = ceil(log2 vocab)) hold the newest token at bit 0, the one before it
@@ -12,9 +19,9 @@
 // n >= 2, so a valid key is never all ones, which marks an empty slot.
 //
 //   FMT16: key of 96 bits (K*b <= 92), 16-byte slot = {key bits 0..63,
-//          key bits 64..95 | row << 32}; two slots per bucket.
+//          key bits 64..95 | row << 32}; 32-byte buckets (one sector).
 //   FMT32: key of 224 bits (K*b <= 220), 32-byte slot = {key 0..63,
-//          64..127, 128..191, key 192..223 | row << 32}; one slot per bucket.
+//          64..127, 128..191, key 192..223 | row << 32}; 64-byte buckets.
 //
 // The row word of an empty slot is 0xFFFFFFFF (row -1).
 
@@ -27,9 +34,9 @@
 
 namespace scone {
 
-constexpr int kBucketBytes = 32;
 constexpr int FMT16 = 0;
 constexpr int FMT32 = 1;
+constexpr int kSlotsPerBucket = 2;
 constexpr uint32_t kEmptyRow = 0xFFFFFFFFu;
 constexpr uint64_t kHashSeed = 0x6A09E667F3BCC908ull;  // frac(sqrt 2), first 64 bits
 
@@ -38,21 +45,26 @@ struct Fmt;
 template <>
 struct Fmt<FMT16> {
   static constexpr int kWords = 2;        // 64-bit key words (96 bits used)
-  static constexpr int kSlotsPerBucket = 2;
+  static constexpr int kSlotBytes = 16;
   static constexpr int kLenShift = 28;    // length field in bits 92..95 (word 1, bits 28..31)
 };
 template <>
 struct Fmt<FMT32> {
   static constexpr int kWords = 4;        // 224 bits used
-  static constexpr int kSlotsPerBucket = 1;
+  static constexpr int kSlotBytes = 32;
   static constexpr int kLenShift = 28;    // bits 220..223 (word 3, bits 28..31)
 };
+template <int FMT>
+__host__ __device__ constexpr int bucket_bytes() {
+  return kSlotsPerBucket * Fmt<FMT>::kSlotBytes;
+}
 
 // What a kernel needs to know about a table (passed by value).
 struct TableView {
-  const uint8_t* slots;      // bucket q at slots + 32 q
+  const uint8_t* slots;      // bucket q at slots + q * bucket_bytes
   uint64_t n_buckets;
-  int64_t probe_limit;       // buckets one lookup may read
+  uint64_t hash_seed;        // seed of the two bucket hashes (chosen at build)
+  int64_t probe_limit;       // buckets one lookup may read: 1 or 2
   int64_t n_fgrams;
   const uint16_t* F;         // device-accessible address of F (HBM or host-mapped)
   const uint16_t* T;
@@ -99,8 +111,8 @@ __device__ __forceinline__ void put_len(KeyBits<Fmt<FMT>::kWords>& k, int n) {
 }
 
 template <int FMT>
-__device__ __forceinline__ uint64_t key_hash(const KeyBits<Fmt<FMT>::kWords>& k) {
-  uint64_t h = kHashSeed;
+__device__ __forceinline__ uint64_t key_hash(const KeyBits<Fmt<FMT>::kWords>& k, uint64_t seed) {
+  uint64_t h = seed;
 #pragma unroll
   for (int q = Fmt<FMT>::kWords - 1; q >= 0; --q) h = fmix64(k.w[q] ^ h);
   return h;
@@ -109,7 +121,16 @@ __device__ __forceinline__ uint64_t key_hash(const KeyBits<Fmt<FMT>::kWords>& k)
 // Lemire's multiply-shift range reduction: maps h uniformly onto [0, n).
 __device__ __forceinline__ uint64_t fastrange(uint64_t h, uint64_t n) { return __umul64hi(h, n); }
 
-// One 256-bit read-only load of a bucket.
+// The key's two candidate buckets (distinct when n >= 2).
+__device__ __forceinline__ void cuckoo_buckets(uint64_t h, uint64_t n, uint64_t* b1,
+                                               uint64_t* b2) {
+  *b1 = fastrange(h, n);
+  uint64_t q = fastrange(fmix64(h + 0x9E3779B97F4A7C15ull), n);
+  if (q == *b1) q = (q + 1 == n) ? 0 : q + 1;
+  *b2 = q;
+}
+
+// One 256-bit read-only load (32 bytes, one sector).
 __device__ __forceinline__ Bucket ld_bucket(const uint8_t* p) {
   Bucket r;
   asm("ld.global.nc.v4.u64 {%0, %1, %2, %3}, [%4];"
@@ -118,23 +139,67 @@ __device__ __forceinline__ Bucket ld_bucket(const uint8_t* p) {
   return r;
 }
 
-// >= 0: the key's row. -1: definitive miss (an empty slot ends the probe run).
-// -2: bucket full of other keys, continue with the next bucket.
+// A whole bucket in registers: one 32-byte load (FMT16) or two (FMT32).
 template <int FMT>
-__device__ __forceinline__ int32_t check_bucket(const Bucket& v,
-                                                const KeyBits<Fmt<FMT>::kWords>& k) {
+struct BucketData {
+  Bucket part[bucket_bytes<FMT>() / 32];
+};
+
+template <int FMT>
+__device__ __forceinline__ BucketData<FMT> ld_bucket_data(const TableView& t, uint64_t q) {
+  BucketData<FMT> v;
+  const uint8_t* p = t.slots + q * bucket_bytes<FMT>();
+#pragma unroll
+  for (int i = 0; i < bucket_bytes<FMT>() / 32; ++i) v.part[i] = ld_bucket(p + 32 * i);
+  return v;
+}
+
+// Whether both slots of the bucket are taken.
+template <int FMT>
+__device__ __forceinline__ bool bucket_full(const BucketData<FMT>& v) {
   if constexpr (FMT == FMT16) {
-    if (v.a == k.w[0] && (uint32_t)v.b == (uint32_t)k.w[1]) return (int32_t)(v.b >> 32);
-    if ((uint32_t)(v.b >> 32) == kEmptyRow) return -1;
-    if (v.c == k.w[0] && (uint32_t)v.e == (uint32_t)k.w[1]) return (int32_t)(v.e >> 32);
-    if ((uint32_t)(v.e >> 32) == kEmptyRow) return -1;
-    return -2;
+    return (uint32_t)(v.part[0].b >> 32) != kEmptyRow && (uint32_t)(v.part[0].e >> 32) != kEmptyRow;
   } else {
-    if (v.a == k.w[0] && v.b == k.w[1] && v.c == k.w[2] && (uint32_t)v.e == (uint32_t)k.w[3])
-      return (int32_t)(v.e >> 32);
-    if ((uint32_t)(v.e >> 32) == kEmptyRow) return -1;
-    return -2;
+    return (uint32_t)(v.part[0].e >> 32) != kEmptyRow && (uint32_t)(v.part[1].e >> 32) != kEmptyRow;
   }
+}
+
+// The key's row if one of the bucket's slots holds it, else -1.
+template <int FMT>
+__device__ __forceinline__ int32_t find_in_bucket(const BucketData<FMT>& v,
+                                                  const KeyBits<Fmt<FMT>::kWords>& k) {
+  if constexpr (FMT == FMT16) {
+    const Bucket& x = v.part[0];
+    if (x.a == k.w[0] && (uint32_t)x.b == (uint32_t)k.w[1]) return (int32_t)(x.b >> 32);
+    if (x.c == k.w[0] && (uint32_t)x.e == (uint32_t)k.w[1]) return (int32_t)(x.e >> 32);
+    return -1;
+  } else {
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+      const Bucket& x = v.part[s];
+      if (x.a == k.w[0] && x.b == k.w[1] && x.c == k.w[2] && (uint32_t)x.e == (uint32_t)k.w[3])
+        return (int32_t)(x.e >> 32);
+    }
+    return -1;
+  }
+}
+
+// Looks a key up: the first bucket, then the second only if the first is
+// full without the key. With a probe limit of 1 the second bucket is never
+// read; a lookup that would need it reports SCONE_ERR_PROBE_LIMIT.
+template <int FMT>
+__device__ __forceinline__ int32_t cuckoo_lookup(const TableView& t,
+                                                 const KeyBits<Fmt<FMT>::kWords>& k, int* err) {
+  uint64_t b1, b2;
+  cuckoo_buckets(key_hash<FMT>(k, t.hash_seed), t.n_buckets, &b1, &b2);
+  const BucketData<FMT> v1 = ld_bucket_data<FMT>(t, b1);
+  const int32_t r = find_in_bucket<FMT>(v1, k);
+  if (r >= 0 || !bucket_full<FMT>(v1)) return r;
+  if (t.probe_limit < 2) {
+    *err = SCONE_ERR_PROBE_LIMIT;
+    return -1;
+  }
+  return find_in_bucket<FMT>(ld_bucket_data<FMT>(t, b2), k);
 }
 
 __device__ __forceinline__ void record_error(int* status, int code) {
@@ -147,15 +212,30 @@ __device__ __forceinline__ bool valid_token(int32_t x, int32_t vocab) {
 
 // Algorithm 1's selection for one position: the longest n in [2, min(K, i+1)]
 // whose window (tok[p-n+1 .. p]) is an f-gram. All candidate lengths are
-// hashed in registers and their home buckets loaded together (K-1 loads in
-// flight), then resolved longest first; a full bucket continues the linear
-// probe. Returns the row (or -1) and sets *len (n, 1 for the token fallback,
-// 0 for an error position) and *err.
+// hashed in registers and their first buckets loaded together (K-1 loads in
+// one round trip); the lengths that still need their second bucket load it
+// together in a second round trip; then the longest hit wins. Returns the
+// row (or -1) and sets *len (n, 1 for the token fallback, 0 for an error
+// position) and *err.
+template <int FMT, int KT>
+__device__ __forceinline__ KeyBits<Fmt<FMT>::kWords> window_key(const int32_t (&w)[KT], int n,
+                                                               int bits) {
+  constexpr int NW = Fmt<FMT>::kWords;
+  KeyBits<NW> k;
+#pragma unroll
+  for (int q = 0; q < NW; ++q) k.w[q] = 0;
+  k.w[0] = (uint32_t)w[0];
+#pragma unroll
+  for (int j = 1; j < KT; ++j)
+    if (j < n) put_field<NW>(k, j * bits, (uint32_t)w[j], bits);
+  put_len<FMT>(k, n);
+  return k;
+}
+
 template <int FMT, int KT>
 __device__ __forceinline__ int32_t match_position(const TableView& t,
                                                   const int32_t* __restrict__ tok, int64_t p,
                                                   int32_t i, int32_t tok_p, int* len, int* err) {
-  constexpr int NW = Fmt<FMT>::kWords;
   if (!valid_token(tok_p, t.vocab)) {
     *err = SCONE_ERR_TOKEN_RANGE;
     *len = 0;
@@ -173,42 +253,59 @@ __device__ __forceinline__ int32_t match_position(const TableView& t,
     if (nvalid == j && j < nmax && valid_token(w[j], t.vocab)) nvalid = j + 1;
   nmax = nvalid;
 
-  KeyBits<NW> acc;
-#pragma unroll
-  for (int q = 0; q < NW; ++q) acc.w[q] = 0;
-  acc.w[0] = (uint32_t)w[0];
-  KeyBits<NW> keys[KT - 1];
-  uint64_t home[KT - 1];
-  Bucket first[KT - 1];
+  // round trip 1: the first bucket of every candidate length
+  BucketData<FMT> v[KT - 1];
 #pragma unroll
   for (int n = 2; n <= KT; ++n) {
-    put_field<NW>(acc, (n - 1) * t.bits, (uint32_t)w[n - 1], t.bits);
-    keys[n - 2] = acc;
-    put_len<FMT>(keys[n - 2], n);
     if (n <= nmax) {
-      home[n - 2] = fastrange(key_hash<FMT>(keys[n - 2]), t.n_buckets);
-      first[n - 2] = ld_bucket(t.slots + home[n - 2] * kBucketBytes);
+      uint64_t b1, b2;
+      cuckoo_buckets(key_hash<FMT>(window_key<FMT, KT>(w, n, t.bits), t.hash_seed), t.n_buckets,
+                     &b1, &b2);
+      v[n - 2] = ld_bucket_data<FMT>(t, b1);
     }
+  }
+  int32_t r1[KT - 1];
+  uint32_t second = 0;   // bit n-2: length n needs its second bucket
+#pragma unroll
+  for (int n = 2; n <= KT; ++n) {
+    r1[n - 2] = -1;
+    if (n <= nmax) {
+      r1[n - 2] = find_in_bucket<FMT>(v[n - 2], window_key<FMT, KT>(w, n, t.bits));
+      if (r1[n - 2] < 0 && bucket_full<FMT>(v[n - 2])) second |= 1u << (n - 2);
+    }
+  }
+  // only lengths longer than the longest first-round hit matter
+  int best = 0;
+#pragma unroll
+  for (int n = 2; n <= KT; ++n)
+    if (r1[n - 2] >= 0) best = n;
+  second &= ~((1u << (best > 1 ? best - 1 : 0)) - 1u);
+  if (second) {
+    if (t.probe_limit < 2) {
+      *err = SCONE_ERR_PROBE_LIMIT;
+      *len = 0;
+      return -1;
+    }
+    // round trip 2: the second buckets still needed
+#pragma unroll
+    for (int n = 2; n <= KT; ++n) {
+      if (second & (1u << (n - 2))) {
+        uint64_t b1, b2;
+        cuckoo_buckets(key_hash<FMT>(window_key<FMT, KT>(w, n, t.bits), t.hash_seed),
+                       t.n_buckets, &b1, &b2);
+        v[n - 2] = ld_bucket_data<FMT>(t, b2);
+      }
+    }
+#pragma unroll
+    for (int n = 2; n <= KT; ++n)
+      if (second & (1u << (n - 2)))
+        r1[n - 2] = find_in_bucket<FMT>(v[n - 2], window_key<FMT, KT>(w, n, t.bits));
   }
 #pragma unroll
   for (int n = KT; n >= 2; --n) {
-    if (n > nmax) continue;
-    int32_t r = check_bucket<FMT>(first[n - 2], keys[n - 2]);
-    uint64_t q = home[n - 2];
-    int64_t reads = 1;
-    while (r == -2) {
-      if (reads >= t.probe_limit) {
-        *err = SCONE_ERR_PROBE_LIMIT;
-        *len = 0;
-        return -1;
-      }
-      q = (q + 1 == t.n_buckets) ? 0 : q + 1;
-      r = check_bucket<FMT>(ld_bucket(t.slots + q * kBucketBytes), keys[n - 2]);
-      ++reads;
-    }
-    if (r >= 0) {
+    if (n <= nmax && r1[n - 2] >= 0) {
       *len = n;
-      return r;
+      return r1[n - 2];
     }
   }
   *len = 1;

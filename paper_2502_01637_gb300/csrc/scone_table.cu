@@ -1,17 +1,21 @@
 // f-gram table build, lifetime and status (C ABI).
 //
-// Build (Sec. 2: "a hash dictionary that maps f-grams to matrix indices"):
+// Build (Sec. 2: "a hash dictionary that maps f-grams to matrix indices") of
+// the bucketized cuckoo table described in scone_device.cuh:
 //   1. the slot array is set to all ones (every row word = empty);
-//   2. one thread per f-gram claims a slot with a 32-bit atomicCAS on the row
-//      word, walking the linear-probe sequence from its home bucket. When a
-//      CAS finds another row there, the thread compares the two f-grams in
-//      the device copy of the input list: equal means a duplicate, otherwise
-//      it moves on. The list is immutable during the build, so no thread
-//      ever waits on another;
-//   3. one thread per slot writes the packed key of the row it holds.
-// Slots are claimed in probe order and never released, so every key sits
-// after an unbroken run of occupied slots from its home bucket: the
-// invariant linear-probe lookups rely on.
+//   2. one thread per f-gram places its row: it tries to claim an empty slot
+//      of either candidate bucket with a 32-bit atomicCAS on the row word;
+//      if both buckets are full it swaps its row into one of them with
+//      atomicExch and carries the evicted row to that row's other bucket
+//      (parallel cuckoo insertion, Alcantara et al. 2009). Rows are compared
+//      through the device copy of the input list, which is immutable during
+//      the build, so no thread ever waits on another. An eviction chain
+//      longer than kMaxKicks fails the attempt, which is retried from an
+//      empty table with a new hash seed;
+//   3. one thread per slot writes the packed key of the row it holds;
+//   4. one thread per f-gram looks its key up in the finished table: it must
+//      find its own row. Finding another row means the list holds the same
+//      n-gram twice (also when two copies raced past the checks in step 2).
 
 #include <sys/mman.h>
 #include <unistd.h>
@@ -32,10 +36,13 @@ namespace scone {
 
 namespace {
 
+constexpr int kMaxKicks = 512;      // eviction steps before an attempt is abandoned
+constexpr int kMaxAttempts = 8;     // hash seeds tried per build
+
 struct BuildFlags {
   int duplicate;
-  int full;
-  int max_probe;
+  int full;        // an eviction chain exceeded kMaxKicks, or a row was lost
+  int max_kicks;   // most evictions one insert needed
 };
 
 template <int FMT>
@@ -62,41 +69,67 @@ __device__ __forceinline__ bool same_fgram(const int32_t* ftok, const uint8_t* f
   return true;
 }
 
+// The row word of slot s of bucket q (the upper half of the slot's last 8 bytes).
 template <int FMT>
-__global__ void insert_kernel(uint8_t* slots, uint64_t n_buckets, const int32_t* ftok,
-                              const uint8_t* flen, int64_t n, int K, int bits, BuildFlags* flags) {
-  constexpr int SPB = Fmt<FMT>::kSlotsPerBucket;
-  constexpr int SLOT = kBucketBytes / SPB;
+__device__ __forceinline__ unsigned int* row_word(uint8_t* slots, uint64_t q, int s) {
+  constexpr int SLOT = Fmt<FMT>::kSlotBytes;
+  return reinterpret_cast<unsigned int*>(slots + q * bucket_bytes<FMT>() + s * SLOT + SLOT - 4);
+}
+
+template <int FMT>
+__global__ void insert_kernel(uint8_t* slots, uint64_t n_buckets, uint64_t seed,
+                              const int32_t* ftok, const uint8_t* flen, int64_t n, int K, int bits,
+                              BuildFlags* flags) {
   for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n;
        r += (int64_t)gridDim.x * blockDim.x) {
-    const auto k = key_of_listed<FMT>(ftok, flen, r, K, bits);
-    uint64_t q = fastrange(key_hash<FMT>(k), n_buckets);
+    unsigned int cur = (unsigned int)r;   // the row this thread is placing
+    uint64_t from = ~0ull;                // the bucket `cur` was just evicted from
     bool done = false;
-    for (uint64_t probe = 0; probe < n_buckets && !done; ++probe) {
+    int kick = 0;
+    for (; kick <= kMaxKicks && !done; ++kick) {
+      const auto k = key_of_listed<FMT>(ftok, flen, (int64_t)cur, K, bits);
+      uint64_t b[2];
+      cuckoo_buckets(key_hash<FMT>(k, seed), n_buckets, &b[0], &b[1]);
 #pragma unroll
-      for (int s = 0; s < SPB && !done; ++s) {
-        // the row word is the upper half of the slot's last 8 bytes
-        unsigned int* rowp =
-            reinterpret_cast<unsigned int*>(slots + q * kBucketBytes + s * SLOT + SLOT - 4);
-        const unsigned int old = atomicCAS(rowp, kEmptyRow, (unsigned int)r);
-        if (old == kEmptyRow) {
-          atomicMax(&flags->max_probe, (int)(probe + 1 < 0x7FFFFFFF ? probe + 1 : 0x7FFFFFFF));
-          done = true;
-        } else if (same_fgram(ftok, flen, (int64_t)old, r, K)) {
-          atomicExch(&flags->duplicate, 1);
-          done = true;
+      for (int i = 0; i < 2 && !done; ++i) {
+#pragma unroll
+        for (int s = 0; s < kSlotsPerBucket && !done; ++s) {
+          const unsigned int old = atomicCAS(row_word<FMT>(slots, b[i], s), kEmptyRow, cur);
+          if (old == kEmptyRow) {
+            done = true;
+          } else if (same_fgram(ftok, flen, (int64_t)old, (int64_t)cur, K)) {
+            atomicExch(&flags->duplicate, 1);
+            done = true;
+          }
         }
       }
-      q = (q + 1 == n_buckets) ? 0 : q + 1;
+      if (done || kick == kMaxKicks) break;
+      // both buckets full: take a slot of the bucket `cur` did not come from
+      const uint64_t vb = b[0] == from ? b[1] : (b[1] == from ? b[0] : b[kick & 1]);
+      const int vs = (int)((cur ^ (unsigned int)kick) & 1);
+      const unsigned int old = atomicExch(row_word<FMT>(slots, vb, vs), cur);
+      if (old == kEmptyRow) {
+        done = true;
+      } else if (same_fgram(ftok, flen, (int64_t)old, (int64_t)cur, K)) {
+        atomicExch(&flags->duplicate, 1);
+        done = true;
+      } else {
+        cur = old;
+        from = vb;
+      }
     }
-    if (!done) atomicExch(&flags->full, 1);
+    if (done) {
+      atomicMax(&flags->max_kicks, kick);
+    } else {
+      atomicExch(&flags->full, 1);
+    }
   }
 }
 
 template <int FMT>
 __global__ void fill_keys_kernel(uint8_t* slots, uint64_t n_slots, const int32_t* ftok,
                                  const uint8_t* flen, int K, int bits) {
-  constexpr int SLOT = kBucketBytes / Fmt<FMT>::kSlotsPerBucket;
+  constexpr int SLOT = Fmt<FMT>::kSlotBytes;
   constexpr int NW = Fmt<FMT>::kWords;
   for (uint64_t s = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; s < n_slots;
        s += (uint64_t)gridDim.x * blockDim.x) {
@@ -107,6 +140,19 @@ __global__ void fill_keys_kernel(uint8_t* slots, uint64_t n_slots, const int32_t
 #pragma unroll
     for (int q = 0; q < NW - 1; ++q) w[q] = k.w[q];
     w[NW - 1] = (uint64_t)(uint32_t)k.w[NW - 1] | ((uint64_t)row << 32);
+  }
+}
+
+template <int FMT>
+__global__ void verify_kernel(TableView t, const int32_t* ftok, const uint8_t* flen, int64_t n,
+                              int K, BuildFlags* flags) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n;
+       r += (int64_t)gridDim.x * blockDim.x) {
+    const auto k = key_of_listed<FMT>(ftok, flen, r, K, t.bits);
+    int err = 0;
+    const int32_t found = cuckoo_lookup<FMT>(t, k, &err);
+    if (found < 0) atomicExch(&flags->full, 1);             // lost in a failed chain
+    else if (found != (int32_t)r) atomicExch(&flags->duplicate, 1);
   }
 }
 
@@ -135,6 +181,56 @@ bool is_device_accessible(const void* p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
+
+// Steps 1-4 of the build into t->slots for a list already on the device.
+// Tries kMaxAttempts hash seeds; sets t->view.hash_seed and *out_flags.
+// Synchronizes the stream. Returns SCONE_OK, DUPLICATE_FGRAM, TABLE_FULL or CUDA.
+int build_slots(scone_table* t, const int32_t* d_tok, const uint8_t* d_len, BuildFlags* d_flags,
+                int64_t n, cudaStream_t s, BuildFlags* out_flags) {
+  const uint64_t nb = (uint64_t)t->info.n_buckets;
+  const uint64_t n_slots = (uint64_t)t->info.n_slots;
+  const int K = t->view.K, bits = t->view.bits;
+  const size_t bytes = (size_t)t->info.table_bytes;
+  const int th = 256;
+  BuildFlags flags = {0, 0, 0};
+  for (int attempt = 0; attempt < kMaxAttempts; ++attempt) {
+    const uint64_t seed = kHashSeed + (uint64_t)attempt * 0x9E3779B97F4A7C15ull;
+    flags = {0, 0, 0};
+    if (cudaMemsetAsync(t->slots, 0xFF, bytes, s) != cudaSuccess) return SCONE_ERR_CUDA;
+    if (n > 0) {
+      if (cudaMemsetAsync(d_flags, 0, sizeof(BuildFlags), s) != cudaSuccess)
+        return SCONE_ERR_CUDA;
+      TableView v = t->view;
+      v.hash_seed = seed;
+      v.probe_limit = 2;
+      if (t->fmt == FMT16) {
+        insert_kernel<FMT16><<<grid_for(n, th), th, 0, s>>>(t->slots, nb, seed, d_tok, d_len, n,
+                                                            K, bits, d_flags);
+        fill_keys_kernel<FMT16><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
+            t->slots, n_slots, d_tok, d_len, K, bits);
+        verify_kernel<FMT16><<<grid_for(n, th), th, 0, s>>>(v, d_tok, d_len, n, K, d_flags);
+      } else {
+        insert_kernel<FMT32><<<grid_for(n, th), th, 0, s>>>(t->slots, nb, seed, d_tok, d_len, n,
+                                                            K, bits, d_flags);
+        fill_keys_kernel<FMT32><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
+            t->slots, n_slots, d_tok, d_len, K, bits);
+        verify_kernel<FMT32><<<grid_for(n, th), th, 0, s>>>(v, d_tok, d_len, n, K, d_flags);
+      }
+      if (cudaGetLastError() != cudaSuccess ||
+          cudaMemcpyAsync(&flags, d_flags, sizeof(BuildFlags), cudaMemcpyDeviceToHost, s) !=
+              cudaSuccess)
+        return SCONE_ERR_CUDA;
+    }
+    if (cudaStreamSynchronize(s) != cudaSuccess) return SCONE_ERR_CUDA;
+    *out_flags = flags;
+    if (flags.duplicate) return SCONE_ERR_DUPLICATE_FGRAM;
+    if (!flags.full) {
+      t->view.hash_seed = seed;
+      return SCONE_OK;
+    }
+  }
+  return SCONE_ERR_TABLE_FULL;
+}
 }  // namespace
 
 }  // namespace scone
@@ -153,7 +249,7 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   if (F_location != SCONE_ROWS_DEVICE && F_location != SCONE_ROWS_HOST_MAPPED)
     return SCONE_ERR_INVALID_ARG;
   if (load_factor == 0.0f) load_factor = 0.5f;
-  if (!(load_factor > 0.0f && load_factor <= 0.95f)) return SCONE_ERR_INVALID_ARG;
+  if (!(load_factor > 0.0f && load_factor <= 0.85f)) return SCONE_ERR_INVALID_ARG;
   const int bits = bits_for_vocab(vocab);
   const int key_bits = K * bits + 4;
   int fmt;
@@ -186,32 +282,60 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
     }
   }
 
-  const int spb = fmt == FMT16 ? 2 : 1;
   int64_t n_slots = (int64_t)std::ceil((double)n_fgrams / (double)load_factor);
   if (n_slots < n_fgrams + 1) n_slots = n_fgrams + 1;
-  if (n_slots < 2) n_slots = 2;
-  const int64_t n_buckets = (n_slots + spb - 1) / spb;
-  n_slots = n_buckets * spb;
+  int64_t n_buckets = (n_slots + kSlotsPerBucket - 1) / kSlotsPerBucket;
+  if (n_buckets < 2) n_buckets = 2;   // two distinct candidate buckets
+  n_slots = n_buckets * kSlotsPerBucket;
+  const int64_t bucket = fmt == FMT16 ? bucket_bytes<FMT16>() : bucket_bytes<FMT32>();
 
   scone_table* t = new (std::nothrow) scone_table();
   if (!t) return SCONE_ERR_NOMEM;
   cudaGetDevice(&t->device);
   cudaStream_t s = (cudaStream_t)stream;
-  if (cudaMalloc(&t->slots, (size_t)n_buckets * kBucketBytes) != cudaSuccess ||
+  if (cudaMalloc(&t->slots, (size_t)(n_buckets * bucket)) != cudaSuccess ||
       cudaMalloc(&t->status, sizeof(int)) != cudaSuccess ||
       cudaMalloc(&t->zero_row, (size_t)d * 2) != cudaSuccess) {
     cudaGetLastError();
     scone_table_destroy(t);
     return SCONE_ERR_NOMEM;
   }
+  t->fmt = fmt;
+  TableView& v = t->view;
+  v.slots = t->slots;
+  v.n_buckets = (uint64_t)n_buckets;
+  v.hash_seed = kHashSeed;
+  v.probe_limit = 2;
+  v.n_fgrams = n_fgrams;
+  v.F = F_dev;
+  v.T = reinterpret_cast<const uint16_t*>(T);
+  v.status = t->status;
+  v.K = K;
+  v.bits = bits;
+  v.vocab = vocab;
+  v.d = d;
+  scone_table_info& in = t->info;
+  in.n_fgrams = n_fgrams;
+  in.n_slots = n_slots;
+  in.n_buckets = n_buckets;
+  in.slot_bytes = fmt == FMT16 ? Fmt<FMT16>::kSlotBytes : Fmt<FMT32>::kSlotBytes;
+  in.key_bits = key_bits;
+  in.bits_per_token = bits;
+  in.K = K;
+  in.vocab = vocab;
+  in.d = d;
+  in.F_location = F_location;
+  in.table_bytes = n_buckets * bucket;
+  in.F_bytes = n_fgrams * (int64_t)d * 2;
+  in.T_bytes = (int64_t)vocab * d * 2;
+
   int rc = SCONE_OK;
   int32_t* d_tok = nullptr;
   uint8_t* d_len = nullptr;
   BuildFlags* d_flags = nullptr;
   BuildFlags flags = {0, 0, 0};
   do {
-    if (cudaMemsetAsync(t->slots, 0xFF, (size_t)n_buckets * kBucketBytes, s) != cudaSuccess ||
-        cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess ||
+    if (cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess ||
         cudaMemsetAsync(t->zero_row, 0, (size_t)d * 2, s) != cudaSuccess) {
       rc = SCONE_ERR_CUDA;
       break;
@@ -226,36 +350,12 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
       if (cudaMemcpyAsync(d_tok, fgram_tok, (size_t)n_fgrams * K * sizeof(int32_t),
                           cudaMemcpyHostToDevice, s) != cudaSuccess ||
           cudaMemcpyAsync(d_len, fgram_len, (size_t)n_fgrams, cudaMemcpyHostToDevice, s) !=
-              cudaSuccess ||
-          cudaMemsetAsync(d_flags, 0, sizeof(BuildFlags), s) != cudaSuccess) {
-        rc = SCONE_ERR_CUDA;
-        break;
-      }
-      const int th = 256;
-      if (fmt == FMT16) {
-        insert_kernel<FMT16><<<grid_for(n_fgrams, th), th, 0, s>>>(
-            t->slots, (uint64_t)n_buckets, d_tok, d_len, n_fgrams, K, bits, d_flags);
-        fill_keys_kernel<FMT16><<<grid_for(n_slots, th), th, 0, s>>>(
-            t->slots, (uint64_t)n_slots, d_tok, d_len, K, bits);
-      } else {
-        insert_kernel<FMT32><<<grid_for(n_fgrams, th), th, 0, s>>>(
-            t->slots, (uint64_t)n_buckets, d_tok, d_len, n_fgrams, K, bits, d_flags);
-        fill_keys_kernel<FMT32><<<grid_for(n_slots, th), th, 0, s>>>(
-            t->slots, (uint64_t)n_slots, d_tok, d_len, K, bits);
-      }
-      if (cudaGetLastError() != cudaSuccess ||
-          cudaMemcpyAsync(&flags, d_flags, sizeof(BuildFlags), cudaMemcpyDeviceToHost, s) !=
               cudaSuccess) {
         rc = SCONE_ERR_CUDA;
         break;
       }
     }
-    if (cudaStreamSynchronize(s) != cudaSuccess) {
-      rc = SCONE_ERR_CUDA;
-      break;
-    }
-    if (flags.duplicate) rc = SCONE_ERR_DUPLICATE_FGRAM;
-    else if (flags.full) rc = SCONE_ERR_TABLE_FULL;
+    rc = build_slots(t, d_tok, d_len, d_flags, n_fgrams, s, &flags);
   } while (0);
   if (d_tok) cudaFree(d_tok);
   if (d_len) cudaFree(d_len);
@@ -265,35 +365,7 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
     scone_table_destroy(t);
     return rc;
   }
-
-  t->fmt = fmt;
-  TableView& v = t->view;
-  v.slots = t->slots;
-  v.n_buckets = (uint64_t)n_buckets;
-  v.probe_limit = n_buckets;
-  v.n_fgrams = n_fgrams;
-  v.F = F_dev;
-  v.T = reinterpret_cast<const uint16_t*>(T);
-  v.status = t->status;
-  v.K = K;
-  v.bits = bits;
-  v.vocab = vocab;
-  v.d = d;
-  scone_table_info& in = t->info;
-  in.n_fgrams = n_fgrams;
-  in.n_slots = n_slots;
-  in.n_buckets = n_buckets;
-  in.slot_bytes = kBucketBytes / spb;
-  in.key_bits = key_bits;
-  in.bits_per_token = bits;
-  in.K = K;
-  in.vocab = vocab;
-  in.d = d;
-  in.F_location = F_location;
-  in.max_insert_probe = flags.max_probe;
-  in.table_bytes = n_buckets * kBucketBytes;
-  in.F_bytes = n_fgrams * (int64_t)d * 2;
-  in.T_bytes = (int64_t)vocab * d * 2;
+  in.max_insert_probe = flags.max_kicks;
   *out = t;
   return SCONE_OK;
 }
@@ -320,8 +392,7 @@ extern "C" int scone_table_get_info(const scone_table* t, scone_table_info* info
 
 extern "C" int scone_table_set_probe_limit(scone_table* t, int64_t max_buckets) {
   if (!t || max_buckets < 1) return SCONE_ERR_INVALID_ARG;
-  t->view.probe_limit =
-      max_buckets > (int64_t)t->view.n_buckets ? (int64_t)t->view.n_buckets : max_buckets;
+  t->view.probe_limit = max_buckets >= 2 ? 2 : 1;
   return SCONE_OK;
 }
 
@@ -517,8 +588,8 @@ extern "C" int scone_table_rebuild_noalloc(scone_table* t, const int32_t* fgram_
   if (!t || n_fgrams < 0) return SCONE_ERR_INVALID_ARG;
   if (n_fgrams > 0 && (!fgram_tok || !fgram_len || !F)) return SCONE_ERR_INVALID_ARG;
   const int K = t->view.K, vocab = t->view.vocab, d = t->view.d;
-  // the new list must fit the existing slot array at load factor <= 0.95
-  if ((double)n_fgrams > 0.95 * (double)t->info.n_slots) return SCONE_ERR_INVALID_ARG;
+  // the new list must fit the existing slot array at load factor <= 0.85
+  if ((double)n_fgrams > 0.85 * (double)t->info.n_slots) return SCONE_ERR_INVALID_ARG;
   // scratch layout: [flags: 64 B][fgram_len: n B][fgram_tok: n * K * 4 B], 256-aligned parts
   const int64_t off_len = 256;
   const int64_t off_tok = off_len + round256(n_fgrams);
@@ -550,14 +621,9 @@ extern "C" int scone_table_rebuild_noalloc(scone_table* t, const int32_t* fgram_
   BuildFlags* d_flags = reinterpret_cast<BuildFlags*>(scratch);
   uint8_t* d_len = scratch + off_len;
   int32_t* d_tok = reinterpret_cast<int32_t*>(scratch + off_tok);
-  const uint64_t n_buckets = (uint64_t)t->info.n_buckets;
-  const uint64_t n_slots = (uint64_t)t->info.n_slots;
   cudaStream_t s = (cudaStream_t)stream;
   BuildFlags flags = {0, 0, 0};
-  // the array keeps the previous call's contents: the flags must start at zero
-  if (cudaMemsetAsync(t->slots, 0xFF, (size_t)n_buckets * kBucketBytes, s) != cudaSuccess ||
-      cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess ||
-      cudaMemsetAsync(d_flags, 0, sizeof(BuildFlags), s) != cudaSuccess) {
+  if (cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess) {
     cudaGetLastError();
     return SCONE_ERR_CUDA;
   }
@@ -569,44 +635,28 @@ extern "C" int scone_table_rebuild_noalloc(scone_table* t, const int32_t* fgram_
       cudaGetLastError();
       return SCONE_ERR_CUDA;
     }
-    const int th = 256;
-    if (t->fmt == FMT16) {
-      insert_kernel<FMT16><<<grid_for(n_fgrams, th), th, 0, s>>>(
-          t->slots, n_buckets, d_tok, d_len, n_fgrams, K, t->view.bits, d_flags);
-      fill_keys_kernel<FMT16><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
-          t->slots, n_slots, d_tok, d_len, K, t->view.bits);
-    } else {
-      insert_kernel<FMT32><<<grid_for(n_fgrams, th), th, 0, s>>>(
-          t->slots, n_buckets, d_tok, d_len, n_fgrams, K, t->view.bits, d_flags);
-      fill_keys_kernel<FMT32><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
-          t->slots, n_slots, d_tok, d_len, K, t->view.bits);
-    }
-    if (cudaGetLastError() != cudaSuccess ||
-        cudaMemcpyAsync(&flags, d_flags, sizeof(BuildFlags), cudaMemcpyDeviceToHost, s) !=
-            cudaSuccess) {
-      cudaGetLastError();
-      return SCONE_ERR_CUDA;
-    }
   }
-  if (cudaStreamSynchronize(s) != cudaSuccess) {
+  // the array keeps the previous call's contents: build_slots clears the
+  // flags (which must start at zero) before every attempt
+  rc = build_slots(t, d_tok, d_len, d_flags, n_fgrams, s, &flags);
+  if (rc == SCONE_ERR_CUDA) {
     cudaGetLastError();
-    return SCONE_ERR_CUDA;
+    return rc;
   }
-  rc = flags.duplicate ? SCONE_ERR_DUPLICATE_FGRAM : (flags.full ? SCONE_ERR_TABLE_FULL : SCONE_OK);
   if (rc != SCONE_OK) {
     // leave a valid, empty table: every position falls back to T
-    if (cudaMemsetAsync(t->slots, 0xFF, (size_t)n_buckets * kBucketBytes, s) != cudaSuccess ||
+    if (cudaMemsetAsync(t->slots, 0xFF, (size_t)t->info.table_bytes, s) != cudaSuccess ||
         cudaStreamSynchronize(s) != cudaSuccess) {
       cudaGetLastError();
       return SCONE_ERR_CUDA;
     }
     n_fgrams = 0;
-    flags.max_probe = 0;
+    flags.max_kicks = 0;
   }
   t->view.n_fgrams = n_fgrams;
   t->view.F = n_fgrams > 0 ? F_dev : t->view.F;
   t->info.n_fgrams = n_fgrams;
-  t->info.max_insert_probe = flags.max_probe;
+  t->info.max_insert_probe = flags.max_kicks;
   t->info.F_bytes = n_fgrams * (int64_t)d * 2;
   return rc;
 }

@@ -64,6 +64,7 @@ def test_host_validation_returns_before_device_work():
     assert _build_rc(ok_tok, ok_len, 3, 10, T=0) == inv     # no T
     assert _build_rc(ok_tok, ok_len, 3, 10, F=0) == inv     # no F with f-grams
     assert _build_rc(ok_tok, ok_len, 3, 10, lf=0.99) == inv  # load factor too high
+    assert _build_rc(ok_tok, ok_len, 3, 10, lf=0.9) == inv   # above the cuckoo bound 0.85
     assert _build_rc(ok_tok, ok_len, 3, 10, lf=-1.0) == inv
     assert _build_rc(ok_tok, ok_len, 3, 10, loc=7) == inv   # unknown F location
     assert _build_rc(ok_tok, np.array([1], np.uint8), 3, 10) == inv   # 1-gram

@@ -66,7 +66,7 @@ def test_rebuild_noalloc_matches_build_on_two_calls_in_a_row():
     F2 = _rows(OTHER, OTHER.n_fgrams)
     tok = synth.query_tokens(BASE)
     table = scone.scone_table_build(fg1_tok, fg1_len, BASE.K, BASE.vocab, BASE.d, F1, T)
-    assert OTHER.n_fgrams <= 0.95 * table.info()["n_slots"]
+    assert OTHER.n_fgrams <= 0.85 * table.info()["n_slots"]
     # two calls in a row, each compared with a table built the ordinary way
     for fg_tok, fg_len, F in ((fg2_tok, fg2_len, F2), (fg1_tok, fg1_len, F1)):
         assert _rebuild_via_c_abi(table, fg_tok, fg_len, F) == scone.SCONE_OK
@@ -92,9 +92,9 @@ def test_rebuild_noalloc_clears_its_flags_and_rejects_oversize_lists():
     # the next call starts from cleared flags and succeeds
     assert _rebuild_via_c_abi(table, fg_tok, fg_len, F) == scone.SCONE_OK
     _same_as_fresh_build(table, fg_tok, fg_len, F, T, tok)
-    # more f-grams than 0.95 of the slots: refused before any device work
+    # more f-grams than 0.85 of the slots: refused before any device work
     n_slots = table.info()["n_slots"]
-    big = int(0.95 * n_slots) + 1
+    big = int(0.85 * n_slots) + 1
     big_tok = np.zeros((big, BASE.K), np.int32)
     big_len = np.full(big, 2, np.uint8)
     assert _rebuild_via_c_abi(table, big_tok, big_len, F) == scone.SCONE_ERR_INVALID_ARG
@@ -121,7 +121,7 @@ def test_rebuild_noalloc_scratch_limit():
     ft0, fl0 = _distinct_trigrams(100_000, vocab)
     F = dev_rows(np.arange(n_over * d, dtype=np.uint16).reshape(n_over, d))
     table = scone.scone_table_build(ft0, fl0, K, vocab, d, F[:100_000], T, load_factor=0.05)
-    assert n_over <= 0.95 * table.info()["n_slots"]     # only the scratch limit applies
+    assert n_over <= 0.85 * table.info()["n_slots"]     # only the scratch limit applies
     ft, fl = _distinct_trigrams(n_under, vocab)
     assert _rebuild_via_c_abi(table, ft, fl, F) == scone.SCONE_OK
     tok = ft[::997][:, :].reshape(-1)[None, :]          # windows that hit many f-grams
