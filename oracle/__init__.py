@@ -1,12 +1,14 @@
-"""CPU oracle for SCONE's inference-time input embedding (Algorithm 1).
+"""CPU oracles for SCONE's input embedding (Algorithm 1) and for the
+construction of its f-gram set (Algorithm 3).
 
 TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU
 baseline leg of ``bench.py`` may import this package. The product path
 (``paper_2502_01637_gb300``) never imports it and has no CPU fallback.
 
 The arithmetic lives in ``scone_oracle.cpp`` (plain C++: a ``std::map`` keyed
-by the exact token tuple, scanned as Algorithm 1 states); this file only
-marshals numpy arrays through ctypes. ``__graft_entry__.build()`` compiles
+by the exact token tuple, scanned as Algorithm 1 states) and
+``discover_oracle.cpp`` (every n-gram counted in a ``std::map``, sorted as
+Algorithm 3 states); this file only marshals numpy arrays through ctypes. ``__graft_entry__.build()`` compiles
 ``liboracle.so`` next to this file.
 """
 
@@ -31,6 +33,7 @@ _i32p = ctypes.POINTER(ctypes.c_int32)
 _i64p = ctypes.POINTER(ctypes.c_int64)
 _u8p = ctypes.POINTER(ctypes.c_uint8)
 _u16p = ctypes.POINTER(ctypes.c_uint16)
+_u32p = ctypes.POINTER(ctypes.c_uint32)
 
 
 def _load():
@@ -60,6 +63,13 @@ def _load():
                                   ctypes.c_int32, _i32p, _u16p, ctypes.c_int64, _u16p,
                                   ctypes.c_int32, _u16p, _i64p, _u8p]
     lib.oracle_decode.restype = ctypes.c_int
+    lib.oracle_discover.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                    ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, _i32p, _u8p,
+                                    _u32p, ctypes.c_int64, _i64p, _i64p, _i64p]
+    lib.oracle_discover.restype = ctypes.c_int
+    lib.oracle_count_ngrams.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                        _i32p, _u8p, ctypes.c_int64, _i64p, _i64p]
+    lib.oracle_count_ngrams.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -178,3 +188,51 @@ class Oracle:
         if rc not in (OK, ERR_TOKEN_RANGE):
             raise OracleError(rc, "oracle_decode")
         return out, row, ln, rc
+
+
+def discover(tok: np.ndarray, K: int, vocab: int, S: int, min_count: int = 1):
+    """Algorithm 3 on a [B, L] corpus: the S most frequent n-grams, n = 2..K,
+    among those appearing at least ``min_count`` times; ties by length, then
+    first occurrence. Listed by length, then first occurrence.
+
+    Returns a dict: ``tok`` [n, K] int32 padded with -1, ``len`` [n] uint8,
+    ``count`` [n] uint32, ``distinct`` and ``frequent`` ([K + 1] int64: per
+    length, the n-grams that appear and those reaching ``min_count``).
+    """
+    tok = np.ascontiguousarray(tok, dtype=np.int32)
+    B, L = tok.shape
+    cap = int(min(S, B * max(L - 1, 0) * (K - 1)))
+    out_tok = np.empty((max(cap, 1), K), np.int32)
+    out_len = np.empty(max(cap, 1), np.uint8)
+    out_cnt = np.empty(max(cap, 1), np.uint32)
+    n_out = ctypes.c_int64()
+    distinct = np.zeros(K + 1, np.int64)
+    frequent = np.zeros(K + 1, np.int64)
+    tp = _ptr(tok, _i32p) if tok.size else None
+    rc = _load().oracle_discover(tp, B, L, vocab, K, S, min_count, _ptr(out_tok, _i32p),
+                                 _ptr(out_len, _u8p), _ptr(out_cnt, _u32p), cap,
+                                 ctypes.byref(n_out), _ptr(distinct, _i64p),
+                                 _ptr(frequent, _i64p))
+    if rc != OK:
+        raise OracleError(rc, "oracle_discover")
+    n = n_out.value
+    return {"tok": out_tok[:n].copy(), "len": out_len[:n].copy(), "count": out_cnt[:n].copy(),
+            "distinct": distinct, "frequent": frequent}
+
+
+def count_ngrams(tok: np.ndarray, K: int, q_tok: np.ndarray, q_len: np.ndarray):
+    """Occurrences of each query n-gram in a [B, L] corpus, by direct window
+    comparison. Returns (count int64 [nq], first occurrence int64 [nq])."""
+    tok = np.ascontiguousarray(tok, dtype=np.int32)
+    B, L = tok.shape
+    q_tok = np.ascontiguousarray(q_tok, dtype=np.int32).reshape(-1, K)
+    q_len = np.ascontiguousarray(q_len, dtype=np.uint8).reshape(-1)
+    nq = q_len.shape[0]
+    counts = np.empty(max(nq, 1), np.int64)
+    first = np.empty(max(nq, 1), np.int64)
+    rc = _load().oracle_count_ngrams(_ptr(tok, _i32p), B, L, K, _ptr(q_tok, _i32p),
+                                     _ptr(q_len, _u8p), nq, _ptr(counts, _i64p),
+                                     _ptr(first, _i64p))
+    if rc != OK:
+        raise OracleError(rc, "oracle_count_ngrams")
+    return counts[:nq], first[:nq]

@@ -1,9 +1,12 @@
 """Mistakes planted in copies of the oracle must fail at least one pin.
 
-Each mutant is a plausible slip in the oracle's C++ (scan order, window
-bound, row or length off by one, token range, duplicate handling, gather
-source, decode history alignment). The copy is compiled on the CPU and the
-pin tests in test_oracle.py run against it in a subprocess; they must fail.
+Each mutant is a plausible slip in the oracle's C++: for Algorithm 1 (scan
+order, window bound, row or length off by one, token range, duplicate
+handling, gather source, decode history alignment) and for Algorithm 3
+(window bound, length range, first occurrence, threshold, sort direction, tie
+order, the top-S cut, sequence boundary). The copy is compiled on the CPU and
+the pin tests in test_oracle.py and test_discover_oracle.py run against it in
+a subprocess; they must fail.
 """
 
 import os
@@ -13,7 +16,10 @@ import sys
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-SRC = os.path.join(ROOT, "oracle", "scone_oracle.cpp")
+SRCS = {"alg1": os.path.join(ROOT, "oracle", "scone_oracle.cpp"),
+        "alg3": os.path.join(ROOT, "oracle", "discover_oracle.cpp")}
+PINS = [os.path.join(ROOT, "tests", "test_oracle.py"),
+        os.path.join(ROOT, "tests", "test_discover_oracle.py")]
 
 SCAN = """  for (int64_t jp = first; jp < i; ++jp) {
     const std::vector<int32_t> window(seq + jp, seq + i + 1);
@@ -40,49 +46,73 @@ GROW_UNTIL_MISS = """  int64_t best = -1;
   return best;"""
 
 MUTANTS = {
-    "shortest_first": ("for (int64_t jp = first; jp < i; ++jp) {",
+    # Algorithm 1
+    "shortest_first": ("alg1", "for (int64_t jp = first; jp < i; ++jp) {",
                        "for (int64_t jp = i - 1; jp >= first; --jp) {"),
-    "grow_until_miss": (SCAN, GROW_UNTIL_MISS),
-    "drop_longest_length": ("int64_t first = i - (t.K - 1);", "int64_t first = i - (t.K - 2);"),
-    "row_off_by_one": ("return it->second;", "return it->second + 1;"),
-    "len_off_by_one": ("*j_out = jp;", "*j_out = jp + 1;"),
-    "vocab_bound": ("return x >= 0 && x < t.vocab;", "return x >= 0 && x <= t.vocab;"),
-    "duplicates_accepted": ("      delete t;\n      return -3;", "      (void)0;"),
-    "fallback_wrong_token": ("T + (int64_t)seq[i] * d", "T + (int64_t)seq[i > 0 ? i - 1 : 0] * d"),
-    "fgram_row_shift": ("F + r * d", "F + (r > 0 ? r - 1 : r) * d"),
-    "decode_history_left_aligned": ("hist + s * hist_stride + (hist_stride - h)",
+    "grow_until_miss": ("alg1", SCAN, GROW_UNTIL_MISS),
+    "drop_longest_length": ("alg1", "int64_t first = i - (t.K - 1);", "int64_t first = i - (t.K - 2);"),
+    "row_off_by_one": ("alg1", "return it->second;", "return it->second + 1;"),
+    "len_off_by_one": ("alg1", "*j_out = jp;", "*j_out = jp + 1;"),
+    "vocab_bound": ("alg1", "return x >= 0 && x < t.vocab;", "return x >= 0 && x <= t.vocab;"),
+    "duplicates_accepted": ("alg1", "      delete t;\n      return -3;", "      (void)0;"),
+    "fallback_wrong_token": ("alg1", "T + (int64_t)seq[i] * d", "T + (int64_t)seq[i > 0 ? i - 1 : 0] * d"),
+    "fgram_row_shift": ("alg1", "F + r * d", "F + (r > 0 ? r - 1 : r) * d"),
+    "decode_history_left_aligned": ("alg1", "hist + s * hist_stride + (hist_stride - h)",
                                     "hist + s * hist_stride"),
+    # Algorithm 3
+    "d_last_window_dropped": ("alg3", "for (int64_t p = 0; p + n <= L; ++p)",
+                              "for (int64_t p = 0; p + n < L; ++p)"),
+    "d_longest_length_dropped": ("alg3", "for (int32_t n = 2; n <= K; ++n)",
+                                 "for (int32_t n = 2; n < K; ++n)"),
+    "d_last_occurrence": ("alg3", "if (e.count == 0) e.first = b * L + p;",
+                          "e.first = b * L + p;"),
+    "d_threshold_strict": ("alg3", "if (kv.second.count < min_count) continue;",
+                           "if (kv.second.count <= min_count) continue;"),
+    "d_least_frequent_first": ("alg3", "if (a.count != b.count) return a.count > b.count;",
+                               "if (a.count != b.count) return a.count < b.count;"),
+    "d_ties_longest_first": ("alg3", "if (a.gram.size() != b.gram.size()) return a.gram.size() < "
+                             "b.gram.size();\n    return a.first < b.first;\n  });\n  if",
+                             "if (a.gram.size() != b.gram.size()) return a.gram.size() > "
+                             "b.gram.size();\n    return a.first < b.first;\n  });\n  if"),
+    "d_cut_one_short": ("alg3", "all.resize((size_t)S);", "all.resize((size_t)(S > 0 ? S - 1 : 0));"),
+    "d_cross_sequences": ("alg3", "for (int64_t p = 0; p + n <= L; ++p) {\n        Entry& e = "
+                          "counts[std::vector<int32_t>(seq + p, seq + p + n)];",
+                          "for (int64_t p = 0; p + n <= L + (b + 1 < B ? n - 1 : 0); ++p) {\n"
+                          "        Entry& e = counts[std::vector<int32_t>(seq + p, seq + p + n)];"),
+    "d_vocab_bound": ("alg3", "if (tok[i] < 0 || tok[i] >= vocab) return -2;",
+                      "if (tok[i] < 0 || tok[i] > vocab) return -2;"),
 }
 
 
 def _run_pins(lib):
     env = dict(os.environ, SCONE_ORACLE_LIB=lib)
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
-                        os.path.join(ROOT, "tests", "test_oracle.py")],
-                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+                        *PINS], cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     return r.returncode, r.stdout[-2000:]
+
+
+def _compile(tmp_path, which=None, old=None, new=None):
+    cpps = []
+    for key, path in sorted(SRCS.items()):
+        src = open(path).read()
+        if key == which:
+            assert old in src, f"mutation site not found: {old[:60]}"
+            src = src.replace(old, new)
+        cpp = tmp_path / f"{key}.cpp"
+        cpp.write_text(src)
+        cpps.append(str(cpp))
+    lib = str(tmp_path / "liboracle_copy.so")
+    subprocess.run(["g++", "-O1", "-std=c++17", "-fPIC", "-shared", *cpps, "-o", lib], check=True)
+    return lib
 
 
 @pytest.mark.parametrize("name", sorted(MUTANTS))
 def test_mutant_is_caught(name, tmp_path):
-    old, new = MUTANTS[name]
-    src = open(SRC).read()
-    assert old in src, f"mutation site for {name} not found"
-    mutated = src.replace(old, new)
-    cpp = tmp_path / "mut.cpp"
-    cpp.write_text(mutated)
-    lib = str(tmp_path / "libmut.so")
-    subprocess.run(["g++", "-O1", "-std=c++17", "-fPIC", "-shared", str(cpp), "-o", lib],
-                   check=True)
-    rc, log = _run_pins(lib)
+    which, old, new = MUTANTS[name]
+    rc, log = _run_pins(_compile(tmp_path, which, old, new))
     assert rc != 0, f"mutant {name} passed every pin:\n{log}"
 
 
 def test_unmutated_copy_passes(tmp_path):
-    cpp = tmp_path / "same.cpp"
-    cpp.write_text(open(SRC).read())
-    lib = str(tmp_path / "libsame.so")
-    subprocess.run(["g++", "-O1", "-std=c++17", "-fPIC", "-shared", str(cpp), "-o", lib],
-                   check=True)
-    rc, log = _run_pins(lib)
+    rc, log = _run_pins(_compile(tmp_path))
     assert rc == 0, log
