@@ -139,12 +139,15 @@ def measured_peaks():
 
 
 def kernel_source_hash() -> str:
-    """Hash of the sources that compile into the fused prefill kernel."""
+    """Hash of the code (comments and whitespace removed) of the sources that
+    compile into the fused prefill kernel."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2502_01637_gb300", "csrc")
     files = [os.path.join(csrc, f) for f in ("scone_embed.cu", "scone_device.cuh", "scone_host.h")]
     for f in files:
-        h.update(open(f, "rb").read())
+        code = re.sub(r"/\*.*?\*/", " ", open(f).read(), flags=re.S)
+        code = re.sub(r"//[^\n]*", " ", code)
+        h.update(" ".join(code.split()).encode())
     return h.hexdigest()[:16]
 
 

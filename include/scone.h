@@ -13,8 +13,9 @@
  * F is stored as "a dense embedding matrix paired with a hash dictionary
  * that maps f-grams to matrix indices" (Sec. 2, "Efficient Indexing for
  * Large Embedding Layers"). Here the dictionary is a GPU bucketized cuckoo
- * hash table (two candidate buckets of two slots per key, both read in one
- * round trip) built once by scone_table_build; the dense matrix stays
+ * hash table (two candidate buckets of two slots per key; a lookup reads the
+ * second bucket only when the first is full without the key) built once by
+ * scone_table_build; the dense matrix stays
  * caller-owned in HBM or in host-pinned, device-mapped memory (the paper's
  * off-accelerator tier, Sec. 4.3).
  *
@@ -180,8 +181,10 @@ int scone_table_set_copy_mode(scone_table* table, int32_t mode);
  * scone_match — the selection step of Algorithm 1 (Sec. 3): for each
  * position, the length of the longest f-gram ending there and its row of F.
  * Probes lengths 2..min(K, i+1), i.e. at most K-1 lookups per token, the
- * bound Sec. 4.3 states ("up to four queries per token" for K = 5); each
- * lookup reads its two candidate buckets at once. Async.
+ * bound Sec. 4.3 states ("up to four queries per token" for K = 5). All
+ * lengths read their first buckets in one round trip; the lengths whose
+ * first bucket is full without the key, and that are longer than the best
+ * first-round hit, read their second buckets in a second one. Async.
  *
  *  tok  int32 [B * L]; row int32 [B * L] (F row, or -1 when T is used or on
  *  error); len uint8 [B * L] or NULL (n in 2..K for an f-gram, 1 for the

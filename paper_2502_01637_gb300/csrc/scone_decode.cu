@@ -5,8 +5,8 @@
 // keeps, per sequence, a device ring of its last K-1 tokens (right-aligned,
 // oldest first) and how many of them are known. One warp serves one
 // sequence: lane j looks up the window of length j + 2 ending at the new
-// token (both cuckoo buckets in one round trip), a warp ballot keeps the
-// longest hit,
+// token (its first cuckoo bucket, and the second only when the first is full
+// without the key), a warp ballot keeps the longest hit,
 // the lanes shift the new token into the history, and the warp copies the
 // selected row (F over the host link in the offloaded tier, or T from HBM)
 // with every lane's loads issued at once.

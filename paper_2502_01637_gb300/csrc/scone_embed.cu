@@ -5,10 +5,11 @@
 // at once, all SMs equally loaded) and the flattened [B x L] positions are
 // split evenly over all its warps, so every warp moves the same number of
 // rows (+-1). A warp walks its range in tiles of up to 32 positions: each
-// lane matches one position (all K-1 candidate lengths probed at once,
-// longest hit kept), the selected row addresses go to shared memory, and the
-// warp then streams the rows to the contiguous output block with 16-byte
-// loads and streaming (evict-first) stores.
+// lane matches one position (the first buckets of all K-1 candidate lengths
+// read at once, then the second buckets still needed; longest hit kept), the
+// selected row addresses go to shared memory, and the warp then streams the
+// rows to the contiguous output block with 16-byte loads and streaming
+// (evict-first) stores.
 //
 // Occupancy: the match of a tile is a chain of dependent loads during which
 // its warp moves no rows, so the kernel wants many resident warps; the copy
