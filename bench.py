@@ -37,6 +37,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "embedded tokens/s at 1 GB300; achieved GB/s vs HBM or host-link roofline"
+METRIC_DISCOVER = "corpus tokens/s of f-gram discovery (Algorithm 3, K-1 counting scans) at 1 GB300"
 
 
 def workload(name):
@@ -46,6 +47,11 @@ def workload(name):
         # the prefill law at a size an ncu capture handles (about 1.5 GB on the device)
         return synth.WORKLOADS["prefill_1b"].scaled("prefill_profile", B=16,
                                                     quotas=((2, 120000), (3, 80000)))
+    if name == "discover_profile":
+        # the discover law at a size a full-section ncu capture handles: 2^24
+        # corpus tokens (a 0.5 GB counting table, larger than L2)
+        return synth.WORKLOADS["discover"].scaled("discover_profile", B=8192,
+                                                  quotas=((2, 150_000), (3, 100_000)))
     if name == "decode_profile":
         # the offloaded-decode law with 2e6 f-grams (8 GB of host rows) for ncu captures
         return synth.WORKLOADS["offload_decode"].scaled(
@@ -643,6 +649,149 @@ def bench_prescan(args, world, rank, local):
     return res
 
 
+# ---------------------------------------------------------- f-gram discovery
+def bench_discover(args, world, rank, local):
+    """Algorithm 3 by K-1 counting scans over a corpus resident in HBM: one
+    step is one whole scone_fgram_discover call (counting scans, selection,
+    list emission)."""
+    import torch
+
+    import synth
+    import paper_2502_01637_gb300 as scone
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = workload(args.workload)
+    n = w.B * w.L
+    S = w.n_fgrams
+    t0 = time.time()
+    tok_np = synth.query_tokens(w)
+    host_tok = torch.from_numpy(tok_np).pin_memory()
+    tok = host_tok.to(dev)
+    out_tok = torch.empty((S, w.K), dtype=torch.int32, device=dev)
+    out_len = torch.empty(S, dtype=torch.uint8, device=dev)
+    out_cnt = torch.empty(S, dtype=torch.int32, device=dev)
+    ws = scone.scone_discover_create()
+    setup_s = time.time() - t0
+    stream = torch.cuda.current_stream()
+
+    def step(src):
+        return scone.scone_fgram_discover(src, w.vocab, w.K, S, w.min_count, out_tok, out_len,
+                                          out_cnt, workspace=ws)
+
+    for _ in range(args.warmup):
+        step(tok)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    stats = []
+    clocks = ClockSampler(local)
+    barrier(world)
+    with clocks:
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            stats.append(step(tok)[3])
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms = max_over_ranks(statistics.mean(a.elapsed_time(b) for a, b in ev), world)
+    st = stats[-1]
+
+    # end to end: corpus from pinned host memory, the call, the list back to the host
+    host_out = [torch.empty_like(t, device="cpu").pin_memory() for t in (out_tok, out_len, out_cnt)]
+    e2e_t = []
+    for k in range(max(2, min(args.steps, 5))):
+        torch.cuda.synchronize()
+        t1 = time.perf_counter()
+        tok.copy_(host_tok, non_blocking=True)
+        ft, fl, fc, _ = step(tok)
+        m = fl.shape[0]
+        for h, d in zip(host_out, (ft, fl, fc)):
+            h[:m].copy_(d, non_blocking=True)
+        torch.cuda.synchronize()
+        e2e_t.append(time.perf_counter() - t1)
+    e2e_ms = max_over_ranks(1e3 * statistics.mean(e2e_t), world)
+    m = int(st["frequent"][2] + sum(st["frequent"][3:]))
+    n_sel = min(S, m)
+
+    # roofline of the dominant kernel: the counting kernel of scan 2 (every window)
+    ms_count = statistics.mean(s_["ms_count"][2] for s_ in stats)
+    flushes = st["flushes"][2]
+    bytes_count = 8 * n + 64 * flushes
+    hbm, peak_src = measured_peaks()
+    achieved = bytes_count / (ms_count * 1e-3) / 1e9
+    res = {
+        "metric": METRIC_DISCOVER,
+        "value": world * n / (ms * 1e-3),
+        "unit": "corpus tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int32",
+        "data": "synthetic corpus (seeded Zipf(1.1) sequences over 1e5 token ids)",
+        "config": {"workload": (f"{w.name}: f-grams of length 2..{w.K} with count >= "
+                                f"{w.min_count}, the {S} most frequent, from {w.B} x {w.L} = "
+                                f"{n} corpus tokens in HBM"),
+                   "l2": "corpus (4.3 GB) and counting table far larger than L2; no flush",
+                   "timing": "CUDA events around each whole scone_fgram_discover call"},
+        "roofline": {
+            "bound": "hbm",
+            "achieved": achieved,
+            "peak": hbm,
+            "unit": "GB/s",
+            "frac": achieved / hbm,
+            "traffic": None,
+            "peak_source": peak_src,
+            "algorithmic_bytes_per_launch": bytes_count,
+            "kernel": "count_kernel of scan 2 (8 B per window + 64 B per global table update)",
+            "kernel_ms": ms_count,
+            "kernel_share_of_step": ms_count / ms,
+        },
+        "e2e": {"value": world * n / (e2e_ms * 1e-3), "unit": "corpus tokens/s",
+                "h2d_bytes_per_step": 4 * n,
+                "d2h_bytes_per_step": n_sel * (4 * w.K + 1 + 4),
+                "what": "pinned corpus -> device, scone_fgram_discover, f-gram list -> "
+                        "pinned host"},
+        # per call: count, flag, scan, assign per scan and next_id between scans;
+        # then 4 radix-select histograms (only when the cut falls inside the
+        # list), select_count, two scans and emit
+        "gpu_launches": args.steps * (5 * (w.K - 1) - 1 + (8 if S < m else 4)),
+        "clocks": clocks.summary(),
+        "discover": {k: st[k] for k in ("candidates", "distinct", "frequent", "flushes",
+                                         "threshold", "selected_at_threshold",
+                                         "table_bytes_max", "ms_count", "ms_scan",
+                                         "ms_select", "ms_total", "ms_alloc_host",
+                                         "workspace_bytes")},
+        "setup_s": setup_s,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        res["cpu_baseline"] = cpu_baseline_discover(w, tok_np)
+    ws.close()
+    return res
+
+
+def cpu_baseline_discover(w, tok, budget_s: float = 10.0):
+    """The discovery oracle (single thread, std::map of every n-gram) on a
+    bounded prefix of the same corpus, grown until it takes about budget_s."""
+    import oracle
+
+    seqs = 64
+    while True:
+        t0 = time.perf_counter()
+        oracle.discover(tok[:seqs], w.K, w.vocab, w.n_fgrams, w.min_count)
+        dt = time.perf_counter() - t0
+        if dt >= budget_s / 3 or seqs >= tok.shape[0]:
+            break
+        seqs *= 2
+    return {"value": seqs * w.L / dt, "unit": "corpus tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"oracle discovery over the first {seqs} x {w.L} tokens of the corpus "
+                      f"({dt:.1f} s)"}
+
+
 # ----------------------------------------------------------- reference arm
 def bench_reference(args, world, rank):
     """The CPU oracle on the host cores, same workload and metric."""
@@ -687,7 +836,8 @@ def main():
     ap.add_argument("--impl", default="scone", choices=["scone", "reference"])
     ap.add_argument("--workload", default="prefill_1b",
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
-                             "offload_decode", "decode_profile", "prescan"])
+                             "offload_decode", "decode_profile", "prescan", "discover",
+                             "discover_k5", "discover_profile"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
@@ -707,6 +857,8 @@ def main():
         res = bench_decode(args, world, rank, local)
     elif args.workload == "prescan":
         res = bench_prescan(args, world, rank, local)
+    elif args.workload in ("discover", "discover_k5", "discover_profile"):
+        res = bench_discover(args, world, rank, local)
     else:
         res = bench_prefill(args, world, rank, local)
     if rank == 0:

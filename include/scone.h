@@ -49,6 +49,7 @@ extern "C" {
 
 typedef struct scone_table scone_table;   /* opaque; owns its slot array and status word */
 typedef struct scone_decode scone_decode; /* opaque; owns the device history ring */
+typedef struct scone_discover scone_discover; /* opaque; reusable workspace of f-gram discovery */
 typedef uint16_t scone_bf16;              /* raw bf16 bits */
 
 enum scone_err {
@@ -197,6 +198,71 @@ int scone_table_set_copy_mode(scone_table* table, int32_t mode);
  */
 int scone_match(const scone_table* table, const int32_t* tok, int32_t B, int32_t L,
                 int32_t* row, uint8_t* len, void* stream);
+
+/*
+ * scone_fgram_discover — constructs V_fgram from a corpus: Algorithm 3
+ * ("Constructing a set of f-grams", Appendix A) by the K-1 counting scans of
+ * Sec. 3.2. C_w is the number of windows equal to the n-gram w, n = 2..K,
+ * over every sequence of the dense [B x L] corpus (windows never span two
+ * sequences; overlapping windows count separately). Only n-grams with
+ * C_w >= min_count are eligible (Sec. 3.2 uses 5; 1 gives Algorithm 3
+ * exactly). The S eligible n-grams with the largest C_w are returned; ties
+ * go to the shorter n-gram, then to the earlier first occurrence (start
+ * position in the flattened corpus). The list is ordered by length, then by
+ * first occurrence, so it can be passed to scone_table_build as is (f-gram
+ * r gets row r). If fewer than S n-grams are eligible, all are returned.
+ *
+ *  ws           a workspace from scone_discover_create, or NULL. The call's
+ *               device buffers are taken from it and stay allocated there
+ *               (grown as needed, never shrunk) until scone_discover_destroy,
+ *               so repeated calls allocate nothing; with NULL they are
+ *               allocated and freed inside the call.
+ *  tok          int32 [B * L], device-accessible (device memory, or host
+ *               memory from scone_host_alloc read over the host link);
+ *               every token in [0, vocab). B * L <= 2^30.
+ *  fgram_tok    int32 [S * K], padded with -1 after each n-gram's tokens;
+ *  fgram_len    uint8 [S]; fgram_count uint32 [S] or NULL. Device-accessible
+ *               (device or host-mapped); entries past *n_out are untouched.
+ *  n_out        host; receives the number of f-grams written (<= S).
+ *  stats        host or NULL; per length n (index n): windows counted after
+ *               pruning, distinct n-grams among them, eligible n-grams,
+ *               global table updates and the counting kernel's device time;
+ *               the count of the S-th f-gram and how many f-grams at that
+ *               count were taken; the largest counting table allocated; the
+ *               device time of the call.
+ *
+ * Synchronous: returns when the lists are written. Working memory: about
+ * 9 bytes per token, a counting table of 32 bytes per counted window at the
+ * largest scan, and the lists of eligible n-grams (4 (n + 1) bytes each). Errors: SCONE_ERR_INVALID_ARG (K outside [2, 8], min_count < 1,
+ * S < 0, null pointers), SCONE_ERR_UNSUPPORTED (B * L > 2^30),
+ * SCONE_ERR_TOKEN_RANGE (a token outside [0, vocab); nothing is written),
+ * SCONE_ERR_NOMEM, SCONE_ERR_CUDA.
+ */
+typedef struct scone_discover_stats {
+  int64_t candidates[9];      /* windows counted in scan n (after pruning for n >= 3) */
+  int64_t distinct[9];        /* distinct n-grams among them */
+  int64_t frequent[9];        /* n-grams with count >= min_count */
+  int64_t flushes[9];         /* global table updates of scan n (distinct keys per chunk) */
+  int64_t threshold;          /* count of the last-ranked selected f-gram; 0 when all taken */
+  int64_t selected_at_threshold; /* f-grams taken at that count (0 when all taken) */
+  int64_t table_bytes_max;    /* largest counting table of a scan */
+  double ms_count[9];         /* device time of scan n's counting kernel (CUDA events) */
+  double ms_scan[9];          /* device time of the whole scan n */
+  double ms_select;           /* device time of the selection and the emission */
+  double ms_total;            /* device time of the whole call, first launch to last */
+  double ms_alloc_host;       /* host time spent in the call's allocations */
+  int64_t workspace_bytes;    /* device bytes held by the workspace after the call */
+} scone_discover_stats;
+
+int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int32_t B, int32_t L,
+                         int32_t vocab, int32_t K, int64_t S, int32_t min_count,
+                         int32_t* fgram_tok, uint8_t* fgram_len, uint32_t* fgram_count,
+                         int64_t* n_out, scone_discover_stats* stats, void* stream);
+
+/* An empty discovery workspace on the current device (no device memory yet). */
+int scone_discover_create(scone_discover** out);
+/* Frees the workspace and its device buffers (NULL is a no-op). */
+int scone_discover_destroy(scone_discover* ws);
 
 /*
  * scone_embed_gather — the emission step of Algorithm 1 (Sec. 3): for each

@@ -68,7 +68,8 @@ def _load():
                                     _u32p, ctypes.c_int64, _i64p, _i64p, _i64p]
     lib.oracle_discover.restype = ctypes.c_int
     lib.oracle_count_ngrams.argtypes = [_i32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
-                                        _i32p, _u8p, ctypes.c_int64, _i64p, _i64p]
+                                        _i32p, _u8p, ctypes.c_int64, _i64p, _i64p,
+                                        ctypes.c_int32]
     lib.oracle_count_ngrams.restype = ctypes.c_int
     _lib = lib
     return lib
@@ -220,9 +221,10 @@ def discover(tok: np.ndarray, K: int, vocab: int, S: int, min_count: int = 1):
             "distinct": distinct, "frequent": frequent}
 
 
-def count_ngrams(tok: np.ndarray, K: int, q_tok: np.ndarray, q_len: np.ndarray):
-    """Occurrences of each query n-gram in a [B, L] corpus, by direct window
-    comparison. Returns (count int64 [nq], first occurrence int64 [nq])."""
+def count_ngrams(tok: np.ndarray, K: int, q_tok: np.ndarray, q_len: np.ndarray, threads: int = 0):
+    """Occurrences of each (distinct) query n-gram in a [B, L] corpus: every
+    window is looked up in a map of the queries. Returns (count int64 [nq],
+    first occurrence int64 [nq]); threads = 0 uses every core."""
     tok = np.ascontiguousarray(tok, dtype=np.int32)
     B, L = tok.shape
     q_tok = np.ascontiguousarray(q_tok, dtype=np.int32).reshape(-1, K)
@@ -232,7 +234,7 @@ def count_ngrams(tok: np.ndarray, K: int, q_tok: np.ndarray, q_len: np.ndarray):
     first = np.empty(max(nq, 1), np.int64)
     rc = _load().oracle_count_ngrams(_ptr(tok, _i32p), B, L, K, _ptr(q_tok, _i32p),
                                      _ptr(q_len, _u8p), nq, _ptr(counts, _i64p),
-                                     _ptr(first, _i64p))
+                                     _ptr(first, _i64p), threads)
     if rc != OK:
         raise OracleError(rc, "oracle_count_ngrams")
     return counts[:nq], first[:nq]

@@ -38,6 +38,8 @@
 #include <algorithm>
 #include <cstdint>
 #include <map>
+#include <thread>
+#include <unordered_map>
 #include <vector>
 
 namespace {
@@ -51,6 +53,26 @@ struct Ranked {
   std::vector<int32_t> gram;
   int64_t count;
   int64_t first;
+};
+
+// An n-gram as a fixed-size tuple (tokens past n are zero), for the query map.
+struct Gram {
+  int32_t t[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  int32_t n = 0;
+  bool operator==(const Gram& o) const {
+    if (n != o.n) return false;
+    for (int j = 0; j < n; ++j)
+      if (t[j] != o.t[j]) return false;
+    return true;
+  }
+};
+
+struct GramHash {
+  size_t operator()(const Gram& g) const {  // FNV-1a over the tokens and the length
+    uint64_t h = 1469598103934665603ull;
+    for (int j = 0; j < g.n; ++j) h = (h ^ (uint32_t)g.t[j]) * 1099511628211ull;
+    return (size_t)((h ^ (uint64_t)g.n) * 1099511628211ull);
+  }
 };
 
 }  // namespace
@@ -116,36 +138,55 @@ extern "C" int oracle_discover(const int32_t* tok, int32_t B, int32_t L, int32_t
   return 0;
 }
 
-// Occurrences of given n-grams in a corpus, by direct comparison of every
-// window with each query of the same last token. Used at sizes where the full
-// count map above would not fit the time of a test: q_tok [nq*K] padded,
-// q_len [nq] in [2, K]; counts[nq] receives the number of windows equal to
-// each query, first[nq] the start of its first occurrence (or -1).
+// Occurrences of given n-grams in a corpus: every window of length 2..K is
+// looked up in a hash map of the queries (exact token tuples). Used at sizes
+// where the full count map above would not fit the time of a test; the
+// corpus is split over `threads` threads by sequence, each with its own
+// tallies, summed at the end. q_tok [nq*K] padded, q_len [nq] in [2, K];
+// counts[nq] receives the number of windows equal to each query, first[nq]
+// the start of its first occurrence in the flattened corpus (or -1).
 extern "C" int oracle_count_ngrams(const int32_t* tok, int32_t B, int32_t L, int32_t K,
                                    const int32_t* q_tok, const uint8_t* q_len, int64_t nq,
-                                   int64_t* counts, int64_t* first) {
+                                   int64_t* counts, int64_t* first, int32_t threads) {
   if (B < 0 || L < 0 || K < 2 || K > 8 || nq < 0 || !counts || !first) return -1;
-  std::map<int32_t, std::vector<int64_t>> by_last;
+  std::unordered_map<Gram, int64_t, GramHash> index;
   for (int64_t q = 0; q < nq; ++q) {
     if (q_len[q] < 2 || q_len[q] > K) return -1;
-    by_last[q_tok[q * K + q_len[q] - 1]].push_back(q);
+    Gram g;
+    g.n = q_len[q];
+    for (int j = 0; j < g.n; ++j) g.t[j] = q_tok[q * K + j];
+    if (!index.emplace(g, q).second) return -1;   // the same query twice
+  }
+  if (threads < 1) threads = (int32_t)std::max(1u, std::thread::hardware_concurrency());
+  std::vector<std::vector<int64_t>> c((size_t)threads, std::vector<int64_t>((size_t)nq, 0));
+  std::vector<std::vector<int64_t>> f((size_t)threads, std::vector<int64_t>((size_t)nq, -1));
+  auto work = [&](int w) {
+    for (int64_t b = w; b < B; b += threads) {
+      const int32_t* seq = tok + b * L;
+      for (int64_t i = 0; i < L; ++i) {
+        Gram g;
+        for (int n = 2; n <= K && n <= i + 1; ++n) {
+          g.n = n;
+          for (int j = 0; j < n; ++j) g.t[j] = seq[i - n + 1 + j];
+          const auto it = index.find(g);
+          if (it == index.end()) continue;
+          const int64_t q = it->second;
+          const int64_t start = b * L + i - n + 1;
+          if (c[w][q] == 0 || start < f[w][q]) f[w][q] = start;
+          c[w][q] += 1;
+        }
+      }
+    }
+  };
+  std::vector<std::thread> pool;
+  for (int w = 0; w < threads; ++w) pool.emplace_back(work, w);
+  for (auto& t : pool) t.join();
+  for (int64_t q = 0; q < nq; ++q) {
     counts[q] = 0;
     first[q] = -1;
-  }
-  for (int64_t b = 0; b < B; ++b) {
-    const int32_t* seq = tok + b * L;
-    for (int64_t i = 0; i < L; ++i) {
-      const auto it = by_last.find(seq[i]);
-      if (it == by_last.end()) continue;
-      for (const int64_t q : it->second) {
-        const int n = q_len[q];
-        if (i + 1 < n) continue;
-        bool eq = true;
-        for (int j = 0; j < n && eq; ++j) eq = seq[i - n + 1 + j] == q_tok[q * K + j];
-        if (!eq) continue;
-        if (counts[q] == 0) first[q] = b * L + i - n + 1;
-        counts[q] += 1;
-      }
+    for (int w = 0; w < threads; ++w) {
+      counts[q] += c[w][q];
+      if (f[w][q] >= 0 && (first[q] < 0 || f[w][q] < first[q])) first[q] = f[w][q];
     }
   }
   return 0;

@@ -42,6 +42,7 @@ EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noal
            "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
+           "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
            "scone_strerror", "scone_version")
 
 _lib = None
@@ -65,6 +66,22 @@ class scone_table_info(ctypes.Structure):
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}
+
+
+class scone_discover_stats(ctypes.Structure):
+    _fields_ = [("candidates", _i64 * 9), ("distinct", _i64 * 9), ("frequent", _i64 * 9),
+                ("flushes", _i64 * 9), ("threshold", _i64), ("selected_at_threshold", _i64),
+                ("table_bytes_max", _i64), ("ms_count", ctypes.c_double * 9),
+                ("ms_scan", ctypes.c_double * 9), ("ms_select", ctypes.c_double),
+                ("ms_total", ctypes.c_double), ("ms_alloc_host", ctypes.c_double),
+                ("workspace_bytes", _i64)]
+
+    def as_dict(self):
+        out = {}
+        for k, _ in self._fields_:
+            v = getattr(self, k)
+            out[k] = list(v) if not isinstance(v, (int, float)) else v
+        return out
 
 
 def load_library():
@@ -93,6 +110,11 @@ def load_library():
     lib.scone_status.argtypes = [_vp, _vp]
     lib.scone_host_alloc.argtypes = [_i64, ctypes.POINTER(_vp)]
     lib.scone_host_free.argtypes = [_vp]
+    lib.scone_fgram_discover.argtypes = [_vp, _vp, _i32, _i32, _i32, _i32, _i64, _i32, _vp, _vp,
+                                         _vp, ctypes.POINTER(_i64),
+                                         ctypes.POINTER(scone_discover_stats), _vp]
+    lib.scone_discover_create.argtypes = [ctypes.POINTER(_vp)]
+    lib.scone_discover_destroy.argtypes = [_vp]
     lib.scone_strerror.argtypes = [ctypes.c_int]
     lib.scone_strerror.restype = ctypes.c_char_p
     lib.scone_version.argtypes = []
@@ -192,7 +214,7 @@ def scone_table_rebuild_noalloc(table: Table, fgram_tok: np.ndarray, fgram_len: 
     allocating: for callers that may not call cudaMalloc at that point (device
     memory owned by another allocator, or threads that must not pay for
     allocation and the device-wide synchronization cudaFree can cause). The
-    list must fit the table (at most 0.95 of its slots) and the library's
+    list must fit the table (at most 0.85 of its slots) and the library's
     fixed device scratch (SCONE_REBUILD_SCRATCH_BYTES); calls that overlap on
     the GPU race on that scratch. Synchronizes the stream.
     """
@@ -343,6 +365,76 @@ def scone_host_alloc(nbytes: int) -> HostBuffer:
 
 def scone_host_free(buf: HostBuffer) -> None:
     buf.free()
+
+
+class DiscoverWorkspace:
+    """Reusable device buffers of scone_fgram_discover (freed by close)."""
+
+    def __init__(self):
+        h = _vp()
+        _check(load_library().scone_discover_create(ctypes.byref(h)), "scone_discover_create")
+        self._h = h
+
+    @property
+    def handle(self):
+        if self._h is None:
+            raise RuntimeError("workspace was closed")
+        return self._h
+
+    def close(self):
+        if self._h is not None:
+            load_library().scone_discover_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def scone_discover_create() -> DiscoverWorkspace:
+    return DiscoverWorkspace()
+
+
+def scone_discover_destroy(ws: DiscoverWorkspace) -> None:
+    ws.close()
+
+
+def scone_fgram_discover(tok, vocab: int, K: int, S: int, min_count: int = 5,
+                         fgram_tok=None, fgram_len=None, fgram_count=None,
+                         workspace: Optional[DiscoverWorkspace] = None, stream=None):
+    """Algorithm 3 by the K-1 counting scans of Sec. 3.2 over a corpus tok
+    [B, L] int32 (device tensor, or a HostBuffer address with shape given as
+    a (ptr, B, L) tuple). Returns (fgram_tok [n, K] int32, fgram_len [n] uint8,
+    fgram_count [n] int32, stats dict); the outputs are device tensors
+    (allocated here unless given, each with room for S f-grams). With a
+    workspace, repeated calls reuse its device buffers."""
+    import torch
+
+    if isinstance(tok, tuple):
+        ptr, B, L = tok
+        dev = torch.device("cuda", torch.cuda.current_device())
+    else:
+        B, L = _bl(tok)
+        ptr = _ptr(tok)
+        dev = tok.device
+    if fgram_tok is None:
+        fgram_tok = torch.empty((max(S, 1), K), dtype=torch.int32, device=dev)
+    if fgram_len is None:
+        fgram_len = torch.empty(max(S, 1), dtype=torch.uint8, device=dev)
+    if fgram_count is None:
+        fgram_count = torch.empty(max(S, 1), dtype=torch.int32, device=dev)
+    n_out = _i64()
+    st = scone_discover_stats()
+    ws = workspace.handle if workspace is not None else None
+    _check(load_library().scone_fgram_discover(ws, ptr, B, L, vocab, K, S, min_count,
+                                               _ptr(fgram_tok), _ptr(fgram_len),
+                                               _ptr(fgram_count), ctypes.byref(n_out),
+                                               ctypes.byref(st), _stream(stream)),
+           "scone_fgram_discover")
+    n = n_out.value
+    return fgram_tok[:n], fgram_len[:n], fgram_count[:n], st.as_dict()
 
 
 def scone_strerror(code: int) -> str:

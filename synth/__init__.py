@@ -17,6 +17,8 @@ large_hbm          1e5    1.1   64x4096 1e7 (60/40)  3    2048  device
 offload_decode     1e5    1.1   512 seq x 256 steps  2e7  3     2048  host-mapped
 stress_k5          1e5    1.05  16x8192 5e6 n=2..5   5    1536  device
 prescan            1e5    1.1   2^19x2048 1e7 (60/40) 3   8     (tokens in host memory)
+discover           1e5    1.1   2^19x2048 S = 1e7    3   -     (corpus in HBM)
+discover_k5        1e5    1.05  2^17x2048 S = 5e6    5   -     (corpus in HBM)
 =================  =====  ====  ======  ===========  ===  ====  ==============
 
 f-gram sets are the first distinct n-grams of a separate Zipf source stream of
@@ -108,6 +110,7 @@ class Workload:
     dec_S: int = 0                       # decode: live sequences
     dec_hist: int = 0                    # decode: history tokens per sequence
     dec_steps: int = 0                   # decode: steps
+    min_count: int = 5                   # f-gram discovery: eligibility threshold (Sec. 3.2)
 
     @property
     def n_fgrams(self) -> int:
@@ -148,6 +151,15 @@ WORKLOADS: Dict[str, Workload] = {
     # 2^19 training sequences of 2048 tokens (1.07e9 tokens) in host memory
     "prescan": Workload("prescan", 6, 100000, 1.1, 1 << 19, 2048,
                         _split(10_000_000, {2: 0.6, 3: 0.4}), 3, 8, location="host_mapped"),
+    # f-gram discovery (Algorithm 3 by K-1 scans): the 1e7 most frequent 2..3-grams
+    # (count >= 5) of a 1.07e9-token corpus (2^19 sequences of 2048) held in HBM;
+    # the quotas give S and its split is not used
+    "discover": Workload("discover", 7, 100000, 1.1, 1 << 19, 2048,
+                         _split(10_000_000, {2: 0.6, 3: 0.4}), 3, 8),
+    # the same with K = 5 over the stress law (phrases injected, so 4- and 5-grams recur)
+    "discover_k5": Workload("discover_k5", 8, 100000, 1.05, 1 << 17, 2048,
+                            _split(5_000_000, {2: 0.5, 3: 0.5}), 5, 8,
+                            inject_p=0.05 / 6, n_phrases=4096),
 }
 
 

@@ -6,7 +6,7 @@ algorithm by brute force over tiny vocabularies (every n-gram of the
 vocabulary counted against every window), closed forms (a repeated token, an
 alternating pair, all-distinct tokens, the sequence boundary), and invariants
 on seeded Zipf corpora (window totals, counts never grow with length, the
-top-S cut, the direct-comparison counter agreeing with the map).
+top-S cut, the query-map counter agreeing with the full count map).
 """
 
 import itertools
@@ -153,7 +153,7 @@ def test_invariants_zipf(K, mc):
     chosen = set(as_list(top))
     rest = [count[g] for g in count if g not in chosen and count[g] >= mc]
     assert min(top["count"]) >= max(rest)
-    # the direct-comparison counter agrees with the map, first occurrences included
+    # the query-map counter agrees with the full count map, first occurrences included
     sample = np.random.default_rng(K).choice(len(grams), 200, replace=False)
     q_tok = full["tok"][sample]
     q_len = full["len"][sample]
@@ -169,7 +169,9 @@ def test_count_ngrams_brute():
     rng = np.random.default_rng(7)
     tok = rng.integers(0, 3, size=(3, 7)).astype(np.int32)
     counts = alg3_counts(tok.tolist(), 3, 4)
-    grams = list(counts) + [(2, 2, 2, 2), (0, 1)]          # some may not appear
+    absent = [g for g in [(2, 2, 2, 2), (0, 1, 0, 1), (1, 1)] if g not in counts]
+    assert absent
+    grams = list(counts) + absent
     q_tok = np.full((len(grams), 4), -1, np.int32)
     q_len = np.array([len(g) for g in grams], np.uint8)
     for i, g in enumerate(grams):

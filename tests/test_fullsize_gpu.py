@@ -177,3 +177,62 @@ def test_prescan_host_mapped_corpus():
     table.close()
     for b in (corpus, tags_len, tags_row):
         b.free()
+
+
+def pack(tok_rows: np.ndarray, lens: np.ndarray) -> np.ndarray:
+    """n-grams of tokens < 2^20 (K <= 3) as int64 keys, for membership tests."""
+    key = lens.astype(np.int64) << 60
+    for j in range(tok_rows.shape[1]):
+        t = np.where(j < lens, tok_rows[:, j], 0).astype(np.int64)
+        key |= t << (40 - 20 * j)
+    return key
+
+
+def test_fullsize_discover():
+    """Algorithm 3 on the 1.07e9-token corpus (K = 3, S = 1e7, count >= 5),
+    as the benchmark runs it. Sampled f-grams: counts and first occurrences
+    from the oracle's counter; list order; the cut at the threshold. Sampled
+    corpus windows: every n-gram above the threshold is selected, none below
+    it is."""
+    w = synth.WORKLOADS["discover"]
+    S = w.n_fgrams
+    tok = synth.query_tokens(w)
+    tok_d = torch.from_numpy(tok).to(DEV)
+    ft, fl, fc, st = scone.scone_fgram_discover(tok_d, w.vocab, w.K, S, w.min_count)
+    n = fl.shape[0]
+    assert n == S and sum(st["frequent"]) > S           # the cut falls inside the list
+    ft, fl, fc = ft.cpu().numpy(), fl.cpu().numpy(), fc.cpu().numpy().astype(np.int64)
+    del tok_d
+    c_star, at_star = st["threshold"], st["selected_at_threshold"]
+    assert (fc >= c_star).all() and (fc >= w.min_count).all()
+    assert (fc == c_star).sum() == at_star and (fc > c_star).sum() == S - at_star
+    assert np.all(np.diff(fl.astype(np.int64)) >= 0)   # by length
+    keys = pack(ft, fl)
+    assert np.unique(keys).size == n                   # no n-gram twice
+    rng = np.random.default_rng(23)
+    # sampled f-grams: exact counts, and first occurrences ascending within a length
+    idx = np.sort(rng.choice(n, 3000, replace=False))
+    cnt, first = oracle.count_ngrams(tok, w.K, ft[idx], fl[idx])
+    assert np.array_equal(cnt, fc[idx]), "counts differ from the oracle's"
+    for L_ in (2, 3):
+        f = first[fl[idx] == L_]
+        assert np.all(np.diff(f) > 0), "not in first-occurrence order"
+    # sampled windows: selected iff above the threshold (ties at c* may go either way)
+    pos = rng.choice(tok.size, 20000, replace=False)
+    flat = tok.reshape(-1)
+    q = {}
+    for p in pos:
+        i = p % w.L
+        for m in range(2, w.K + 1):
+            if i + 1 >= m:
+                q.setdefault(tuple(int(x) for x in flat[p - m + 1:p + 1]), None)
+    grams = list(q)
+    q_tok = np.full((len(grams), w.K), -1, np.int32)
+    q_len = np.array([len(g) for g in grams], np.uint8)
+    for k, g in enumerate(grams):
+        q_tok[k, :len(g)] = g
+    qc, _ = oracle.count_ngrams(tok, w.K, q_tok, q_len)
+    chosen = np.isin(pack(q_tok, q_len), keys)
+    assert chosen[qc > c_star].all(), "an n-gram above the threshold is missing"
+    assert not chosen[(qc < c_star) | (qc < w.min_count)].any(), "an n-gram below it is selected"
+    assert chosen.any() and (~chosen).any()
