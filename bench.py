@@ -649,6 +649,156 @@ def bench_prescan(args, world, rank, local):
     return res
 
 
+# ------------------------------------------------------ mixed serving batch
+def mixed_batch(w, k, n_prefill_seq=48, n_decode=512):
+    """Batch k of a serving step over the prefill_1b law: n_prefill_seq prompt
+    chunks of seeded ragged lengths and n_decode one-token decode chunks, the
+    same 65,536 tokens as a prefill_1b batch. Returns (tokens, cu_seqlens,
+    slot of each sequence)."""
+    import synth
+
+    n_tok = w.B * w.L
+    rng = np.random.default_rng(1000 + k)
+    raw = rng.uniform(0.25, 1.75, n_prefill_seq)
+    lens = np.floor(raw / raw.sum() * (n_tok - n_decode)).astype(np.int64)
+    lens[0] += n_tok - n_decode - lens.sum()
+    lens = np.concatenate([lens, np.ones(n_decode, np.int64)])
+    order = rng.permutation(lens.size)               # prefill and decode chunks interleaved
+    lens = lens[order]
+    tok = synth.query_tokens(w.scaled(w.name + "_mixed", B=1, L=n_tok), range(k, k + 1))[0]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    slots = rng.permutation(2048)[:lens.size].astype(np.int32)
+    return tok, cu, slots
+
+
+def bench_mixed(args, world, rank, local):
+    """scone_embed_varlen on mixed serving batches: chunked-prefill pieces and
+    decode tokens of 560 sequences in one launch, continuing 2048 slots of a
+    decode state (the prefill_1b table, F and T)."""
+    import torch
+
+    import synth
+    import paper_2502_01637_gb300 as scone
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = synth.WORKLOADS["prefill_1b"]
+    n_tok = w.B * w.L
+    t0 = time.time()
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    stream = torch.cuda.current_stream()
+    F = torch.empty((w.n_fgrams, w.d), dtype=torch.int16, device=dev)
+    T = torch.empty((w.vocab, w.d), dtype=torch.int16, device=dev)
+    synth.rows_gpu(synth.F_seed(w), w.d, 0, w.n_fgrams, F.data_ptr(), stream.cuda_stream)
+    synth.rows_gpu(synth.T_seed(w), w.d, 0, w.vocab, T.data_ptr(), stream.cuda_stream)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, F, T,
+                                    load_factor=w.load_factor)
+    S = 2048
+    H = w.K - 1
+    hist0 = synth.query_tokens(w.scaled("mixed_hist", B=S, L=H))
+    state = scone.scone_decode_create(table, hist0, np.full(S, H, np.int32))
+    batches = [mixed_batch(w, k) for k in range(N_BATCHES)]
+    dev_b = [(torch.from_numpy(t).to(dev), torch.from_numpy(c).to(dev), torch.from_numpy(s).to(dev))
+             for t, c, s in batches]
+    out = torch.empty((n_tok, w.d), dtype=torch.int16, device=dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    setup_s = time.time() - t0
+
+    def step(k):
+        t, c, s_ = dev_b[k % N_BATCHES]
+        scone.scone_embed_varlen(table, t, c, out, state=state, seq_slot=s_)
+
+    for k in range(args.warmup):
+        flush_l2(flush)
+        step(k)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    barrier(world)
+    with clocks:
+        for k in range(args.steps):
+            flush_l2(flush)
+            ev[k][0].record(stream)
+            step(k)
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    scone.scone_status(table)
+    per_step_ms = [a.elapsed_time(b) for a, b in ev]
+    kernel_ms = statistics.mean(per_step_ms)
+    ms_step = max_over_ranks(kernel_ms, world)
+
+    # end to end: pinned tokens, offsets and slots in; status word out
+    host_b = [tuple(torch.from_numpy(x).pin_memory() for x in b) for b in batches]
+    e2e_t = []
+    for k in range(max(3, min(args.steps, 50))):
+        flush_l2(flush)
+        torch.cuda.synchronize()
+        t1 = time.perf_counter()
+        t, c, s_ = dev_b[0]
+        for d_, h_ in zip((t, c, s_), host_b[k % N_BATCHES]):
+            d_[:h_.numel()].copy_(h_, non_blocking=True)
+        scone.scone_embed_varlen(table, t, c, out, state=state, seq_slot=s_)
+        scone.scone_status(table)
+        e2e_t.append(time.perf_counter() - t1)
+    e2e_ms = max_over_ranks(1e3 * statistics.mean(e2e_t), world)
+    n_seq = batches[0][1].size - 1
+    per_tok = algorithmic_bytes_per_token(w.K, w.d)
+    bytes_launch = per_tok * n_tok
+    hbm, peak_src = measured_peaks()
+    achieved = bytes_launch / (kernel_ms * 1e-3) / 1e9
+    res = {
+        "metric": METRIC,
+        "value": world * n_tok / (ms_step * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded Zipf token streams and f-gram sets, N(0,0.02)-like bf16 rows)",
+        "config": {
+            "workload": (f"mixed_serving: {n_tok} tokens per launch in {n_seq} sequences "
+                         f"(48 ragged prompt chunks + 512 one-token decode chunks), each "
+                         f"continuing one of {S} decode-state slots; prefill_1b table "
+                         f"({w.n_fgrams} f-grams, K={w.K}, d={w.d}), F in HBM"),
+            "l2": f"flushed between timed steps ({FLUSH_BYTES >> 20} MB write + read back); "
+                  f"steps rotate over {N_BATCHES} batches",
+            "timing": "CUDA events around each step (embedding and history launches)",
+        },
+        "roofline": {
+            "bound": "hbm",
+            "achieved": achieved,
+            "peak": hbm,
+            "unit": "GB/s",
+            "frac": achieved / hbm,
+            "traffic": None,
+            "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
+            "algorithmic_bytes_per_launch": bytes_launch,
+            "kernel": "varlen_embed_kernel (fused match + gather over packed sequences)",
+        },
+        "e2e": {
+            "value": world * n_tok / (e2e_ms * 1e-3),
+            "unit": "tokens/s",
+            "h2d_bytes_per_step": 4 * n_tok + 4 * (n_seq + 1) + 4 * n_seq,
+            "d2h_bytes_per_step": 4,
+            "what": "pinned tokens, offsets and slots -> device, scone_embed_varlen, "
+                    "scone_status",
+        },
+        "gpu_launches": 2 * args.steps,
+        "clocks": clocks.summary(),
+        "kernel_ms_min": min(per_step_ms),
+        "setup_s": setup_s,
+    }
+    state.close()
+    table.close()
+    return res
+
+
 # ---------------------------------------------------------- f-gram discovery
 def bench_discover(args, world, rank, local):
     """Algorithm 3 by K-1 counting scans over a corpus resident in HBM: one
@@ -837,7 +987,7 @@ def main():
     ap.add_argument("--workload", default="prefill_1b",
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
                              "offload_decode", "decode_profile", "prescan", "discover",
-                             "discover_k5", "discover_profile"])
+                             "discover_k5", "discover_profile", "mixed_serving"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
@@ -857,6 +1007,8 @@ def main():
         res = bench_decode(args, world, rank, local)
     elif args.workload == "prescan":
         res = bench_prescan(args, world, rank, local)
+    elif args.workload == "mixed_serving":
+        res = bench_mixed(args, world, rank, local)
     elif args.workload in ("discover", "discover_k5", "discover_profile"):
         res = bench_discover(args, world, rank, local)
     else:

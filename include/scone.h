@@ -284,6 +284,31 @@ int scone_embed(const scone_table* table, const int32_t* tok, int32_t B, int32_t
                 scone_bf16* out, int32_t* row, uint8_t* len, void* stream);
 
 /*
+ * scone_embed_varlen — Algorithm 1 over a packed ragged batch, optionally
+ * continuing sequences held in a decode state: chunked prefill, decode, and
+ * batches that mix them in one launch. Async.
+ *
+ *  tok         device int32 [n_tok]: n_seq sequences packed back to back.
+ *  cu_seqlens  device int32 [n_seq + 1]: sequence b is tok[cu[b] .. cu[b+1]);
+ *              cu[0] = 0, nondecreasing, cu[n_seq] = n_tok (empty sequences
+ *              allowed). Not checked on the host.
+ *  state       NULL: every sequence starts at its first token (with equal
+ *              lengths L this is scone_embed). Otherwise a decode state of the
+ *              same table: sequence b continues slot seq_slot[b] (device int32
+ *              [n_seq], distinct slots; NULL = slot b, then n_seq <= S). The
+ *              slot's history (its last K-1 tokens so far) precedes the chunk,
+ *              so windows reach back into it; after the launch the history is
+ *              the last K-1 tokens of history ++ chunk. A slot outside [0, S)
+ *              is a device-detected INVALID_ARG: zero rows, row -1, len 0.
+ *  out, row, len  as in scone_embed, one entry per packed position.
+ * n_tok <= 2^31 - 1.
+ */
+int scone_embed_varlen(const scone_table* table, const int32_t* tok, int64_t n_tok,
+                       const int32_t* cu_seqlens, int32_t n_seq, scone_decode* state,
+                       const int32_t* seq_slot, scone_bf16* out, int32_t* row, uint8_t* len,
+                       void* stream);
+
+/*
  * Decode (Sec. 3.2: T stays on the accelerator "for decoding", F is looked
  * up per generated token). A decode state holds, per live sequence, its last
  * K-1 tokens on the device, which is all Algorithm 1 needs for the next

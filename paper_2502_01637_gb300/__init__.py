@@ -42,7 +42,7 @@ EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noal
            "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
-           "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
+           "scone_embed_varlen", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
            "scone_strerror", "scone_version")
 
 _lib = None
@@ -103,6 +103,7 @@ def load_library():
     lib.scone_match.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp]
     lib.scone_embed_gather.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_embed.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]
+    lib.scone_embed_varlen.argtypes = [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]
     lib.scone_decode_create.argtypes = [_vp, _i32, _vp, _vp, ctypes.POINTER(_vp)]
     lib.scone_decode_step.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp]
     lib.scone_decode_get_history.argtypes = [_vp, _vp, _vp]
@@ -271,6 +272,18 @@ def scone_embed(table: Table, tok, out, row=None, len=None, stream=None) -> None
     B, L = _bl(tok)
     _check(load_library().scone_embed(table.handle, _ptr(tok), B, L, _ptr(out), _ptr(row),
                                       _ptr(len), _stream(stream)), "scone_embed")
+
+
+def scone_embed_varlen(table: Table, tok, cu_seqlens, out, state=None, seq_slot=None, row=None,
+                       len=None, stream=None) -> None:
+    """Packed ragged batch: tok [n_tok] int32, cu_seqlens [n_seq + 1] int32
+    (device); with a DecodeState, sequence b continues slot seq_slot[b] (or
+    b) and the slots' histories advance."""
+    n_seq = cu_seqlens.numel() - 1
+    _check(load_library().scone_embed_varlen(
+        table.handle, _ptr(tok), tok.numel(), _ptr(cu_seqlens), n_seq,
+        state.handle if state is not None else None, _ptr(seq_slot), _ptr(out), _ptr(row),
+        _ptr(len), _stream(stream)), "scone_embed_varlen")
 
 
 class DecodeState:

@@ -312,6 +312,84 @@ __device__ __forceinline__ int32_t match_position(const TableView& t,
   return -1;
 }
 
+// The same selection for a window whose tokens come from back(j), the token
+// j places before the position, for 1 <= j < nmax (nmax <= K: the longest
+// window within the sequence and its known history); tok_p is the
+// position's own, valid token. Used where a window can reach past the start
+// of the packed tokens (ragged and continued batches). match_position keeps
+// its own copy of these steps: written through this function, the dense
+// kernels' compiled code differs and measured about 1% slower.
+struct Match {
+  int32_t row;   // F row, or -1
+  int len;       // n, 1 for the token fallback, 0 on error
+  int err;       // 0 or a SCONE_ERR_* code
+};
+
+template <int FMT, int KT, class Back>
+__device__ __forceinline__ Match match_window(const TableView& t, int32_t tok_p, int nmax,
+                                              Back back) {
+  int32_t w[KT];
+  w[0] = tok_p;
+#pragma unroll
+  for (int j = 1; j < KT; ++j) w[j] = (j < nmax) ? back(j) : 0;
+  // a window is usable only if all its tokens are valid
+  int nvalid = 1;
+#pragma unroll
+  for (int j = 1; j < KT; ++j)
+    if (nvalid == j && j < nmax && valid_token(w[j], t.vocab)) nvalid = j + 1;
+  nmax = nvalid;
+
+  // round trip 1: the first bucket of every candidate length
+  BucketData<FMT> v[KT - 1];
+#pragma unroll
+  for (int n = 2; n <= KT; ++n) {
+    if (n <= nmax) {
+      uint64_t b1, b2;
+      cuckoo_buckets(key_hash<FMT>(window_key<FMT, KT>(w, n, t.bits), t.hash_seed), t.n_buckets,
+                     &b1, &b2);
+      v[n - 2] = ld_bucket_data<FMT>(t, b1);
+    }
+  }
+  int32_t r1[KT - 1];
+  uint32_t second = 0;   // bit n-2: length n needs its second bucket
+#pragma unroll
+  for (int n = 2; n <= KT; ++n) {
+    r1[n - 2] = -1;
+    if (n <= nmax) {
+      r1[n - 2] = find_in_bucket<FMT>(v[n - 2], window_key<FMT, KT>(w, n, t.bits));
+      if (r1[n - 2] < 0 && bucket_full<FMT>(v[n - 2])) second |= 1u << (n - 2);
+    }
+  }
+  // only lengths longer than the longest first-round hit matter
+  int best = 0;
+#pragma unroll
+  for (int n = 2; n <= KT; ++n)
+    if (r1[n - 2] >= 0) best = n;
+  second &= ~((1u << (best > 1 ? best - 1 : 0)) - 1u);
+  if (second) {
+    if (t.probe_limit < 2) return Match{-1, 0, SCONE_ERR_PROBE_LIMIT};
+    // round trip 2: the second buckets still needed
+#pragma unroll
+    for (int n = 2; n <= KT; ++n) {
+      if (second & (1u << (n - 2))) {
+        uint64_t b1, b2;
+        cuckoo_buckets(key_hash<FMT>(window_key<FMT, KT>(w, n, t.bits), t.hash_seed),
+                       t.n_buckets, &b1, &b2);
+        v[n - 2] = ld_bucket_data<FMT>(t, b2);
+      }
+    }
+#pragma unroll
+    for (int n = 2; n <= KT; ++n)
+      if (second & (1u << (n - 2)))
+        r1[n - 2] = find_in_bucket<FMT>(v[n - 2], window_key<FMT, KT>(w, n, t.bits));
+  }
+#pragma unroll
+  for (int n = KT; n >= 2; --n) {
+    if (n <= nmax && r1[n - 2] >= 0) return Match{r1[n - 2], n, 0};
+  }
+  return Match{-1, 1, 0};
+}
+
 // ------------------------------------------------------------- row copies
 template <typename E>
 __device__ __forceinline__ E ld_row(const E* p) {

@@ -55,6 +55,7 @@ constexpr uint32_t kNone = 0xFFFFFFFFu;
 // ran within 3%: the kernel is bound by the random global updates.
 constexpr int kCountThreads = 512;
 constexpr int kHotSlots = 2048;                 // per-block cache of hot keys (power of 2)
+constexpr int kWin = 4;                         // windows in flight per thread
 constexpr uint32_t kHotTag = 0x80000000u;       // slot_of tag: a cache slot, not a table slot
 constexpr int kWarpSpan = 1024;           // positions (or list entries) per warp chunk
 constexpr int kScanThreads = 1024;
@@ -129,50 +130,76 @@ count_kernel(const int32_t* __restrict__ tok, const uint32_t* __restrict__ names
   unsigned long long my_cand = 0, my_flush = 0;
   const int64_t stride = (int64_t)gridDim.x * kCountThreads;
   const int64_t i0 = (int64_t)blockIdx.x * kCountThreads + threadIdx.x;
-  for (int64_t i = i0; i < N; i += stride) {
-    const int32_t t = tok[i];
-    uint32_t out = kNone;
-    bool cand = true;
-    uint32_t pre = 0;
-    if (n == 2 && (t < 0 || t >= vocab)) {
-      atomicExch(&err->token_range, 1);
-      cand = false;
-    }
-    const int64_t p = i % L;
-    if (cand && p < n - 1) cand = false;
-    if (cand) {
-      if (n == 2) {
-        const int32_t tp = tok[i - 1];
-        cand = tp >= 0 && tp < vocab;
-        pre = (uint32_t)tp;
-      } else {
-        pre = names[i - 1];
-        cand = pre != kNone && names[i] != kNone;
+  // kWin windows per thread and pass (i, i + stride, ...), so that their
+  // loads and their global CAS operations are in flight together
+  for (int64_t ib = i0; ib < N; ib += stride * kWin) {
+    uint64_t key[kWin];
+    uint32_t start[kWin], out[kWin];
+    bool cold[kWin];
+#pragma unroll
+    for (int u = 0; u < kWin; ++u) {
+      const int64_t i = ib + u * stride;
+      key[u] = 0;
+      out[u] = kNone;
+      cold[u] = false;
+      start[u] = 0;
+      if (i >= N) continue;
+      const int32_t t = tok[i];
+      bool cand = true;
+      uint32_t pre = 0;
+      if (n == 2 && (t < 0 || t >= vocab)) {
+        atomicExch(&err->token_range, 1);
+        cand = false;
+      }
+      if (cand && i % L < n - 1) cand = false;
+      if (cand) {
+        if (n == 2) {
+          const int32_t tp = tok[i - 1];
+          cand = tp >= 0 && tp < vocab;
+          pre = (uint32_t)tp;
+        } else {
+          pre = names[i - 1];
+          cand = pre != kNone && names[i] != kNone;
+        }
+      }
+      if (cand) {
+        key[u] = ((uint64_t)(pre + 1u) << 32) | (uint32_t)t;
+        start[u] = (uint32_t)(i - n + 1);
       }
     }
-    if (cand) {
+    // the block's cache first; the windows it does not take go global
+    uint64_t home[kWin];
+    unsigned long long prev[kWin];
+#pragma unroll
+    for (int u = 0; u < kWin; ++u) {
+      if (!key[u]) continue;
       ++my_cand;
-      const uint64_t key = ((uint64_t)(pre + 1u) << 32) | (uint32_t)t;
-      const uint32_t start = (uint32_t)(i - n + 1);
-      const uint32_t h = (uint32_t)(fmix64(key) & (kHotSlots - 1));
-      const unsigned long long prev = atomicCAS(&hkey[h], 0ull, (unsigned long long)key);
-      if (prev == 0 || prev == key) {
+      const uint32_t h = (uint32_t)(fmix64(key[u]) & (kHotSlots - 1));
+      const unsigned long long hp = atomicCAS(&hkey[h], 0ull, (unsigned long long)key[u]);
+      if (hp == 0 || hp == key[u]) {
         atomicAdd(&hcnt[h], 1u);
-        atomicMin(&hfirst[h], start);
-        out = kHotTag | h;
+        atomicMin(&hfirst[h], start[u]);
+        out[u] = kHotTag | h;
       } else {
-        const uint64_t home = slot_home(key, cap);
-        const unsigned long long gp = atomicCAS(&table[home].key, 0ull, key);
-        const uint32_t g = probe_rest(table, cap, key, home, gp, err);
+        cold[u] = true;
+        home[u] = slot_home(key[u], cap);
+        prev[u] = atomicCAS(&table[home[u]].key, 0ull, (unsigned long long)key[u]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kWin; ++u) {
+      if (cold[u]) {
+        const uint32_t g = probe_rest(table, cap, key[u], home[u], prev[u], err);
         ++my_flush;
         if (g != kNone) {
           atomicAdd(&table[g].count, 1u);
-          atomicMax(&table[g].first_inv, ~start);
+          atomicMax(&table[g].first_inv, ~start[u]);
         }
-        out = g;
+        out[u] = g;
       }
+      const int64_t i = ib + u * stride;
+      if (i < N) slot_of[i] = out[u];
     }
-    slot_of[i] = out;
   }
   __syncthreads();
   // flush the cache: the first probe of every owned slot is issued before

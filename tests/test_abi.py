@@ -91,6 +91,12 @@ def test_null_handles_rejected():
     assert lib.scone_decode_destroy(None) == 0
     assert lib.scone_table_get_info(None, None) == inv
     assert lib.scone_table_set_probe_limit(None, 1) == inv
+    assert lib.scone_embed_varlen(None, None, 0, None, 0, None, None, None, None, None,
+                                  None) == inv
+    assert lib.scone_fgram_discover(None, None, 1, 1, 10, 1, 5, 1, None, None, None, None, None,
+                                    None) == inv             # no n_out
+    assert lib.scone_discover_create(None) == inv
+    assert lib.scone_discover_destroy(None) == 0
 
 
 def test_key_format_boundaries():
