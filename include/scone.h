@@ -309,6 +309,22 @@ int scone_embed_varlen(const scone_table* table, const int32_t* tok, int64_t n_t
                        void* stream);
 
 /*
+ * scone_gemm_bf16 — the tensor-core (tcgen05) GEMM behind the f-gram model's
+ * dense layers (exported for testing): C = epilogue(A B^T) with A [M x K] and
+ * B [N x K] bf16, row-major, K contiguous; fp32 accumulation. Epilogues:
+ * SCONE_GEMM_STORE (C [M x N] = A B^T), SCONE_GEMM_RESIDUAL (C = R + A B^T,
+ * R [M x N], C may equal R), SCONE_GEMM_SWIGLU (C [M x N/2]: in every group of
+ * 32 columns of A B^T, the first 16 are gates g and the next 16 ups u of 16
+ * consecutive outputs, C = silu(g) u). N must be a multiple of 256, K of 64,
+ * all pointers device memory aligned to 16 bytes. status: device int that
+ * receives SCONE_ERR_CUDA if a pipeline wait timed out (left untouched
+ * otherwise). Async.
+ */
+enum scone_gemm_epilogue { SCONE_GEMM_STORE = 0, SCONE_GEMM_RESIDUAL = 1, SCONE_GEMM_SWIGLU = 2 };
+int scone_gemm_bf16(const scone_bf16* A, const scone_bf16* B, const scone_bf16* R, scone_bf16* C,
+                    int32_t M, int32_t N, int32_t K, int32_t epilogue, int* status, void* stream);
+
+/*
  * Decode (Sec. 3.2: T stays on the accelerator "for decoding", F is looked
  * up per generated token). A decode state holds, per live sequence, its last
  * K-1 tokens on the device, which is all Algorithm 1 needs for the next

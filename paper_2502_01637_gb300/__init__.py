@@ -36,13 +36,16 @@ SCONE_ROWS_HOST_MAPPED = 1
 SCONE_COPY_AUTO = 0
 SCONE_COPY_REGISTERS = 1
 SCONE_COPY_BULK = 2
+SCONE_GEMM_STORE = 0
+SCONE_GEMM_RESIDUAL = 1
+SCONE_GEMM_SWIGLU = 2
 
 EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noalloc",
            "scone_table_get_info",
            "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
-           "scone_embed_varlen", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
+           "scone_embed_varlen", "scone_gemm_bf16", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
            "scone_strerror", "scone_version")
 
 _lib = None
@@ -104,6 +107,7 @@ def load_library():
     lib.scone_embed_gather.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_embed.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]
     lib.scone_embed_varlen.argtypes = [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]
+    lib.scone_gemm_bf16.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp]
     lib.scone_decode_create.argtypes = [_vp, _i32, _vp, _vp, ctypes.POINTER(_vp)]
     lib.scone_decode_step.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp]
     lib.scone_decode_get_history.argtypes = [_vp, _vp, _vp]
@@ -284,6 +288,27 @@ def scone_embed_varlen(table: Table, tok, cu_seqlens, out, state=None, seq_slot=
         table.handle, _ptr(tok), tok.numel(), _ptr(cu_seqlens), n_seq,
         state.handle if state is not None else None, _ptr(seq_slot), _ptr(out), _ptr(row),
         _ptr(len), _stream(stream)), "scone_embed_varlen")
+
+
+def scone_gemm_bf16(A, B, C, R=None, epilogue: int = SCONE_GEMM_STORE, status=None,
+                    stream=None) -> None:
+    """C = epilogue(A B^T) on the tensor cores; A [M, K], B [N, K], C [M, N]
+    (or [M, N/2] for SwiGLU), bf16 (or int16 raw bits) device tensors. status:
+    a device int32 tensor of one element (allocated here if None; SconeError
+    if a pipeline wait timed out)."""
+    import torch
+
+    M, K = A.shape
+    N = B.shape[0]
+    own = status is None
+    if own:
+        status = torch.zeros(1, dtype=torch.int32, device=A.device)
+    _check(load_library().scone_gemm_bf16(_ptr(A), _ptr(B), _ptr(R), _ptr(C), M, N, K, epilogue,
+                                           _ptr(status), _stream(stream)), "scone_gemm_bf16")
+    if own:
+        code = int(status.item())
+        if code:
+            raise SconeError(code, "scone_gemm_bf16 (device)")
 
 
 class DecodeState:

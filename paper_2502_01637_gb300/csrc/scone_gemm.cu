@@ -1,0 +1,373 @@
+// bf16 GEMM on the 5th-generation tensor cores (tcgen05) for the f-gram
+// model's dense layers: C[M x N] = epilogue(A[M x K] . B[N x K]^T), A and B
+// row-major with K contiguous (activations x weights), fp32 accumulation in
+// tensor memory.
+//
+// One CTA computes a 128 x 256 tile of C with 4 warps:
+//   * thread 0 streams K-slices of 64 (A: 128 x 64, B: 256 x 64, 48 KB) into a
+//     ring of kStages shared-memory stages with TMA (cp.async.bulk.tensor,
+//     128-byte swizzle), each stage completed on an mbarrier by byte count;
+//   * thread 32 issues tcgen05.mma (M = 128, N = 256, K = 16, bf16 x bf16 ->
+//     fp32) over each stage, four per slice, accumulating into 256 columns
+//     of tensor memory, and releases the stage with tcgen05.commit;
+//   * after the last commit all four warps read the accumulator back with
+//     tcgen05.ld (warp w owns tensor-memory lanes 32w .. 32w + 31, i.e. rows)
+//     and apply the epilogue: store, add a residual, or SwiGLU of interleaved
+//     gate/up column pairs.
+// Every mbarrier wait is bounded (kGemmSpin polls); past it the CTA records
+// SCONE_ERR_CUDA, stops issuing, drains what it issued, frees its tensor
+// memory and returns.
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+#include <mutex>
+
+#include "scone_gemm.h"
+#include "scone_host.h"
+
+namespace scone {
+
+namespace {
+
+constexpr int kBM = 128, kBN = 256, kBK = 64;
+constexpr int kStages = 4;
+constexpr int kGemmThreads = 128;
+constexpr uint32_t kStageA = kBM * kBK * 2;   // 16 KB
+constexpr uint32_t kStageB = kBN * kBK * 2;   // 32 KB
+constexpr uint32_t kStageBytes = kStageA + kStageB;
+constexpr uint32_t kTmemCols = kBN;           // fp32 accumulator: 256 columns x 128 lanes
+constexpr uint32_t kGemmSpin = 1u << 22;   // polls; each try_wait may also suspend briefly
+constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + 1024 /* align */ + 256 /* barriers */;
+
+__device__ __forceinline__ uint32_t saddr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n"
+      " mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait; false on timeout.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kGemmSpin; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major tile whose rows are 128 bytes
+// (64 bf16) with the 128-byte swizzle: 8-row atoms of 1024 bytes, stride
+// between atoms 1024 bytes; the leading-dimension offset is unused for this
+// layout. Bits: start >> 4 at 0, LBO >> 4 at 16, SBO >> 4 at 32, version 1 at
+// 46, swizzle mode 2 (128 B) at 61.
+__device__ __forceinline__ uint64_t desc_k128(uint32_t smem_byte_addr) {
+  uint64_t d = (uint64_t)((smem_byte_addr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A and B bf16 (bits
+// 7-9, 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at 17, M >> 4 at 24.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) |
+                            ((uint32_t)(kBM >> 4) << 24);
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n"
+      " setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+      "%28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);   // a in the low half
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+template <int EPI>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_bf16_kernel(const __grid_constant__ CUtensorMap map_a,
+                     const __grid_constant__ CUtensorMap map_b, int M, int N, int K,
+                     const uint16_t* __restrict__ R, uint16_t* __restrict__ C, int ldc,
+                     int* status) {
+  extern __shared__ uint8_t gsm_raw[];
+  // 1024-byte alignment: the 128-byte swizzle pattern repeats every 1024 bytes
+  uint8_t* gsm = reinterpret_cast<uint8_t*>(((uintptr_t)gsm_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = reinterpret_cast<uint64_t*>(gsm + kStages * kStageBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* done = empty + kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  __shared__ int failed;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * kBN;
+  const int kt_n = K / kBK;
+
+  if (threadIdx.x == 0) {
+    failed = 0;
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(saddr(&full[s]), 1);
+      mbar_init(saddr(&empty[s]), 1);
+    }
+    mbar_init(saddr(done), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     saddr(tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+
+  if (threadIdx.x == 0) {
+    // producer: K-slices into the ring
+    int issued = 0;
+    for (int kt = 0; kt < kt_n; ++kt) {
+      const int s = kt % kStages;
+      if (kt >= kStages && !mbar_wait(saddr(&empty[s]), ((kt / kStages) - 1) & 1)) {
+        atomicExch(&failed, 1);
+        break;
+      }
+      if (*reinterpret_cast<volatile int*>(&failed)) break;
+      const uint32_t a_dst = saddr(gsm + s * kStageBytes);
+      const uint32_t b_dst = a_dst + kStageA;
+      mbar_expect_tx(saddr(&full[s]), kStageBytes);
+      tma_load_2d(a_dst, &map_a, kt * kBK, m0, saddr(&full[s]));
+      tma_load_2d(b_dst, &map_b, kt * kBK, n0, saddr(&full[s]));
+      ++issued;
+    }
+    // drain: every issued slice must have landed before the CTA may exit
+    for (int kt = 0; kt < issued; ++kt)
+      if (kt + kStages >= issued) mbar_wait(saddr(&full[kt % kStages]), (kt / kStages) & 1);
+  } else if (threadIdx.x == 32) {
+    // MMA issuer
+    bool ok = true;
+    for (int kt = 0; kt < kt_n && ok; ++kt) {
+      const int s = kt % kStages;
+      if (!mbar_wait(saddr(&full[s]), (kt / kStages) & 1) ||
+          *reinterpret_cast<volatile int*>(&failed)) {
+        atomicExch(&failed, 1);
+        ok = false;
+        break;
+      }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t a_base = saddr(gsm + s * kStageBytes);
+      const uint32_t b_base = a_base + kStageA;
+#pragma unroll
+      for (int k = 0; k < kBK / 16; ++k)
+        umma_bf16(tmem, desc_k128(a_base + 32 * k), desc_k128(b_base + 32 * k),
+                  (kt > 0 || k > 0) ? 1u : 0u);
+      umma_commit(saddr(&empty[s]));
+    }
+    umma_commit(saddr(done));   // arrives once every MMA issued above has completed
+  }
+  __syncwarp();
+
+  // epilogue: all 128 threads, one accumulator row (tensor-memory lane) each
+  const bool ok = mbar_wait(saddr(done), 0);
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  if (!ok) atomicExch(&failed, 1);
+  __syncthreads();
+  if (failed) {
+    if (threadIdx.x == 0) atomicCAS(status, 0, (int)SCONE_ERR_CUDA);
+  } else {
+    const int row = m0 + warp * 32 + lane;
+    const uint32_t t_row = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll 1
+    for (int c0 = 0; c0 < kBN; c0 += 32) {
+      float v[32];
+      tmem_ld32(t_row + c0, v);   // every lane takes part (.sync.aligned)
+      if (row >= M) {
+      } else if constexpr (EPI == GEMM_EPI_SWIGLU) {
+        // 32 columns = 16 gates then 16 ups of outputs (n0 + c0) / 2 ..
+        uint32_t o[8];
+#pragma unroll
+        for (int j = 0; j < 16; j += 2) {
+          const float g0 = v[j], g1 = v[j + 1], u0 = v[16 + j], u1 = v[17 + j];
+          const float a0 = g0 / (1.f + expf(-g0)) * u0;
+          const float a1 = g1 / (1.f + expf(-g1)) * u1;
+          o[j / 2] = pack_bf16(a0, a1);
+        }
+        uint4* dst = reinterpret_cast<uint4*>(C + (int64_t)row * ldc + (n0 + c0) / 2);
+        dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+        dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+      } else {
+        uint32_t o[16];
+        if constexpr (EPI == GEMM_EPI_RESIDUAL) {
+          const uint4* src = reinterpret_cast<const uint4*>(R + (int64_t)row * ldc + n0 + c0);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint4 r4 = src[q];
+            const uint32_t rw[4] = {r4.x, r4.y, r4.z, r4.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int j = q * 8 + e * 2;
+              o[q * 4 + e] = pack_bf16(v[j] + bf16_lo(rw[e]), v[j + 1] + bf16_hi(rw[e]));
+            }
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) o[j / 2] = pack_bf16(v[j], v[j + 1]);
+        }
+        uint4* dst = reinterpret_cast<uint4*>(C + (int64_t)row * ldc + n0 + c0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          dst[q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+      }
+    }
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 0)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols)
+                 : "memory");
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    else
+      cudaGetLastError();
+  });
+  return fn;
+}
+
+// 2-D map of a row-major bf16 matrix [rows x cols] (cols contiguous), box
+// 64 columns x box_rows rows, 128-byte swizzle; rows past the end read zero.
+bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int box_rows) {
+  const auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
+template <int EPI>
+bool set_smem_attr() {
+  static std::once_flag once;
+  static bool ok = false;
+  std::call_once(once, [] {
+    ok = cudaFuncSetAttribute(gemm_bf16_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)kGemmSmem) == cudaSuccess;
+    if (!ok) cudaGetLastError();
+  });
+  return ok;
+}
+
+}  // namespace
+
+int gemm_bf16(const uint16_t* A, const uint16_t* B, const uint16_t* R, uint16_t* C, int M, int N,
+              int K, int epi, int* status, cudaStream_t s) {
+  if (M < 0 || N <= 0 || K <= 0 || N % kBN || K % kBK || !A || !B || !C || !status)
+    return SCONE_ERR_INVALID_ARG;
+  if (epi == GEMM_EPI_RESIDUAL && !R) return SCONE_ERR_INVALID_ARG;
+  if (((uintptr_t)A | (uintptr_t)B | (uintptr_t)C | (uintptr_t)R) & 15)
+    return SCONE_ERR_INVALID_ARG;
+  if (M == 0) return SCONE_OK;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, A, M, K, kBM) || !make_map(&mb, B, N, K, kBN)) return SCONE_ERR_CUDA;
+  const dim3 grid((unsigned)((M + kBM - 1) / kBM), (unsigned)(N / kBN));
+  const int ldc = epi == GEMM_EPI_SWIGLU ? N / 2 : N;
+  switch (epi) {
+    case GEMM_EPI_STORE:
+      if (!set_smem_attr<GEMM_EPI_STORE>()) return SCONE_ERR_CUDA;
+      gemm_bf16_kernel<GEMM_EPI_STORE><<<grid, kGemmThreads, kGemmSmem, s>>>(ma, mb, M, N, K, R,
+                                                                            C, ldc, status);
+      break;
+    case GEMM_EPI_RESIDUAL:
+      if (!set_smem_attr<GEMM_EPI_RESIDUAL>()) return SCONE_ERR_CUDA;
+      gemm_bf16_kernel<GEMM_EPI_RESIDUAL><<<grid, kGemmThreads, kGemmSmem, s>>>(
+          ma, mb, M, N, K, R, C, ldc, status);
+      break;
+    case GEMM_EPI_SWIGLU:
+      if (!set_smem_attr<GEMM_EPI_SWIGLU>()) return SCONE_ERR_CUDA;
+      gemm_bf16_kernel<GEMM_EPI_SWIGLU><<<grid, kGemmThreads, kGemmSmem, s>>>(ma, mb, M, N, K, R,
+                                                                             C, ldc, status);
+      break;
+    default:
+      return SCONE_ERR_INVALID_ARG;
+  }
+  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}
+
+}  // namespace scone
+
+extern "C" int scone_gemm_bf16(const scone_bf16* A, const scone_bf16* B, const scone_bf16* R,
+                               scone_bf16* C, int32_t M, int32_t N, int32_t K, int32_t epilogue,
+                               int* status, void* stream) {
+  return scone::gemm_bf16(A, B, R, C, M, N, K, epilogue, status, (cudaStream_t)stream);
+}

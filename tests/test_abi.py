@@ -20,7 +20,7 @@ HEADER = os.path.join(ROOT, "include", "scone.h")
 def declared_functions():
     src = open(HEADER).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(scone_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(scone_[a-z_0-9]+)\s*\(", src)))
 
 
 def test_every_declared_symbol_is_exported():
@@ -31,7 +31,7 @@ def test_every_declared_symbol_is_exported():
         assert hasattr(lib, n), n
     out = subprocess.run(["nm", "-D", "--defined-only", scone.LIB_PATH], capture_output=True,
                          text=True, check=True).stdout
-    exported = set(re.findall(r"\bT (scone_[a-z_]+)", out))
+    exported = set(re.findall(r"\bT (scone_[a-z_0-9]+)", out))
     assert set(names) <= exported, set(names) - exported
     assert set(scone.EXPORTS) == set(names)
 
