@@ -41,7 +41,7 @@ import numpy as np
 MASTER_SEED = 20250203
 
 # stream ids
-S_QUERY, S_SOURCE, S_FROWS, S_TROWS, S_PHRASES, S_DEC_HIST, S_DEC_TOK = range(7)
+S_QUERY, S_SOURCE, S_FROWS, S_TROWS, S_PHRASES, S_DEC_HIST, S_DEC_TOK, S_MODEL = range(8)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "libsynth.so")
@@ -289,3 +289,73 @@ def decode_inputs(w: Workload):
     for s in range(S):
         new[:, s] = zipf_tokens(w, stream_seed(w, S_DEC_TOK, s), w.dec_steps, inject=False)
     return hist, hl, new
+
+
+# ------------------------------------------------------------ f-gram model
+@dataclasses.dataclass(frozen=True)
+class FgramModel:
+    """Shape of the f-gram transformer (A_fgram) whose weights are drawn here.
+
+    The packed weight buffer holds, per layer, four row-major bf16 matrices:
+    qkv [3d x d] (query, key, value rows), o [d x d], gu [2 ffw x d] (gate and
+    up rows interleaved in groups of 16: rows 32g..32g+15 are the gates of
+    features 16g..16g+15, the next 16 rows their ups), down [d x ffw]. Every
+    entry is an independent draw of the bf16 row generator (std 0.02).
+    """
+    name: str
+    mid: int          # model id, mixed into every seed
+    d: int
+    n_heads: int
+    ffw: int
+    n_layers: int
+
+    def shapes(self):
+        d, f = self.d, self.ffw
+        return (("qkv", 3 * d, d), ("o", d, d), ("gu", 2 * f, d), ("down", d, f))
+
+    @property
+    def layer_elems(self) -> int:
+        return sum(r * c for _, r, c in self.shapes())
+
+    @property
+    def n_elems(self) -> int:
+        return self.n_layers * self.layer_elems
+
+    def offset(self, layer: int, which: str) -> int:
+        off = layer * self.layer_elems
+        for name, r, c in self.shapes():
+            if name == which:
+                return off
+            off += r * c
+        raise KeyError(which)
+
+
+MODELS: Dict[str, FgramModel] = {
+    # small enough for the fp64 oracle on every f-gram of a test
+    "tiny": FgramModel("tiny", 20, 256, 4, 512, 2),
+    # the 711M OLMo shape the paper uses for its smaller f-gram model
+    # (d_model 2048, ffw 8192, 12 layers; 16 heads of 128)
+    "olmo_711m": FgramModel("olmo_711m", 21, 2048, 16, 8192, 12),
+}
+
+
+def model_seed(m: FgramModel, layer: int, which: int) -> int:
+    return int(_load().synth_stream_seed(MASTER_SEED, m.mid, S_MODEL, layer * 4 + which))
+
+
+def model_weights_cpu(m: FgramModel) -> np.ndarray:
+    """The packed weight buffer as raw bf16 words, [n_elems] uint16."""
+    out = np.empty(m.n_elems, np.uint16)
+    for layer in range(m.n_layers):
+        for k, (name, r, c) in enumerate(m.shapes()):
+            off = m.offset(layer, name)
+            out[off:off + r * c] = rows_range_cpu(model_seed(m, layer, k), c, 0, r).reshape(-1)
+    return out
+
+
+def model_weights_gpu(m: FgramModel, out_ptr: int, stream_ptr: int) -> None:
+    """The same buffer written at a device address (2 bytes per element)."""
+    for layer in range(m.n_layers):
+        for k, (name, r, c) in enumerate(m.shapes()):
+            rows_gpu(model_seed(m, layer, k), c, 0, r, out_ptr + 2 * m.offset(layer, name),
+                     stream_ptr)

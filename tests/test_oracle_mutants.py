@@ -4,9 +4,11 @@ Each mutant is a plausible slip in the oracle's C++: for Algorithm 1 (scan
 order, window bound, row or length off by one, token range, duplicate
 handling, gather source, decode history alignment) and for Algorithm 3
 (window bound, length range, first occurrence, threshold, sort direction, tie
-order, the top-S cut, sequence boundary). The copy is compiled on the CPU and
-the pin tests in test_oracle.py and test_discover_oracle.py run against it in
-a subprocess; they must fail.
+order, the top-S cut, sequence boundary), and in the f-gram model oracle
+(rotation direction and base, causal mask, score scale, layer-norm epsilon,
+gate/up swap, a dropped residual, the output position, bf16 tie rounding).
+The copy is compiled (C++) or loaded (Python) on the CPU and the pin tests
+run against it in a subprocess; they must fail.
 """
 
 import os
@@ -20,6 +22,21 @@ SRCS = {"alg1": os.path.join(ROOT, "oracle", "scone_oracle.cpp"),
         "alg3": os.path.join(ROOT, "oracle", "discover_oracle.cpp")}
 PINS = [os.path.join(ROOT, "tests", "test_oracle.py"),
         os.path.join(ROOT, "tests", "test_discover_oracle.py")]
+MODEL_SRC = os.path.join(ROOT, "oracle", "fgram_model.py")
+MODEL_PINS = os.path.join(ROOT, "tests", "test_fgram_model_oracle.py")
+
+MODEL_MUTANTS = {
+    "m_rope_direction": ("[a * c - b * s, b * c + a * s]", "[a * c + b * s, b * c - a * s]"),
+    "m_rope_base": ("ROPE_BASE = 10000.0", "ROPE_BASE = 1000.0"),
+    "m_no_causal_mask": ("scores = np.where(np.tril(np.ones((n, n), bool)), scores, -np.inf)",
+                         "scores = scores"),
+    "m_no_score_scale": ("scores = qh @ kh.T / np.sqrt(hd)", "scores = qh @ kh.T"),
+    "m_ln_eps": ("LN_EPS = 1e-5", "LN_EPS = 1e-3"),
+    "m_gate_up_swapped": ('mats["gate"] = gu[:, 0].reshape(f, d)', 'mats["gate"] = gu[:, 1].reshape(f, d)'),
+    "m_attention_residual_dropped": ('x = r(x + o @ L["o"].T)', 'x = r(o @ L["o"].T)'),
+    "m_first_position": ("f = layer_norm(x[-1:])[0]", "f = layer_norm(x[:1])[0]"),
+    "m_round_half_up": ("np.round(m * 256.0)", "np.floor(m * 256.0 + 0.5)"),
+}
 
 SCAN = """  for (int64_t jp = first; jp < i; ++jp) {
     const std::vector<int32_t> window(seq + jp, seq + i + 1);
@@ -116,3 +133,17 @@ def test_mutant_is_caught(name, tmp_path):
 def test_unmutated_copy_passes(tmp_path):
     rc, log = _run_pins(_compile(tmp_path))
     assert rc == 0, log
+
+
+@pytest.mark.parametrize("name", sorted(MODEL_MUTANTS))
+def test_model_mutant_is_caught(name, tmp_path):
+    old, new = MODEL_MUTANTS[name]
+    src = open(MODEL_SRC).read()
+    assert old in src, f"mutation site for {name} not found"
+    path = tmp_path / "fgram_model_mut.py"
+    path.write_text(src.replace(old, new))
+    env = dict(os.environ, SCONE_FGRAM_ORACLE_FILE=str(path))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        MODEL_PINS], cwd=ROOT, env=env, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode != 0, f"mutant {name} passed every pin:\n{r.stdout[-2000:]}"
