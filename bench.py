@@ -799,6 +799,157 @@ def bench_mixed(args, world, rank, local):
     return res
 
 
+# ------------------------------------------------------- F precompute (NEXT-3)
+def model_flops_per_token(m) -> int:
+    """Dense-layer FLOPs of one token through the f-gram model (2 per MAC)."""
+    return 2 * m.n_layers * (4 * m.d * m.d + 3 * m.d * m.ffw)
+
+
+def bench_precompute(args, world, rank, local):
+    """F rows of 65,536 f-grams (prefill_1b's list: 2- and 3-grams) by the
+    12-layer, d = 2048 f-gram model (the paper's 711M OLMo shape, random
+    weights): one step is one scone_fgram_precompute call."""
+    import torch
+
+    import synth
+    import paper_2502_01637_gb300 as scone
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = synth.WORKLOADS["prefill_1b"]
+    m = synth.MODELS["olmo_711m"]
+    n_f = 65536
+    t0 = time.time()
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    fg_tok, fg_len = fg_tok[:n_f], fg_len[:n_f]
+    stream = torch.cuda.current_stream()
+    weights = torch.empty(m.n_elems, dtype=torch.int16, device=dev)
+    synth.model_weights_gpu(m, weights.data_ptr(), stream.cuda_stream)
+    T = torch.empty((w.vocab, m.d), dtype=torch.int16, device=dev)
+    synth.rows_gpu(synth.T_seed(w), m.d, 0, w.vocab, T.data_ptr(), stream.cuda_stream)
+    tok_d = torch.from_numpy(fg_tok).to(dev)
+    len_d = torch.from_numpy(fg_len).to(dev)
+    F = torch.empty((n_f, m.d), dtype=torch.int16, device=dev)
+    model = scone.FgramModel(m.d, m.n_heads, m.ffw, m.n_layers, weights, batch=16384)
+    setup_s = time.time() - t0
+    tokens = int(fg_len.astype(np.int64).sum())
+    flops = model_flops_per_token(m) * tokens
+
+    def step():
+        scone.scone_fgram_precompute(model, tok_d, len_d, T, F)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    barrier(world)
+    with clocks:
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms = max_over_ranks(statistics.mean(a.elapsed_time(b) for a, b in ev), world)
+
+    # the dominant kernel timed alone with CUDA events: the gate/up GEMM of one
+    # 16,384-f-gram batch (M = its tokens, N = 2 ffw, K = d) with SwiGLU
+    M = int(fg_len[:16384].astype(np.int64).sum())
+    A = torch.empty((M, m.d), dtype=torch.int16, device=dev)
+    synth.rows_gpu(99, m.d, 0, M, A.data_ptr(), stream.cuda_stream)
+    Bw = weights[m.offset(0, "gu"):m.offset(0, "gu") + 2 * m.ffw * m.d].view(2 * m.ffw, m.d)
+    C = torch.empty((M, m.ffw), dtype=torch.int16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    for _ in range(3):
+        scone.scone_gemm_bf16(A, Bw, C, epilogue=scone.SCONE_GEMM_SWIGLU, status=status)
+    gev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(20)]
+    for a, b in gev:
+        a.record(stream)
+        scone.scone_gemm_bf16(A, Bw, C, epilogue=scone.SCONE_GEMM_SWIGLU, status=status)
+        b.record(stream)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    g_ms = statistics.mean(a.elapsed_time(b) for a, b in gev)
+    g_tflops = 2.0 * M * 2 * m.ffw * m.d / (g_ms * 1e-3) / 1e12
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) \
+        if os.path.exists(os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
+    peak = float(peaks.get("bf16_tflops", 1900.0))
+    res = {
+        "metric": "precomputed F rows/s at 1 GB300 (f-gram model forward, Sec. 3.2)",
+        "value": world * n_f / (ms * 1e-3),
+        "unit": "f-gram rows/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (random bf16 weights, seeded f-gram list and T rows)",
+        "config": {"workload": (f"precompute: {n_f} f-grams ({tokens} tokens) of prefill_1b's "
+                                f"list through a {m.n_layers}-layer model, d={m.d}, "
+                                f"{m.n_heads} heads, ffw={m.ffw} (SwiGLU), "
+                                f"{m.n_elems / 1e6:.0f}M parameters; batches of 16384 f-grams"),
+                   "l2": "weights (1.6 GB) and activations far larger than L2; no flush",
+                   "timing": "CUDA events around each scone_fgram_precompute call"},
+        "model_tflops": flops / (ms * 1e-3) / 1e12,
+        "roofline": {
+            "bound": "tensor",
+            "achieved": g_tflops,
+            "peak": peak,
+            "unit": "TFLOP/s",
+            "frac": g_tflops / peak,
+            "traffic": None,
+            "peak_source": "measured (MEASURED_PEAKS.json bf16_tflops, burst)" if peaks
+                           else "fallback",
+            "kernel": f"gemm_bf16_kernel<SWIGLU>: M={M}, N={2 * m.ffw}, K={m.d} "
+                      "(gate/up of one batch), timed alone",
+            "kernel_ms": g_ms,
+            "algorithmic_flops_per_launch": 2 * M * 2 * m.ffw * m.d,
+        },
+        "e2e": {"value": world * n_f / (ms * 1e-3), "unit": "f-gram rows/s",
+                "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0,
+                "what": "the f-gram list and F stay on the device (F is written where the "
+                        "table will read it)"},
+        "gpu_launches": args.steps * (4 * (3 + m.n_layers * 7)),
+        "clocks": clocks.summary(),
+        "setup_s": setup_s,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        res["cpu_baseline"] = cpu_baseline_precompute(m, fg_tok, fg_len, w)
+    model.close()
+    return res
+
+
+def cpu_baseline_precompute(m, fg_tok, fg_len, w, budget_s: float = 10.0):
+    """The float64 oracle forward (numpy; its BLAS may use several threads) on
+    the first f-grams of the same list, until about budget_s."""
+    import synth
+    from oracle import fgram_model as fm
+
+    packed = synth.model_weights_cpu(m)
+    W = fm.Weights(packed, m)
+    used = np.unique(fg_tok[:64][fg_tok[:64] >= 0])
+    T = np.zeros((w.vocab, m.d), np.uint16)
+    T[used] = synth.rows_cpu(synth.T_seed(w), m.d, used)
+    t0 = time.perf_counter()
+    done = 0
+    while done < 64:
+        fm.fgram_row(fg_tok[done][:fg_len[done]], T, W, emulate_bf16=True)
+        done += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": done / dt, "unit": "f-gram rows/s", "cores": os.cpu_count() or 1,
+            "kind": "oracle",
+            "sample": f"float64 oracle forward of the first {done} f-grams ({dt:.1f} s; numpy "
+                      "BLAS threads as configured)"}
+
+
 # ---------------------------------------------------------- f-gram discovery
 def bench_discover(args, world, rank, local):
     """Algorithm 3 by K-1 counting scans over a corpus resident in HBM: one
@@ -987,7 +1138,7 @@ def main():
     ap.add_argument("--workload", default="prefill_1b",
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
                              "offload_decode", "decode_profile", "prescan", "discover",
-                             "discover_k5", "discover_profile", "mixed_serving"])
+                             "discover_k5", "discover_profile", "mixed_serving", "precompute"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
@@ -1009,6 +1160,8 @@ def main():
         res = bench_prescan(args, world, rank, local)
     elif args.workload == "mixed_serving":
         res = bench_mixed(args, world, rank, local)
+    elif args.workload == "precompute":
+        res = bench_precompute(args, world, rank, local)
     elif args.workload in ("discover", "discover_k5", "discover_profile"):
         res = bench_discover(args, world, rank, local)
     else:

@@ -325,6 +325,43 @@ int scone_gemm_bf16(const scone_bf16* A, const scone_bf16* B, const scone_bf16* 
                     int32_t M, int32_t N, int32_t K, int32_t epilogue, int* status, void* stream);
 
 /*
+ * Precomputing F with the f-gram model (Sec. 3.2: after training F is
+ * precomputed and stored; Algorithm 1 embeds an f-gram by A_fgram(T(s_j), ..,
+ * T(s_i)) in training). The model is a pre-LN transformer: per layer
+ * h = x + Attn(LN(x)), x = h + MLP(LN(h)); LN is the non-parametric layer norm
+ * (eps 1e-5); Attn is causal multi-head attention with rotary positions
+ * (rotate-half pairs (i, i + hd/2), angle pos * 10000^(-2i/hd)), scaled by
+ * 1/sqrt(hd); MLP is SwiGLU. F(w) = LN of the last position's final state.
+ *
+ * scone_fgram_model_create: d (multiple of 256, d/256 a power of two up to
+ * 16), n_heads (head size d/n_heads in {64, 128, 256}), ffw (multiple of 128),
+ * n_layers; weights: device bf16, packed per layer as qkv [3d x d] (query,
+ * key, value rows), o [d x d], gu [2 ffw x d] (rows 32g..32g+15 are the gates
+ * of features 16g..16g+15, the next 16 rows their ups), down [d x ffw],
+ * row-major; borrowed, must outlive the model. batch: f-grams per internal
+ * batch (0 = 16384); the workspace grows with the tokens of a batch.
+ * Synchronous.
+ */
+typedef struct scone_fgram_model scone_fgram_model;
+int scone_fgram_model_create(int32_t d, int32_t n_heads, int32_t ffw, int32_t n_layers,
+                             const scone_bf16* weights, int64_t batch, scone_fgram_model** out);
+int scone_fgram_model_destroy(scone_fgram_model* model);
+
+/*
+ * scone_fgram_precompute: F rows of n f-grams. fgram_tok device int32 [n * K]
+ * (f-gram r's tokens first, padding ignored), fgram_len device uint8 [n] in
+ * [2, K] (lengths outside [1, K] are read as 1 and reported), T device
+ * [vocab * d], F device or host-mapped [n * d] (16-byte aligned). The f-grams
+ * of a batch are packed without padding and every dense layer is a
+ * tensor-core GEMM over all their tokens. Synchronous; returns SCONE_OK or
+ * the first device-detected error (TOKEN_RANGE: that token's row is zero;
+ * INVALID_ARG: a length outside [1, K]; CUDA: a GEMM pipeline timed out).
+ */
+int scone_fgram_precompute(scone_fgram_model* model, const int32_t* fgram_tok,
+                           const uint8_t* fgram_len, int64_t n, int32_t K, const scone_bf16* T,
+                           int32_t vocab, scone_bf16* F, void* stream);
+
+/*
  * Decode (Sec. 3.2: T stays on the accelerator "for decoding", F is looked
  * up per generated token). A decode state holds, per live sequence, its last
  * K-1 tokens on the device, which is all Algorithm 1 needs for the next

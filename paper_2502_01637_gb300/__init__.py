@@ -45,7 +45,8 @@ EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noal
            "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
-           "scone_embed_varlen", "scone_gemm_bf16", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
+           "scone_embed_varlen", "scone_gemm_bf16", "scone_fgram_model_create",
+           "scone_fgram_model_destroy", "scone_fgram_precompute", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
            "scone_strerror", "scone_version")
 
 _lib = None
@@ -108,6 +109,10 @@ def load_library():
     lib.scone_embed.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]
     lib.scone_embed_varlen.argtypes = [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]
     lib.scone_gemm_bf16.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp]
+    lib.scone_fgram_model_create.argtypes = [_i32, _i32, _i32, _i32, _vp, _i64,
+                                             ctypes.POINTER(_vp)]
+    lib.scone_fgram_model_destroy.argtypes = [_vp]
+    lib.scone_fgram_precompute.argtypes = [_vp, _vp, _vp, _i64, _i32, _vp, _i32, _vp, _vp]
     lib.scone_decode_create.argtypes = [_vp, _i32, _vp, _vp, ctypes.POINTER(_vp)]
     lib.scone_decode_step.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp]
     lib.scone_decode_get_history.argtypes = [_vp, _vp, _vp]
@@ -309,6 +314,55 @@ def scone_gemm_bf16(A, B, C, R=None, epilogue: int = SCONE_GEMM_STORE, status=No
         code = int(status.item())
         if code:
             raise SconeError(code, "scone_gemm_bf16 (device)")
+
+
+class FgramModel:
+    """The f-gram model on the device (borrows its packed weights)."""
+
+    def __init__(self, d: int, n_heads: int, ffw: int, n_layers: int, weights, batch: int = 0):
+        h = _vp()
+        _check(load_library().scone_fgram_model_create(d, n_heads, ffw, n_layers, _ptr(weights),
+                                                       batch, ctypes.byref(h)),
+               "scone_fgram_model_create")
+        self._h = h
+        self._keep = weights
+        self.d = d
+
+    @property
+    def handle(self):
+        if self._h is None:
+            raise RuntimeError("model was closed")
+        return self._h
+
+    def close(self):
+        if self._h is not None:
+            load_library().scone_fgram_model_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def scone_fgram_model_create(d, n_heads, ffw, n_layers, weights, batch=0) -> FgramModel:
+    return FgramModel(d, n_heads, ffw, n_layers, weights, batch)
+
+
+def scone_fgram_model_destroy(model: FgramModel) -> None:
+    model.close()
+
+
+def scone_fgram_precompute(model: FgramModel, fgram_tok, fgram_len, T, F, vocab: Optional[int] = None,
+                           stream=None) -> None:
+    """F rows of the f-grams: fgram_tok [n, K] int32 and fgram_len [n] uint8 device
+    tensors, T [vocab, d] device, F [n, d] device tensor (or host-mapped address)."""
+    n, K = fgram_tok.shape
+    vocab = T.shape[0] if vocab is None else vocab
+    _check(load_library().scone_fgram_precompute(model.handle, _ptr(fgram_tok), _ptr(fgram_len), n,
+                                                 K, _ptr(T), vocab, _ptr(F), _stream(stream)),
+           "scone_fgram_precompute")
 
 
 class DecodeState:

@@ -1,0 +1,406 @@
+// Precomputing F with the f-gram model (C ABI).
+//
+// At inference F(w) is the f-gram model's output for w, computed once and
+// stored (Sec. 3.2; Algorithm 1 uses A_fgram(T(s_j), .., T(s_i)) in training
+// and the stored F(s_j, .., s_i) at inference). The model is a pre-LN
+// transformer: per layer h = x + Attn(LN(x)), x = h + MLP(LN(h)), with
+// non-parametric layer norm (eps 1e-5), causal multi-head attention with
+// rotary positions (rotate-half pairs, base 10000) and a SwiGLU MLP; F(w) is
+// the layer norm of the last position's final state.
+//
+// The f-grams of a batch are packed token after token (no padding) into one
+// [M x d] activation matrix, M = sum of their lengths, so every dense layer
+// is one GEMM over all tokens of the batch on the tensor cores
+// (scone_gemm.cu): qkv, the output projection with the residual added in
+// its epilogue, gate/up with SwiGLU in its epilogue, and down with the
+// residual. What is not a contraction runs on the CUDA cores, one warp per
+// row or per (f-gram, head): the token-row gather, layer norm, attention over
+// at most K positions, and the final layer norm written to F.
+
+#include <cuda_bf16.h>
+
+#include <new>
+
+#include "scone_gemm.h"
+#include "scone_host.h"
+
+struct scone_fgram_model {
+  int device = 0;
+  int32_t d = 0, n_heads = 0, ffw = 0, n_layers = 0;
+  const uint16_t* weights = nullptr;     // borrowed, packed layout
+  int64_t batch = 0;                     // f-grams per batch
+  int64_t cap_rows = 0;                  // workspace rows (tokens)
+  int32_t* off = nullptr;                // [batch + 1] token offsets
+  int* status = nullptr;                 // sticky device error
+  uint16_t *X = nullptr, *Xn = nullptr, *QKV = nullptr, *Act = nullptr;
+};
+
+namespace scone {
+
+namespace {
+
+constexpr float kLnEps = 1e-5f;
+constexpr int kRowsPerBlock = 8;       // one warp per row, 8 warps per block
+
+__device__ __forceinline__ void set_error(int* status, int code) {
+  if (*reinterpret_cast<volatile int*>(status) == 0) atomicCAS(status, 0, code);
+}
+
+__device__ __forceinline__ float lo_f(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float hi_f(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// Exclusive prefix sum of the batch's lengths (one block): off[0..n].
+__global__ void __launch_bounds__(1024)
+    offsets_kernel(const uint8_t* __restrict__ len, int64_t n, int32_t K, int32_t* __restrict__ off,
+                   int* status) {
+  __shared__ int32_t part[1024];
+  const int64_t per = (n + 1023) / 1024;
+  const int64_t b = threadIdx.x * per, e = b + per < n ? b + per : n;
+  int32_t s = 0;
+  for (int64_t i = b; i < e; ++i) {
+    int32_t l = len[i];
+    if (l < 1 || l > K) {
+      set_error(status, SCONE_ERR_INVALID_ARG);
+      l = 1;
+    }
+    s += l;
+  }
+  part[threadIdx.x] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int32_t run = 0;
+    for (int t = 0; t < 1024; ++t) {
+      const int32_t v = part[t];
+      part[t] = run;
+      run += v;
+    }
+    off[n] = run;
+  }
+  __syncthreads();
+  int32_t run = part[threadIdx.x];
+  for (int64_t i = b; i < e; ++i) {
+    off[i] = run;
+    int32_t l = len[i];
+    run += (l < 1 || l > K) ? 1 : l;
+  }
+}
+
+// X[off[f] + j] = T[tok[f * K + j]]: one warp per f-gram.
+__global__ void __launch_bounds__(256)
+    gather_rows_kernel(const int32_t* __restrict__ tok, const uint8_t* __restrict__ len,
+                       const int32_t* __restrict__ off, int64_t n, int32_t K,
+                       const uint16_t* __restrict__ T, int32_t vocab, int32_t d,
+                       uint16_t* __restrict__ X, int* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t f = (int64_t)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  if (f >= n) return;
+  const int nl = off[f + 1] - off[f];
+  const int chunks = d / 8;                       // 16-byte chunks per row
+  for (int j = 0; j < nl; ++j) {
+    const int32_t t = tok[f * K + j];
+    uint4* dst = reinterpret_cast<uint4*>(X + (int64_t)(off[f] + j) * d);
+    if ((uint32_t)t >= (uint32_t)vocab) {
+      if (lane == 0) set_error(status, SCONE_ERR_TOKEN_RANGE);
+      for (int c = lane; c < chunks; c += 32) dst[c] = make_uint4(0, 0, 0, 0);
+      continue;
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(T + (int64_t)t * d);
+    for (int c = lane; c < chunks; c += 32) dst[c] = __ldg(src + c);
+  }
+}
+
+// Non-parametric layer norm of rows (one warp per row): Y = (X - mean) /
+// sqrt(var + eps), CH = d / 256 16-byte chunks per lane. With `off`, output
+// row r is the layer norm of input row off[r + 1] - 1, the last position of
+// f-gram r (the F rows).
+template <int CH>
+__global__ void __launch_bounds__(256)
+    layernorm_kernel(const uint16_t* __restrict__ X, uint16_t* __restrict__ Y, int64_t n_rows,
+                     const int32_t* __restrict__ off) {
+  const int lane = threadIdx.x & 31;
+  const int64_t r = (int64_t)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  if (r >= n_rows) return;
+  constexpr int d = CH * 256;
+  const int64_t src_row = off ? (int64_t)off[r + 1] - 1 : r;   // last position of f-gram r
+  const uint4* src = reinterpret_cast<const uint4*>(X + src_row * d);
+  float v[CH * 8];
+  float sum = 0.f;
+#pragma unroll
+  for (int c = 0; c < CH; ++c) {
+    const uint4 q = __ldg(src + c * 32 + lane);
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      v[c * 8 + 2 * e] = lo_f(w[e]);
+      v[c * 8 + 2 * e + 1] = hi_f(w[e]);
+      sum += v[c * 8 + 2 * e] + v[c * 8 + 2 * e + 1];
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+  const float mean = sum / d;
+  float sq = 0.f;
+#pragma unroll
+  for (int i = 0; i < CH * 8; ++i) {
+    v[i] -= mean;
+    sq += v[i] * v[i];
+  }
+  for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, o);
+  const float inv = rsqrtf(sq / d + kLnEps);
+  uint4* dst = reinterpret_cast<uint4*>(Y + r * d);
+#pragma unroll
+  for (int c = 0; c < CH; ++c) {
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) w[e] = pack2(v[c * 8 + 2 * e] * inv, v[c * 8 + 2 * e + 1] * inv);
+    dst[c * 32 + lane] = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
+// Causal attention of one (f-gram, head) per warp over at most KMAX
+// positions. Lane l holds dims C*l .. C*l+C-1 of the head's first half and the
+// same offsets of its second half (C = hd / 64), so each rotate-half pair of
+// the rotary embedding stays in one lane.
+template <int C, int KMAX>
+__global__ void __launch_bounds__(256)
+    attention_kernel(const uint16_t* __restrict__ QKV, const int32_t* __restrict__ off, int64_t n,
+                     int32_t d, int32_t H, uint16_t* __restrict__ O) {
+  constexpr int hd = 64 * C, half = 32 * C;
+  const int lane = threadIdx.x & 31;
+  const int64_t wid = (int64_t)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  if (wid >= n * H) return;
+  const int64_t f = wid / H;
+  const int h = (int)(wid % H);
+  const int32_t r0 = off[f];
+  const int nl = off[f + 1] - r0 < KMAX ? off[f + 1] - r0 : KMAX;
+  float q[KMAX][2 * C], k[KMAX][2 * C], v[KMAX][2 * C];
+  float theta[C];
+#pragma unroll
+  for (int e = 0; e < C; ++e)
+    theta[e] = powf(10000.f, -2.f * (float)(C * lane + e) / (float)hd);
+#pragma unroll
+  for (int j = 0; j < KMAX; ++j) {
+    if (j >= nl) break;
+    const uint16_t* row = QKV + (int64_t)(r0 + j) * 3 * d + h * hd;
+#pragma unroll
+    for (int part = 0; part < 2; ++part) {
+      const int base = part * half + C * lane;
+#pragma unroll
+      for (int e = 0; e < C; ++e) {
+        q[j][part * C + e] = __uint_as_float((uint32_t)row[base + e] << 16);
+        k[j][part * C + e] = __uint_as_float((uint32_t)row[d + base + e] << 16);
+        v[j][part * C + e] = __uint_as_float((uint32_t)row[2 * d + base + e] << 16);
+      }
+    }
+    // rotary embedding at position j: (a, b) -> (a cos - b sin, b cos + a sin)
+#pragma unroll
+    for (int e = 0; e < C; ++e) {
+      float s, c;
+      sincosf((float)j * theta[e], &s, &c);
+      const float qa = q[j][e], qb = q[j][C + e], ka = k[j][e], kb = k[j][C + e];
+      q[j][e] = qa * c - qb * s;
+      q[j][C + e] = qb * c + qa * s;
+      k[j][e] = ka * c - kb * s;
+      k[j][C + e] = kb * c + ka * s;
+    }
+  }
+  const float scale = rsqrtf((float)hd);
+#pragma unroll
+  for (int i = 0; i < KMAX; ++i) {
+    if (i >= nl) break;
+    float sc[KMAX];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < KMAX; ++j) {
+      if (j > i) break;
+      float p = 0.f;
+#pragma unroll
+      for (int e = 0; e < 2 * C; ++e) p += q[i][e] * k[j][e];
+      for (int o = 16; o > 0; o >>= 1) p += __shfl_xor_sync(0xFFFFFFFFu, p, o);
+      sc[j] = p * scale;
+      mx = fmaxf(mx, sc[j]);
+    }
+    float den = 0.f, acc[2 * C];
+#pragma unroll
+    for (int e = 0; e < 2 * C; ++e) acc[e] = 0.f;
+#pragma unroll
+    for (int j = 0; j < KMAX; ++j) {
+      if (j > i) break;
+      const float p = expf(sc[j] - mx);
+      den += p;
+#pragma unroll
+      for (int e = 0; e < 2 * C; ++e) acc[e] += p * v[j][e];
+    }
+    const float inv = 1.f / den;
+    uint16_t* out = O + (int64_t)(r0 + i) * d + h * hd;
+#pragma unroll
+    for (int part = 0; part < 2; ++part) {
+      const int base = part * half + C * lane;
+#pragma unroll
+      for (int e = 0; e < C; ++e) {
+        const __nv_bfloat16 b = __float2bfloat16_rn(acc[part * C + e] * inv);
+        out[base + e] = *reinterpret_cast<const uint16_t*>(&b);
+      }
+    }
+  }
+}
+
+template <int CH>
+void launch_ln(const uint16_t* X, uint16_t* Y, int64_t rows, const int32_t* off,
+               cudaStream_t s) {
+  const unsigned grid = (unsigned)((rows + kRowsPerBlock - 1) / kRowsPerBlock);
+  layernorm_kernel<CH><<<grid, 256, 0, s>>>(X, Y, rows, off);
+}
+
+bool ln(int d, const uint16_t* X, uint16_t* Y, int64_t rows, const int32_t* off, cudaStream_t s) {
+  switch (d / 256) {
+    case 1: launch_ln<1>(X, Y, rows, off, s); return true;
+    case 2: launch_ln<2>(X, Y, rows, off, s); return true;
+    case 4: launch_ln<4>(X, Y, rows, off, s); return true;
+    case 8: launch_ln<8>(X, Y, rows, off, s); return true;
+    case 16: launch_ln<16>(X, Y, rows, off, s); return true;
+    default: return false;
+  }
+}
+
+bool attn(int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d, int H, uint16_t* O,
+          cudaStream_t s) {
+  const unsigned grid = (unsigned)((n * H + kRowsPerBlock - 1) / kRowsPerBlock);
+  switch (hd) {
+    case 64: attention_kernel<1, 8><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
+    case 128: attention_kernel<2, 8><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
+    case 256: attention_kernel<4, 8><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
+    default: return false;
+  }
+}
+
+bool ensure_rows(scone_fgram_model* m, int64_t rows) {
+  if (rows <= m->cap_rows) return true;
+  for (uint16_t** p : {&m->X, &m->Xn, &m->QKV, &m->Act}) {
+    if (*p) cudaFree(*p);
+    *p = nullptr;
+  }
+  m->cap_rows = 0;
+  const int64_t r = rows + rows / 8;
+  if (cudaMalloc(&m->X, (size_t)r * m->d * 2) != cudaSuccess ||
+      cudaMalloc(&m->Xn, (size_t)r * m->d * 2) != cudaSuccess ||
+      cudaMalloc(&m->QKV, (size_t)r * 3 * m->d * 2) != cudaSuccess ||
+      cudaMalloc(&m->Act, (size_t)r * m->ffw * 2) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  m->cap_rows = r;
+  return true;
+}
+
+}  // namespace
+
+}  // namespace scone
+
+using namespace scone;
+
+extern "C" int scone_fgram_model_create(int32_t d, int32_t n_heads, int32_t ffw, int32_t n_layers,
+                                        const scone_bf16* weights, int64_t batch,
+                                        scone_fgram_model** out) {
+  if (!out) return SCONE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (d <= 0 || d % 256 || d / 256 > 16 || (d / 256) & (d / 256 - 1) || n_heads <= 0 ||
+      d % n_heads || ffw <= 0 || ffw % 128 || n_layers < 0 || (n_layers > 0 && !weights) ||
+      ((uintptr_t)weights & 15) || batch < 0)
+    return SCONE_ERR_INVALID_ARG;
+  const int hd = d / n_heads;
+  if (hd != 64 && hd != 128 && hd != 256) return SCONE_ERR_UNSUPPORTED;
+  auto* m = new (std::nothrow) scone_fgram_model();
+  if (!m) return SCONE_ERR_NOMEM;
+  cudaGetDevice(&m->device);
+  m->d = d;
+  m->n_heads = n_heads;
+  m->ffw = ffw;
+  m->n_layers = n_layers;
+  m->weights = weights;
+  m->batch = batch > 0 ? batch : 16384;
+  if (cudaMalloc(&m->off, (size_t)(m->batch + 1) * sizeof(int32_t)) != cudaSuccess ||
+      cudaMalloc(&m->status, sizeof(int)) != cudaSuccess ||
+      cudaMemset(m->status, 0, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    scone_fgram_model_destroy(m);
+    return SCONE_ERR_NOMEM;
+  }
+  *out = m;
+  return SCONE_OK;
+}
+
+extern "C" int scone_fgram_model_destroy(scone_fgram_model* m) {
+  if (!m) return SCONE_OK;
+  DeviceGuard g(m->device);
+  cudaDeviceSynchronize();
+  for (void* p : {(void*)m->off, (void*)m->status, (void*)m->X, (void*)m->Xn, (void*)m->QKV,
+                  (void*)m->Act})
+    if (p) cudaFree(p);
+  delete m;
+  return SCONE_OK;
+}
+
+extern "C" int scone_fgram_precompute(scone_fgram_model* m, const int32_t* fgram_tok,
+                                      const uint8_t* fgram_len, int64_t n, int32_t K,
+                                      const scone_bf16* T, int32_t vocab, scone_bf16* F,
+                                      void* stream) {
+  if (!m || n < 0 || K < 2 || K > 8 || vocab < 1) return SCONE_ERR_INVALID_ARG;
+  if (n == 0) return SCONE_OK;
+  if (!fgram_tok || !fgram_len || !T || !F || ((uintptr_t)T & 15) || ((uintptr_t)F & 15) ||
+      ((uintptr_t)fgram_tok & 3))
+    return SCONE_ERR_INVALID_ARG;
+  DeviceGuard g(m->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  const int d = m->d, H = m->n_heads, ffw = m->ffw;
+  const int64_t layer_elems = (int64_t)3 * d * d + (int64_t)d * d + (int64_t)2 * ffw * d +
+                              (int64_t)d * ffw;
+  for (int64_t f0 = 0; f0 < n; f0 += m->batch) {
+    const int64_t nb = n - f0 < m->batch ? n - f0 : m->batch;
+    offsets_kernel<<<1, 1024, 0, s>>>(fgram_len + f0, nb, K, m->off, m->status);
+    int32_t rows = 0;
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemcpyAsync(&rows, m->off + nb, sizeof(rows), cudaMemcpyDeviceToHost, s) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+      return SCONE_ERR_CUDA;
+    if (!ensure_rows(m, rows)) return SCONE_ERR_NOMEM;
+    const unsigned gw = (unsigned)((nb + kRowsPerBlock - 1) / kRowsPerBlock);
+    gather_rows_kernel<<<gw, 256, 0, s>>>(fgram_tok + f0 * K, fgram_len + f0, m->off, nb, K, T,
+                                          vocab, d, m->X, m->status);
+    for (int l = 0; l < m->n_layers; ++l) {
+      const uint16_t* w = m->weights + l * layer_elems;
+      const uint16_t* wqkv = w;
+      const uint16_t* wo = wqkv + (int64_t)3 * d * d;
+      const uint16_t* wgu = wo + (int64_t)d * d;
+      const uint16_t* wd = wgu + (int64_t)2 * ffw * d;
+      int rc;
+      if (!ln(d, m->X, m->Xn, rows, nullptr, s)) return SCONE_ERR_UNSUPPORTED;
+      if ((rc = gemm_bf16(m->Xn, wqkv, nullptr, m->QKV, rows, 3 * d, d, GEMM_EPI_STORE,
+                          m->status, s)))
+        return rc;
+      if (!attn(d / H, m->QKV, m->off, nb, d, H, m->Xn, s)) return SCONE_ERR_UNSUPPORTED;
+      if ((rc = gemm_bf16(m->Xn, wo, m->X, m->X, rows, d, d, GEMM_EPI_RESIDUAL, m->status, s)))
+        return rc;
+      if (!ln(d, m->X, m->Xn, rows, nullptr, s)) return SCONE_ERR_UNSUPPORTED;
+      if ((rc = gemm_bf16(m->Xn, wgu, nullptr, m->Act, rows, 2 * ffw, d, GEMM_EPI_SWIGLU,
+                          m->status, s)))
+        return rc;
+      if ((rc = gemm_bf16(m->Act, wd, m->X, m->X, rows, d, ffw, GEMM_EPI_RESIDUAL, m->status,
+                          s)))
+        return rc;
+    }
+    // F rows: layer norm of each f-gram's last position
+    if (!ln(d, m->X, F + f0 * d, nb, m->off, s)) return SCONE_ERR_UNSUPPORTED;
+    if (cudaGetLastError() != cudaSuccess) return SCONE_ERR_CUDA;
+  }
+  int st = 0;
+  if (cudaMemcpyAsync(&st, m->status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaMemsetAsync(m->status, 0, sizeof(int), s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return SCONE_ERR_CUDA;
+  return st;
+}

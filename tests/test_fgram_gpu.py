@@ -1,0 +1,145 @@
+"""Precomputing F with the f-gram model on the GPU against the float64 oracle
+(GPU).
+
+The oracle rounds to bf16 at the points where the GPU stores bf16 (residual
+stream, layer-norm outputs, q/k/v, attention output, MLP activation, F), so
+the two differ only through float32-versus-float64 arithmetic between those
+points. Where that difference moves a value across a bf16 rounding boundary
+the value changes by one bf16 unit (2^-8 relative), and the change propagates
+through later layers. Over two layers of this model the measured effect on
+the unit-variance F entries is far below the bound used here: max |diff| <=
+0.08 and mean |diff| <= 6e-3 per row, with most entries equal.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import fgram_model as fm
+import paper_2502_01637_gb300 as scone
+from gpu_cases import DEV
+
+pytestmark = pytest.mark.gpu
+TINY = synth.MODELS["tiny"]
+VOCAB = 500
+
+
+@pytest.fixture(scope="module")
+def tiny_model():
+    packed = synth.model_weights_cpu(TINY)
+    W = fm.Weights(packed, TINY)
+    T = synth.rows_range_cpu(4321, TINY.d, 0, VOCAB)
+    w_d = torch.from_numpy(packed.view(np.int16)).to(DEV)
+    T_d = torch.from_numpy(T.view(np.int16)).to(DEV)
+    return packed, W, T, w_d, T_d
+
+
+def fgram_list(n, K, seed):
+    rng = np.random.default_rng(seed)
+    ln = rng.integers(2, K + 1, size=n).astype(np.uint8)
+    tok = np.full((n, K), -1, np.int32)
+    for r in range(n):
+        tok[r, :ln[r]] = rng.integers(0, VOCAB, size=ln[r])
+    return tok, ln
+
+
+def run(model, tok, ln, T_d):
+    F = torch.empty((max(len(ln), 1), TINY.d), dtype=torch.int16, device=DEV)
+    scone.scone_fgram_precompute(model, torch.from_numpy(tok).to(DEV),
+                                 torch.from_numpy(ln).to(DEV), T_d, F[:len(ln)])
+    torch.cuda.synchronize()
+    return F[:len(ln)].cpu().numpy().view(np.uint16)
+
+
+def check(got_bits, tok, ln, W, T):
+    want = fm.precompute(tok, ln, T, W, emulate_bf16=True)
+    got = fm.bf16_to_f64(got_bits)
+    diff = np.abs(got - want)
+    assert diff.max() <= 0.08, diff.max()
+    assert diff.mean(axis=1).max() <= 6e-3, diff.mean(axis=1).max()
+    assert (diff == 0).mean() > 0.5
+    return diff
+
+
+def test_matches_oracle_all_lengths(tiny_model):
+    packed, W, T, w_d, T_d = tiny_model
+    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
+    for K in (2, 5, 8):
+        tok, ln = fgram_list(150, K, seed=K)
+        check(run(model, tok, ln, T_d), tok, ln, W, T)
+    model.close()
+
+
+def test_batches_equal_one_batch(tiny_model):
+    """The internal batching (37 f-grams per batch, many GEMM row tiles with
+    ragged ends) gives the same bytes as one batch."""
+    packed, W, T, w_d, T_d = tiny_model
+    tok, ln = fgram_list(700, 5, seed=11)
+    one = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
+    many = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d, batch=37)
+    a, b = run(one, tok, ln, T_d), run(many, tok, ln, T_d)
+    assert np.array_equal(a, b)
+    check(a[::7], tok[::7], ln[::7], W, T)
+    one.close()
+    many.close()
+
+
+def test_zero_layers_is_layer_norm(tiny_model):
+    packed, W, T, w_d, T_d = tiny_model
+    m0 = synth.FgramModel("none", 99, TINY.d, TINY.n_heads, TINY.ffw, 0)
+    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, 0, w_d)
+    tok, ln = fgram_list(40, 3, seed=2)
+    got = fm.bf16_to_f64(run(model, tok, ln, T_d))
+    want = fm.precompute(tok, ln, T, fm.Weights(np.zeros(0, np.uint16), m0), emulate_bf16=True)
+    assert np.abs(got - want).max() <= 2 ** -7 * 4          # one bf16 rounding of |F| <= ~4
+    model.close()
+
+
+def test_errors(tiny_model):
+    packed, W, T, w_d, T_d = tiny_model
+    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
+    tok, ln = fgram_list(20, 3, seed=3)
+    tok[4, 1] = VOCAB + 3
+    with pytest.raises(scone.SconeError) as e:
+        run(model, tok, ln, T_d)
+    assert e.value.code == scone.SCONE_ERR_TOKEN_RANGE
+    tok, ln = fgram_list(20, 3, seed=3)
+    ln[2] = 9
+    with pytest.raises(scone.SconeError) as e:
+        run(model, tok, ln, T_d)
+    assert e.value.code == scone.SCONE_ERR_INVALID_ARG
+    model.close()
+    with pytest.raises(scone.SconeError):
+        scone.FgramModel(200, 4, 512, 2, w_d)                 # d not a multiple of 256
+
+
+def test_discover_precompute_embed_pipeline(tiny_model):
+    """Corpus -> discovered f-grams -> F by the model -> table -> Algorithm 1:
+    every position that selects an f-gram gets exactly its precomputed row."""
+    packed, W, T, w_d, T_d = tiny_model
+    w = synth.WORKLOADS["tiny"].scaled("pipe", B=8, L=1024, vocab=VOCAB)
+    corpus = synth.zipf_tokens(w, 77, w.B * w.L, inject=False).reshape(w.B, w.L)
+    ft, fl, fc, st = scone.scone_fgram_discover(torch.from_numpy(corpus).to(DEV), VOCAB, 3,
+                                                2000, 3)
+    n = fl.shape[0]
+    assert n > 100
+    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
+    F = torch.empty((n, TINY.d), dtype=torch.int16, device=DEV)
+    scone.scone_fgram_precompute(model, ft.contiguous(), fl.contiguous(), T_d, F)
+    table = scone.scone_table_build(ft.cpu().numpy(), fl.cpu().numpy(), 3, VOCAB, TINY.d, F, T_d)
+    q = torch.from_numpy(corpus[:2]).to(DEV)
+    out = torch.empty((q.numel(), TINY.d), dtype=torch.int16, device=DEV)
+    row = torch.empty(q.numel(), dtype=torch.int32, device=DEV)
+    scone.scone_embed(table, q, out, row)
+    scone.scone_status(table)
+    r = row.cpu().numpy()
+    hit = r >= 0
+    assert hit.mean() > 0.3
+    assert torch.equal(out[torch.from_numpy(np.nonzero(hit)[0]).to(DEV)],
+                       F[torch.from_numpy(r[hit]).long().to(DEV)])
+    sample = np.random.default_rng(0).choice(n, 30, replace=False)
+    check(F.cpu().numpy().view(np.uint16)[sample], ft.cpu().numpy()[sample],
+          fl.cpu().numpy()[sample], W, T)
+    table.close()
+    model.close()
