@@ -3,19 +3,23 @@
 // row-major with K contiguous (activations x weights), fp32 accumulation in
 // tensor memory.
 //
-// One CTA computes a 128 x 256 tile of C with 4 warps:
-//   * thread 0 streams K-slices of 64 (A: 128 x 64, B: 256 x 64, 48 KB) into a
+// Tiles of 128 x 256, persistent (one CTA per SM walks its share of the
+// tiles in a grouped order: 8 row tiles at a time sweep every column tile, so
+// the tiles in flight share their A and B slices in L2), warp-specialized:
+//   * warp 0 streams K-slices of 64 (A: 128 x 64, B: 256 x 64, 48 KB) into a
 //     ring of kStages shared-memory stages with TMA (cp.async.bulk.tensor,
 //     128-byte swizzle), each stage completed on an mbarrier by byte count;
-//   * thread 32 issues tcgen05.mma (M = 128, N = 256, K = 16, bf16 x bf16 ->
-//     fp32) over each stage, four per slice, accumulating into 256 columns
-//     of tensor memory, and releases the stage with tcgen05.commit;
-//   * after the last commit all four warps read the accumulator back with
-//     tcgen05.ld (warp w owns tensor-memory lanes 32w .. 32w + 31, i.e. rows)
-//     and apply the epilogue: store, add a residual, or SwiGLU of interleaved
-//     gate/up column pairs.
+//   * warp 1 issues tcgen05.mma (M = 128, N = 256, K = 16, bf16 x bf16 ->
+//     fp32), four per slice, into one of two 256-column accumulators in
+//     tensor memory, frees each stage with tcgen05.commit and hands a
+//     finished accumulator to the epilogue with another commit;
+//   * warps 2..5 read the other accumulator back with tcgen05.ld (warp w owns
+//     tensor-memory lanes 32 (w % 4) .. + 31, i.e. rows) and apply the
+//     epilogue: store, add a residual, or SwiGLU of interleaved gate/up
+//     column pairs; then they release the accumulator.
+// So the epilogue of one tile overlaps the main loop of the next.
 // Every mbarrier wait is bounded (kGemmSpin polls); past it the CTA records
-// SCONE_ERR_CUDA, stops issuing, drains what it issued, frees its tensor
+// SCONE_ERR_CUDA, stops issuing, waits for what it issued, frees its tensor
 // memory and returns.
 
 #include <cuda.h>
@@ -34,11 +38,13 @@ namespace {
 
 constexpr int kBM = 128, kBN = 256, kBK = 64;
 constexpr int kStages = 4;
-constexpr int kGemmThreads = 128;
+constexpr int kEpiWarps = 4;
+constexpr int kGemmThreads = 32 * (2 + kEpiWarps);   // loader, MMA issuer, 4 epilogue warps
+constexpr int kGroupM = 8;                            // row tiles per group of the tile order
 constexpr uint32_t kStageA = kBM * kBK * 2;   // 16 KB
 constexpr uint32_t kStageB = kBN * kBK * 2;   // 32 KB
 constexpr uint32_t kStageBytes = kStageA + kStageB;
-constexpr uint32_t kTmemCols = kBN;           // fp32 accumulator: 256 columns x 128 lanes
+constexpr uint32_t kTmemCols = 2 * kBN;       // two fp32 accumulators of 256 columns x 128 lanes
 constexpr uint32_t kGemmSpin = 1u << 22;   // polls; each try_wait may also suspend briefly
 constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + 1024 /* align */ + 256 /* barriers */;
 
@@ -139,6 +145,69 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// Tile t of the grouped order: kGroupM row tiles at a time sweep all column
+// tiles, so the CTAs running at once share a few A tiles and a few B tiles in
+// L2 instead of each streaming its own A.
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int* m_tile,
+                                            int* n_tile) {
+  const int per_group = kGroupM * num_n;
+  const int first_m = (t / per_group) * kGroupM;
+  const int gm = num_m - first_m < kGroupM ? num_m - first_m : kGroupM;
+  const int local = t % per_group;
+  *m_tile = first_m + local % gm;
+  *n_tile = local / gm;
+}
+
+// Epilogue of one 32-column chunk of one row: v holds columns c .. c+31 of
+// the accumulator row.
+template <int EPI>
+__device__ __forceinline__ void store_chunk(const float (&v)[32], int row, int col,
+                                            const uint16_t* __restrict__ R,
+                                            uint16_t* __restrict__ C, int ldc) {
+  if constexpr (EPI == GEMM_EPI_SWIGLU) {
+    // 16 gates then 16 ups of outputs col / 2 ..
+    uint32_t o[8];
+#pragma unroll
+    for (int j = 0; j < 16; j += 2) {
+      const float g0 = v[j], g1 = v[j + 1], u0 = v[16 + j], u1 = v[17 + j];
+      o[j / 2] = pack_bf16(g0 / (1.f + expf(-g0)) * u0, g1 / (1.f + expf(-g1)) * u1);
+    }
+    uint4* dst = reinterpret_cast<uint4*>(C + (int64_t)row * ldc + col / 2);
+    dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+    dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+  } else {
+    uint32_t o[16];
+    if constexpr (EPI == GEMM_EPI_RESIDUAL) {
+      const uint4* src = reinterpret_cast<const uint4*>(R + (int64_t)row * ldc + col);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 r4 = src[q];
+        const uint32_t rw[4] = {r4.x, r4.y, r4.z, r4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int j = q * 8 + e * 2;
+          o[q * 4 + e] = pack_bf16(v[j] + bf16_lo(rw[e]), v[j + 1] + bf16_hi(rw[e]));
+        }
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; j += 2) o[j / 2] = pack_bf16(v[j], v[j + 1]);
+    }
+    uint4* dst = reinterpret_cast<uint4*>(C + (int64_t)row * ldc + col);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      dst[q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+  }
+}
+
+// Persistent, warp-specialized: warp 0 loads (TMA), warp 1 issues the MMAs
+// into one of two tensor-memory accumulators, warps 2..5 drain the other
+// accumulator through the epilogue, so the epilogue of tile i overlaps the
+// main loop of tile i + 1.
 template <int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap map_a,
@@ -150,12 +219,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint8_t* gsm = reinterpret_cast<uint8_t*>(((uintptr_t)gsm_raw + 1023) & ~(uintptr_t)1023);
   uint64_t* full = reinterpret_cast<uint64_t*>(gsm + kStages * kStageBytes);
   uint64_t* empty = full + kStages;
-  uint64_t* done = empty + kStages;
+  uint64_t* tfull = empty + kStages;     // [2] accumulator ready (MMA -> epilogue)
+  uint64_t* tempty = tfull + 2;          // [2] accumulator drained (epilogue -> MMA)
+  uint64_t* done = tempty + 2;           // every issued MMA completed
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   __shared__ int failed;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * kBN;
+  const int num_m = (M + kBM - 1) / kBM, num_n = N / kBN;
+  const int tiles = num_m * num_n;
   const int kt_n = K / kBK;
 
   if (threadIdx.x == 0) {
@@ -164,11 +236,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_init(saddr(&full[s]), 1);
       mbar_init(saddr(&empty[s]), 1);
     }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(saddr(&tfull[a]), 1);
+      mbar_init(saddr(&tempty[a]), kEpiWarps);
+    }
     mbar_init(saddr(done), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncwarp();
-  if (warp == 0) {
+  if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      saddr(tmem_slot)),
                  "r"(kTmemCols)
@@ -179,107 +255,96 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
+  volatile int* vfailed = &failed;
 
-  if (threadIdx.x == 0) {
-    // producer: K-slices into the ring
-    int issued = 0;
-    for (int kt = 0; kt < kt_n; ++kt) {
-      const int s = kt % kStages;
-      if (kt >= kStages && !mbar_wait(saddr(&empty[s]), ((kt / kStages) - 1) & 1)) {
-        atomicExch(&failed, 1);
-        break;
+  if (warp == 0) {
+    if (lane == 0) {
+      // producer: K-slices of every tile of this CTA into the ring
+      int it = 0;
+      for (int t = blockIdx.x; t < tiles && !*vfailed; t += gridDim.x) {
+        int mt, nt;
+        tile_coords(t, num_m, num_n, &mt, &nt);
+        for (int kt = 0; kt < kt_n; ++kt, ++it) {
+          const int s = it % kStages;
+          if (it >= kStages && !mbar_wait(saddr(&empty[s]), ((it / kStages) - 1) & 1)) {
+            *vfailed = 1;
+            break;
+          }
+          if (*vfailed) break;
+          const uint32_t a_dst = saddr(gsm + s * kStageBytes);
+          mbar_expect_tx(saddr(&full[s]), kStageBytes);
+          tma_load_2d(a_dst, &map_a, kt * kBK, mt * kBM, saddr(&full[s]));
+          tma_load_2d(a_dst + kStageA, &map_b, kt * kBK, nt * kBN, saddr(&full[s]));
+        }
       }
-      if (*reinterpret_cast<volatile int*>(&failed)) break;
-      const uint32_t a_dst = saddr(gsm + s * kStageBytes);
-      const uint32_t b_dst = a_dst + kStageA;
-      mbar_expect_tx(saddr(&full[s]), kStageBytes);
-      tma_load_2d(a_dst, &map_a, kt * kBK, m0, saddr(&full[s]));
-      tma_load_2d(b_dst, &map_b, kt * kBK, n0, saddr(&full[s]));
-      ++issued;
+      // drain: the last issued slices must have landed before the CTA exits
+      for (int j = it - kStages < 0 ? 0 : it - kStages; j < it; ++j)
+        mbar_wait(saddr(&full[j % kStages]), (j / kStages) & 1);
     }
-    // drain: every issued slice must have landed before the CTA may exit
-    for (int kt = 0; kt < issued; ++kt)
-      if (kt + kStages >= issued) mbar_wait(saddr(&full[kt % kStages]), (kt / kStages) & 1);
-  } else if (threadIdx.x == 32) {
-    // MMA issuer
-    bool ok = true;
-    for (int kt = 0; kt < kt_n && ok; ++kt) {
-      const int s = kt % kStages;
-      if (!mbar_wait(saddr(&full[s]), (kt / kStages) & 1) ||
-          *reinterpret_cast<volatile int*>(&failed)) {
-        atomicExch(&failed, 1);
-        ok = false;
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // MMA issuer
+      int it = 0, lt = 0;
+      for (int t = blockIdx.x; t < tiles && !*vfailed; t += gridDim.x, ++lt) {
+        const int acc = lt & 1;
+        if (lt >= 2 && !mbar_wait(saddr(&tempty[acc]), ((lt >> 1) - 1) & 1)) {
+          *vfailed = 1;
+          break;
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t d_tmem = tmem + acc * kBN;
+        bool ok = true;
+        for (int kt = 0; kt < kt_n; ++kt, ++it) {
+          const int s = it % kStages;
+          if (!mbar_wait(saddr(&full[s]), (it / kStages) & 1) || *vfailed) {
+            *vfailed = 1;
+            ok = false;
+            break;
+          }
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t a_base = saddr(gsm + s * kStageBytes);
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            umma_bf16(d_tmem, desc_k128(a_base + 32 * k), desc_k128(a_base + kStageA + 32 * k),
+                      (kt > 0 || k > 0) ? 1u : 0u);
+          umma_commit(saddr(&empty[s]));
+        }
+        if (!ok) break;
+        umma_commit(saddr(&tfull[acc]));
+      }
+      umma_commit(saddr(done));   // arrives when every MMA issued above has completed
+      mbar_wait(saddr(done), 0);
+    }
+  } else {
+    // epilogue warps: warp w reads tensor-memory lanes 32 (w % 4) .. + 31
+    const int q = warp & 3;
+    int lt = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
+      const int acc = lt & 1;
+      const bool ok = mbar_wait(saddr(&tfull[acc]), (lt >> 1) & 1);
+      if (!ok || *vfailed) {
+        *vfailed = 1;
         break;
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const uint32_t a_base = saddr(gsm + s * kStageBytes);
-      const uint32_t b_base = a_base + kStageA;
-#pragma unroll
-      for (int k = 0; k < kBK / 16; ++k)
-        umma_bf16(tmem, desc_k128(a_base + 32 * k), desc_k128(b_base + 32 * k),
-                  (kt > 0 || k > 0) ? 1u : 0u);
-      umma_commit(saddr(&empty[s]));
-    }
-    umma_commit(saddr(done));   // arrives once every MMA issued above has completed
-  }
-  __syncwarp();
-
-  // epilogue: all 128 threads, one accumulator row (tensor-memory lane) each
-  const bool ok = mbar_wait(saddr(done), 0);
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-  if (!ok) atomicExch(&failed, 1);
-  __syncthreads();
-  if (failed) {
-    if (threadIdx.x == 0) atomicCAS(status, 0, (int)SCONE_ERR_CUDA);
-  } else {
-    const int row = m0 + warp * 32 + lane;
-    const uint32_t t_row = tmem + ((uint32_t)(warp * 32) << 16);
+      int mt, nt;
+      tile_coords(t, num_m, num_n, &mt, &nt);
+      const int row = mt * kBM + q * 32 + lane;
+      const uint32_t t_row = tmem + acc * kBN + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
-    for (int c0 = 0; c0 < kBN; c0 += 32) {
-      float v[32];
-      tmem_ld32(t_row + c0, v);   // every lane takes part (.sync.aligned)
-      if (row >= M) {
-      } else if constexpr (EPI == GEMM_EPI_SWIGLU) {
-        // 32 columns = 16 gates then 16 ups of outputs (n0 + c0) / 2 ..
-        uint32_t o[8];
-#pragma unroll
-        for (int j = 0; j < 16; j += 2) {
-          const float g0 = v[j], g1 = v[j + 1], u0 = v[16 + j], u1 = v[17 + j];
-          const float a0 = g0 / (1.f + expf(-g0)) * u0;
-          const float a1 = g1 / (1.f + expf(-g1)) * u1;
-          o[j / 2] = pack_bf16(a0, a1);
-        }
-        uint4* dst = reinterpret_cast<uint4*>(C + (int64_t)row * ldc + (n0 + c0) / 2);
-        dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
-        dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
-      } else {
-        uint32_t o[16];
-        if constexpr (EPI == GEMM_EPI_RESIDUAL) {
-          const uint4* src = reinterpret_cast<const uint4*>(R + (int64_t)row * ldc + n0 + c0);
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const uint4 r4 = src[q];
-            const uint32_t rw[4] = {r4.x, r4.y, r4.z, r4.w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int j = q * 8 + e * 2;
-              o[q * 4 + e] = pack_bf16(v[j] + bf16_lo(rw[e]), v[j + 1] + bf16_hi(rw[e]));
-            }
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < 32; j += 2) o[j / 2] = pack_bf16(v[j], v[j + 1]);
-        }
-        uint4* dst = reinterpret_cast<uint4*>(C + (int64_t)row * ldc + n0 + c0);
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          dst[q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+      for (int c0 = 0; c0 < kBN; c0 += 32) {
+        float v[32];
+        tmem_ld32(t_row + c0, v);   // every lane takes part (.sync.aligned)
+        if (row < M) store_chunk<EPI>(v, row, nt * kBN + c0, R, C, ldc);
       }
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(saddr(&tempty[acc]));
     }
   }
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
-  if (warp == 0)
+  if (*vfailed && threadIdx.x == 0) atomicCAS(status, 0, (int)SCONE_ERR_CUDA);
+  if (warp == 1)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(kTmemCols)
                  : "memory");
@@ -340,7 +405,9 @@ int gemm_bf16(const uint16_t* A, const uint16_t* B, const uint16_t* R, uint16_t*
   if (M == 0) return SCONE_OK;
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, M, K, kBM) || !make_map(&mb, B, N, K, kBN)) return SCONE_ERR_CUDA;
-  const dim3 grid((unsigned)((M + kBM - 1) / kBM), (unsigned)(N / kBN));
+  const int64_t tiles = (int64_t)((M + kBM - 1) / kBM) * (N / kBN);
+  const int64_t sms = sm_count();
+  const dim3 grid((unsigned)(tiles < sms ? tiles : sms));
   const int ldc = epi == GEMM_EPI_SWIGLU ? N / 2 : N;
   switch (epi) {
     case GEMM_EPI_STORE:
