@@ -925,6 +925,68 @@ def bench_precompute(args, world, rank, local):
     return res
 
 
+def bench_gemm(args, world, rank, local):
+    """The tensor-core GEMM alone at the f-gram model's gate/up shape with the
+    SwiGLU epilogue (M = 16384 tokens, N = 2 ffw = 16384, K = d = 2048): the
+    case the ncu summaries of the kernel are taken on."""
+    import torch
+
+    import synth
+    import paper_2502_01637_gb300 as scone
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    M, N, K = 16384, 16384, 2048
+    A = torch.empty((M, K), dtype=torch.int16, device=dev)
+    B = torch.empty((N, K), dtype=torch.int16, device=dev)
+    synth.rows_gpu(5, K, 0, M, A.data_ptr(), stream.cuda_stream)
+    synth.rows_gpu(6, K, 0, N, B.data_ptr(), stream.cuda_stream)
+    C = torch.empty((M, N // 2), dtype=torch.int16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def step():
+        scone.scone_gemm_bf16(A, B, C, epilogue=scone.SCONE_GEMM_SWIGLU, status=status)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    with clocks:
+        for a, b in ev:
+            a.record(stream)
+            step()
+            b.record(stream)
+        torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    flops = 2.0 * M * N * K
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) \
+        if os.path.exists(os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
+    peak = float(peaks.get("bf16_tflops", 1900.0))
+    tf = flops / (ms * 1e-3) / 1e12
+    return {
+        "metric": "bf16 GEMM TFLOP/s at 1 GB300 (tcgen05, SwiGLU epilogue)",
+        "value": tf, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"gemm_profile: M={M}, N={N}, K={K}, C = silu(gate) up "
+                               f"[{M} x {N // 2}]",
+                   "l2": "operands 134 MB, output 268 MB (larger than L2); no flush"},
+        "roofline": {"bound": "tensor", "achieved": tf, "peak": peak, "unit": "TFLOP/s",
+                     "frac": tf / peak, "traffic": None,
+                     "peak_source": "measured (MEASURED_PEAKS.json bf16_tflops, burst)"
+                                    if peaks else "fallback",
+                     "kernel": "gemm_bf16_kernel<SWIGLU>",
+                     "algorithmic_flops_per_launch": flops},
+        "e2e": {"value": tf, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0, "what": "operands stay on the device"},
+        "gpu_launches": args.steps, "clocks": clocks.summary(),
+    }
+
+
 def cpu_baseline_precompute(m, fg_tok, fg_len, w, budget_s: float = 10.0):
     """The float64 oracle forward (numpy; its BLAS may use several threads) on
     the first f-grams of the same list, until about budget_s."""
@@ -1138,7 +1200,8 @@ def main():
     ap.add_argument("--workload", default="prefill_1b",
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
                              "offload_decode", "decode_profile", "prescan", "discover",
-                             "discover_k5", "discover_profile", "mixed_serving", "precompute"])
+                             "discover_k5", "discover_profile", "mixed_serving", "precompute",
+                             "gemm_profile"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
@@ -1162,6 +1225,8 @@ def main():
         res = bench_mixed(args, world, rank, local)
     elif args.workload == "precompute":
         res = bench_precompute(args, world, rank, local)
+    elif args.workload == "gemm_profile":
+        res = bench_gemm(args, world, rank, local)
     elif args.workload in ("discover", "discover_k5", "discover_profile"):
         res = bench_discover(args, world, rank, local)
     else:
