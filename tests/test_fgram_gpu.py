@@ -6,9 +6,11 @@ stream, layer-norm outputs, q/k/v, attention output, MLP activation, F), so
 the two differ only through float32-versus-float64 arithmetic between those
 points. Where that difference moves a value across a bf16 rounding boundary
 the value changes by one bf16 unit (2^-8 relative), and the change propagates
-through later layers. Over two layers of this model the measured effect on
-the unit-variance F entries is far below the bound used here: max |diff| <=
-0.08 and mean |diff| <= 6e-3 per row, with most entries equal.
+through later layers. Measured on GB300 over two layers of this model (300
+f-grams for each of K = 2, 5, 8): max |diff| 0.031 (one bf16 unit at |F| near
+4), largest row mean 0.0031, 87-92% of entries equal; the GPU is as close to
+exact float64 as the emulating oracle is (both about 0.0038 mean). Bound used
+here: max |diff| <= 0.08, row mean <= 6e-3, more than 75% of entries equal.
 """
 
 import numpy as np
@@ -58,7 +60,7 @@ def check(got_bits, tok, ln, W, T):
     diff = np.abs(got - want)
     assert diff.max() <= 0.08, diff.max()
     assert diff.mean(axis=1).max() <= 6e-3, diff.mean(axis=1).max()
-    assert (diff == 0).mean() > 0.5
+    assert (diff == 0).mean() > 0.75
     return diff
 
 
