@@ -362,6 +362,39 @@ int scone_fgram_precompute(scone_fgram_model* model, const int32_t* fgram_tok,
                            int32_t vocab, scone_bf16* F, void* stream);
 
 /*
+ * Row store: F in a file, beyond host memory (the paper's storage tier:
+ * f-gram embeddings on solid-state drives, Sec. 4.3). The file holds F row
+ * after row (n_rows x d bf16, no header). The store caches rows in HBM
+ * (cache_rows slots, direct-mapped by row id); a gather copies hits from the
+ * cache, reads misses from the file (pread on `threads` reader threads, 0 =
+ * one per core; O_DIRECT when a row is a multiple of 4 KiB) and fills the
+ * cache with them.
+ *
+ * scone_rowstore_open: d a multiple of 8; the file must hold n_rows rows.
+ * Synchronous. scone_rowstore_gather: out[t] = F[row[t]] (row[t] >= 0) or
+ * T[tok[t]] (row[t] < 0, T from the table, whose d must equal the store's);
+ * row as written by scone_match, scone_embed_varlen or scone_decode_step;
+ * tok, row device [n]; out device [n * d], 16-byte aligned. Synchronous (the
+ * host reads the misses). A row id >= n_rows or a token outside the vocab is
+ * a device-detected error (zero row, sticky table status); a failed read
+ * returns SCONE_ERR_CUDA.
+ */
+typedef struct scone_rowstore scone_rowstore;
+typedef struct scone_rowstore_stats {
+  int64_t positions;   /* positions gathered since open */
+  int64_t misses;      /* positions whose row was not in the cache */
+  int64_t rows_read;   /* distinct rows read from the file */
+  int64_t bytes_read;
+  int32_t direct_io;   /* 1 if the file is read with O_DIRECT */
+} scone_rowstore_stats;
+int scone_rowstore_open(const char* path, int64_t n_rows, int32_t d, int64_t cache_rows,
+                        int32_t threads, scone_rowstore** out);
+int scone_rowstore_gather(scone_rowstore* store, const scone_table* table, const int32_t* tok,
+                          const int32_t* row, int64_t n, scone_bf16* out, void* stream);
+int scone_rowstore_get_stats(const scone_rowstore* store, scone_rowstore_stats* out);
+int scone_rowstore_close(scone_rowstore* store);
+
+/*
  * Decode (Sec. 3.2: T stays on the accelerator "for decoding", F is looked
  * up per generated token). A decode state holds, per live sequence, its last
  * K-1 tokens on the device, which is all Algorithm 1 needs for the next
@@ -378,7 +411,9 @@ int scone_decode_create(const scone_table* table, int32_t S, const int32_t* hist
  * scone_decode_step: appends new_tok[s] (device int32 [S]) to sequence s,
  * embeds it by Algorithm 1 over the sequence so far, and writes
  * out device [S * d]; row device int32 [S] and len device uint8 [S] may be
- * NULL. Async; steps on one state must be ordered on one stream.
+ * NULL. out may be NULL when row is given: the step then only selects (for
+ * rows gathered from a row store, scone_rowstore_gather). Async; steps on
+ * one state must be ordered on one stream.
  */
 int scone_decode_step(scone_decode* state, const int32_t* new_tok, scone_bf16* out, int32_t* row,
                       uint8_t* len, void* stream);

@@ -45,7 +45,8 @@ EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noal
            "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
-           "scone_embed_varlen", "scone_gemm_bf16", "scone_fgram_model_create",
+           "scone_embed_varlen", "scone_rowstore_open", "scone_rowstore_gather",
+           "scone_rowstore_get_stats", "scone_rowstore_close", "scone_gemm_bf16", "scone_fgram_model_create",
            "scone_fgram_model_destroy", "scone_fgram_precompute", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
            "scone_strerror", "scone_version")
 
@@ -67,6 +68,14 @@ class scone_table_info(ctypes.Structure):
                 ("K", _i32), ("vocab", _i32), ("d", _i32), ("F_location", _i32),
                 ("max_insert_probe", _i32), ("table_bytes", _i64), ("F_bytes", _i64),
                 ("T_bytes", _i64)]
+
+    def as_dict(self):
+        return {k: getattr(self, k) for k, _ in self._fields_}
+
+
+class scone_rowstore_stats(ctypes.Structure):
+    _fields_ = [("positions", _i64), ("misses", _i64), ("rows_read", _i64), ("bytes_read", _i64),
+                ("direct_io", _i32)]
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}
@@ -108,6 +117,11 @@ def load_library():
     lib.scone_embed_gather.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_embed.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]
     lib.scone_embed_varlen.argtypes = [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]
+    lib.scone_rowstore_open.argtypes = [ctypes.c_char_p, _i64, _i32, _i64, _i32,
+                                        ctypes.POINTER(_vp)]
+    lib.scone_rowstore_gather.argtypes = [_vp, _vp, _vp, _vp, _i64, _vp, _vp]
+    lib.scone_rowstore_get_stats.argtypes = [_vp, ctypes.POINTER(scone_rowstore_stats)]
+    lib.scone_rowstore_close.argtypes = [_vp]
     lib.scone_gemm_bf16.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp]
     lib.scone_fgram_model_create.argtypes = [_i32, _i32, _i32, _i32, _vp, _i64,
                                              ctypes.POINTER(_vp)]
@@ -363,6 +377,59 @@ def scone_fgram_precompute(model: FgramModel, fgram_tok, fgram_len, T, F, vocab:
     _check(load_library().scone_fgram_precompute(model.handle, _ptr(fgram_tok), _ptr(fgram_len), n,
                                                  K, _ptr(T), vocab, _ptr(F), _stream(stream)),
            "scone_fgram_precompute")
+
+
+class RowStore:
+    """F in a file with an HBM row cache (scone_rowstore_*)."""
+
+    def __init__(self, path: str, n_rows: int, d: int, cache_rows: int, threads: int = 0):
+        h = _vp()
+        _check(load_library().scone_rowstore_open(os.fsencode(path), n_rows, d, cache_rows,
+                                                  threads, ctypes.byref(h)),
+               "scone_rowstore_open")
+        self._h = h
+
+    @property
+    def handle(self):
+        if self._h is None:
+            raise RuntimeError("row store was closed")
+        return self._h
+
+    def stats(self) -> dict:
+        st = scone_rowstore_stats()
+        _check(load_library().scone_rowstore_get_stats(self.handle, ctypes.byref(st)),
+               "scone_rowstore_get_stats")
+        return st.as_dict()
+
+    def close(self):
+        if self._h is not None:
+            load_library().scone_rowstore_close(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def scone_rowstore_open(path, n_rows, d, cache_rows, threads=0) -> RowStore:
+    return RowStore(path, n_rows, d, cache_rows, threads)
+
+
+def scone_rowstore_close(store: RowStore) -> None:
+    store.close()
+
+
+def scone_rowstore_get_stats(store: RowStore) -> dict:
+    return store.stats()
+
+
+def scone_rowstore_gather(store: RowStore, table: Table, tok, row, out, stream=None) -> None:
+    """out[t] = F[row[t]] from the store (or T[tok[t]] where row[t] < 0)."""
+    _check(load_library().scone_rowstore_gather(store.handle, table.handle, _ptr(tok), _ptr(row),
+                                                row.numel(), _ptr(out), _stream(stream)),
+           "scone_rowstore_gather")
 
 
 class DecodeState:

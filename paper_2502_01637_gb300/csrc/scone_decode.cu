@@ -97,7 +97,8 @@ __global__ void __launch_bounds__(kDecThreads)
       src_s[warp][0] = src;
     }
     __syncwarp();
-    warp_copy_rows_w<W>(src_s[warp], out + s * (int64_t)row_bytes, 1, row_bytes, width, lane);
+    if (out)   // NULL: selection only (the rows are gathered elsewhere, e.g. from a row store)
+      warp_copy_rows_w<W>(src_s[warp], out + s * (int64_t)row_bytes, 1, row_bytes, width, lane);
     __syncwarp();
   }
 }
@@ -163,7 +164,7 @@ extern "C" int scone_decode_step(scone_decode* st, const int32_t* new_tok, scone
                                  int32_t* row, uint8_t* len, void* stream) {
   if (!st || !st->table) return SCONE_ERR_INVALID_ARG;
   if (st->S == 0) return SCONE_OK;
-  if (!new_tok || !out || ((uintptr_t)new_tok & 3) || ((uintptr_t)out & 1) ||
+  if (!new_tok || (!out && !row) || ((uintptr_t)new_tok & 3) || ((uintptr_t)out & 1) ||
       (row && ((uintptr_t)row & 3)))
     return SCONE_ERR_INVALID_ARG;
   const scone_table* tb = st->table;

@@ -1,0 +1,120 @@
+"""The row store (F in a file, rows cached in HBM) against the oracle (GPU).
+
+F is written to a file in the test's temporary directory; the table's F
+pointer is a small dummy, so every F row the output holds came through the
+store (cache hit or file read). A cache much smaller than F forces misses,
+evictions and slot conflicts; repeating a batch turns misses into hits.
+Outputs must equal the oracle's bytes exactly.
+"""
+
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+import paper_2502_01637_gb300 as scone
+from gpu_cases import DEV, SmallCase, dev_rows
+
+pytestmark = pytest.mark.gpu
+
+W = synth.WORKLOADS["tiny"].scaled("rowstore", B=6, L=700, d=64, quotas=((2, 6000), (3, 4000)))
+
+
+@pytest.fixture(scope="module")
+def case(tmp_path_factory):
+    c = SmallCase(W)
+    path = os.path.join(str(tmp_path_factory.mktemp("rows")), "F.bin")
+    c.F.tofile(path)
+    # the table's own F is never read by the store path: a one-row stand-in
+    c.table = scone.scone_table_build(c.fg_tok, c.fg_len, W.K, W.vocab, W.d,
+                                      dev_rows(c.F[:1]), dev_rows(c.T))
+    c.path = path
+    yield c
+    c.table.close()
+
+
+def gather(case, store, tok):
+    t = torch.from_numpy(np.ascontiguousarray(tok, np.int32)).to(DEV)
+    n = t.numel()
+    row = torch.empty(n, dtype=torch.int32, device=DEV)
+    out = torch.empty((n, W.d), dtype=torch.int16, device=DEV)
+    scone.scone_match(case.table, t, row)
+    scone.scone_rowstore_gather(store, case.table, t.reshape(-1), row, out)
+    scone.scone_status(case.table)
+    return out.cpu().numpy().view(np.uint16)
+
+
+def test_matches_oracle_with_small_cache(case):
+    store = scone.RowStore(case.path, case.F.shape[0], W.d, cache_rows=97, threads=4)
+    exp, _, _, rc = case.expected()
+    assert rc == 0
+    exp = exp.reshape(-1, W.d)
+    got = gather(case, store, case.tok)
+    assert np.array_equal(got, exp)
+    s1 = store.stats()
+    assert s1["misses"] > 0 and s1["rows_read"] > 0
+    got2 = gather(case, store, case.tok)            # same batch again: hot rows now cached
+    assert np.array_equal(got2, exp)
+    s2 = store.stats()
+    assert s2["misses"] - s1["misses"] < s1["misses"]
+    store.close()
+
+
+def test_large_cache_reads_each_row_once(case):
+    store = scone.RowStore(case.path, case.F.shape[0], W.d, cache_rows=1 << 16, threads=2)
+    exp = case.expected()[0].reshape(-1, W.d)
+    for _ in range(3):
+        assert np.array_equal(gather(case, store, case.tok), exp)
+    s = store.stats()
+    # a cache much larger than the rows used: each distinct row read once,
+    # unless two of them share a slot
+    used = np.unique(case.expected()[1][case.expected()[1] >= 0])
+    assert s["rows_read"] <= used.size * 1.05 and s["rows_read"] >= used.size * 0.9
+    store.close()
+
+
+def test_decode_selection_then_store(case):
+    """scone_decode_step without rows (out = NULL) then the store equals the
+    fused decode step over the table's full F."""
+    full = scone.scone_table_build(case.fg_tok, case.fg_len, W.K, W.vocab, W.d, dev_rows(case.F),
+                                   dev_rows(case.T))
+    store = scone.RowStore(case.path, case.F.shape[0], W.d, cache_rows=211)
+    S, H = 64, W.K - 1
+    hist = case.tok[:, :H].repeat(11, axis=0)[:S]
+    hl = np.full(S, H, np.int32)
+    a = scone.scone_decode_create(full, hist, hl)
+    b = scone.scone_decode_create(case.table, hist, hl)
+    for k in range(5):
+        new = torch.from_numpy(np.ascontiguousarray(case.tok.reshape(-1)[k * S:(k + 1) * S]))
+        new = new.to(DEV)
+        out_a = torch.empty((S, W.d), dtype=torch.int16, device=DEV)
+        scone.scone_decode_step(a, new, out_a)
+        row_b = torch.empty(S, dtype=torch.int32, device=DEV)
+        lib = scone.load_library()
+        assert lib.scone_decode_step(b.handle, new.data_ptr(), None, row_b.data_ptr(), None,
+                                     torch.cuda.current_stream().cuda_stream) == 0
+        out_b = torch.empty((S, W.d), dtype=torch.int16, device=DEV)
+        scone.scone_rowstore_gather(store, case.table, new, row_b, out_b)
+        assert torch.equal(out_a, out_b), k
+    a.close()
+    b.close()
+    store.close()
+    full.close()
+
+
+def test_errors(case, tmp_path):
+    with pytest.raises(scone.SconeError):
+        scone.RowStore(case.path, case.F.shape[0] + 1, W.d, 16)      # file too short
+    with pytest.raises(scone.SconeError):
+        scone.RowStore(str(tmp_path / "missing.bin"), 10, W.d, 16)
+    store = scone.RowStore(case.path, 100, W.d, 16)                 # rows >= 100 are invalid
+    t = torch.from_numpy(case.tok[0]).to(DEV)
+    row = torch.empty(t.numel(), dtype=torch.int32, device=DEV)
+    scone.scone_match(case.table, t, row)
+    assert int((row >= 100).sum()) > 0
+    out = torch.empty((t.numel(), W.d), dtype=torch.int16, device=DEV)
+    scone.scone_rowstore_gather(store, case.table, t, row, out)
+    assert scone.scone_status(case.table, raise_on_error=False) == scone.SCONE_ERR_INVALID_ARG
+    store.close()
