@@ -649,6 +649,112 @@ def bench_prescan(args, world, rank, local):
     return res
 
 
+# ------------------------------------------------ decode with F in a file
+def bench_store(args, world, rank, local):
+    """Decode steps with F in a file (the storage tier): 512 live sequences,
+    each step selects on the GPU (scone_decode_step without rows), then
+    scone_rowstore_gather copies cached rows and reads the missed ones from
+    the file (O_DIRECT, 4 KiB rows) into the HBM cache. 2e6 f-grams, d = 2048
+    (an 8.2 GB file); cache of 65,536 rows (256 MiB of HBM)."""
+    import torch
+
+    import synth
+    import paper_2502_01637_gb300 as scone
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = workload("decode_profile")
+    cache_rows = 65536
+    t0 = time.time()
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    path = os.path.join(ROOT, "_store_F.bin")
+    rows_per = 1 << 16
+    with open(path, "wb") as f:
+        for r0 in range(0, w.n_fgrams, rows_per):
+            synth.rows_range_cpu(synth.F_seed(w), w.d, r0,
+                                 min(rows_per, w.n_fgrams - r0)).tofile(f)
+    os.sync()
+    stream = torch.cuda.current_stream()
+    T = torch.empty((w.vocab, w.d), dtype=torch.int16, device=dev)
+    synth.rows_gpu(synth.T_seed(w), w.d, 0, w.vocab, T.data_ptr(), stream.cuda_stream)
+    F_stub = torch.zeros((1, w.d), dtype=torch.int16, device=dev)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, F_stub, T)
+    store = scone.RowStore(path, w.n_fgrams, w.d, cache_rows)
+    setup_s = time.time() - t0
+    hist, hl, new = synth.decode_inputs(w)
+    S, steps = w.dec_S, w.dec_steps
+    new_d = torch.from_numpy(new).to(dev)
+    out = torch.empty((S, w.d), dtype=torch.int16, device=dev)
+    row = torch.empty(S, dtype=torch.int32, device=dev)
+    lib = scone.load_library()
+    st = scone.scone_decode_create(table, hist, hl)
+
+    def step(k):
+        rc = lib.scone_decode_step(st.handle, new_d[k % steps].data_ptr(), None, row.data_ptr(),
+                                   None, stream.cuda_stream)
+        assert rc == 0
+        scone.scone_rowstore_gather(store, table, new_d[k % steps], row, out)
+
+    for k in range(args.warmup):
+        step(k)
+    s0 = store.stats()
+    n_steps = max(args.steps, 1)
+    clocks = ClockSampler(local)
+    torch.cuda.synchronize()
+    with clocks:
+        t1 = time.perf_counter()
+        for k in range(n_steps):
+            step(args.warmup + k)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t1
+    scone.scone_status(table)
+    s1 = store.stats()
+    ms = 1e3 * wall / n_steps
+    misses = s1["misses"] - s0["misses"]
+    positions = s1["positions"] - s0["positions"]
+    rows_read = s1["rows_read"] - s0["rows_read"]
+    res = {
+        "metric": "embedded tokens/s at 1 GB300, F in a file (storage tier), decode",
+        "value": world * S / (ms * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": n_steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded Zipf decode tokens; F rows written to a file on the box)",
+        "config": {"workload": (f"store_decode: {S} sequences per step, {w.n_fgrams} f-grams, "
+                                f"d={w.d}, F in an {w.n_fgrams * w.d * 2 / 1e9:.1f} GB file, "
+                                f"HBM row cache of {cache_rows} rows"),
+                   "timing": "host wall clock per step (each step synchronizes: the host "
+                             "reads the misses)",
+                   "io": "O_DIRECT pread" if s1["direct_io"] else "buffered pread"},
+        "roofline": {"bound": "storage", "achieved": rows_read * w.d * 2 / wall / 1e9,
+                     "peak": None, "unit": "GB/s read from the file", "frac": None,
+                     "traffic": None,
+                     "kernel": "lookup_kernel + file reads + fill_kernel (host-driven)"},
+        "store": {"hit_rate": 1.0 - misses / max(1, positions), "positions": positions,
+                  "misses": misses, "rows_read": rows_read,
+                  "rows_read_per_step": rows_read / n_steps,
+                  "direct_io": bool(s1["direct_io"])},
+        "e2e": {"value": world * S / (ms * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0,
+                "what": "decode tokens already on the device; the timed loop includes the "
+                        "host's file reads"},
+        "gpu_launches": n_steps * 3,
+        "clocks": clocks.summary(),
+        "setup_s": setup_s,
+    }
+    st.close()
+    store.close()
+    table.close()
+    os.remove(path)
+    return res
+
+
 # ------------------------------------------------------ mixed serving batch
 def mixed_batch(w, k, n_prefill_seq=48, n_decode=512):
     """Batch k of a serving step over the prefill_1b law: n_prefill_seq prompt
@@ -1201,7 +1307,7 @@ def main():
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
                              "offload_decode", "decode_profile", "prescan", "discover",
                              "discover_k5", "discover_profile", "mixed_serving", "precompute",
-                             "gemm_profile"])
+                             "gemm_profile", "store_decode"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
@@ -1227,6 +1333,8 @@ def main():
         res = bench_precompute(args, world, rank, local)
     elif args.workload == "gemm_profile":
         res = bench_gemm(args, world, rank, local)
+    elif args.workload == "store_decode":
+        res = bench_store(args, world, rank, local)
     elif args.workload in ("discover", "discover_k5", "discover_profile"):
         res = bench_discover(args, world, rank, local)
     else:
