@@ -20,6 +20,7 @@
 #include <cuda_bf16.h>
 
 #include <new>
+#include <type_traits>
 
 #include "scone_gemm.h"
 #include "scone_host.h"
@@ -160,6 +161,33 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// C consecutive bf16 moved as one 2-, 4- or 8-byte word.
+template <int C>
+struct Lanes {
+  using Word = typename std::conditional<C == 1, uint16_t,
+                                         typename std::conditional<C == 2, uint32_t,
+                                                                   uint2>::type>::type;
+  union {
+    Word w;
+    uint16_t h[C];
+  } u;
+  __device__ __forceinline__ static Lanes load(const uint16_t* p) {
+    Lanes x;
+    x.u.w = __ldg(reinterpret_cast<const Word*>(p));
+    return x;
+  }
+  __device__ __forceinline__ float get(int e) const {
+    return __uint_as_float((uint32_t)u.h[e] << 16);
+  }
+  __device__ __forceinline__ void set(int e, float f) {
+    const __nv_bfloat16 b = __float2bfloat16_rn(f);
+    u.h[e] = *reinterpret_cast<const uint16_t*>(&b);
+  }
+  __device__ __forceinline__ void store(uint16_t* p) const {
+    *reinterpret_cast<Word*>(p) = u.w;
+  }
+};
+
 // Causal attention of one (f-gram, head) per warp over at most KMAX
 // positions. Lane l holds dims C*l .. C*l+C-1 of the head's first half and the
 // same offsets of its second half (C = hd / 64), so each rotate-half pair of
@@ -188,11 +216,14 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
     for (int part = 0; part < 2; ++part) {
       const int base = part * half + C * lane;
+      const Lanes<C> a = Lanes<C>::load(row + base);
+      const Lanes<C> b = Lanes<C>::load(row + d + base);
+      const Lanes<C> c = Lanes<C>::load(row + 2 * d + base);
 #pragma unroll
       for (int e = 0; e < C; ++e) {
-        q[j][part * C + e] = __uint_as_float((uint32_t)row[base + e] << 16);
-        k[j][part * C + e] = __uint_as_float((uint32_t)row[d + base + e] << 16);
-        v[j][part * C + e] = __uint_as_float((uint32_t)row[2 * d + base + e] << 16);
+        q[j][part * C + e] = a.get(e);
+        k[j][part * C + e] = b.get(e);
+        v[j][part * C + e] = c.get(e);
       }
     }
     // rotary embedding at position j: (a, b) -> (a cos - b sin, b cos + a sin)
@@ -238,12 +269,10 @@ __global__ void __launch_bounds__(256)
     uint16_t* out = O + (int64_t)(r0 + i) * d + h * hd;
 #pragma unroll
     for (int part = 0; part < 2; ++part) {
-      const int base = part * half + C * lane;
+      Lanes<C> o;
 #pragma unroll
-      for (int e = 0; e < C; ++e) {
-        const __nv_bfloat16 b = __float2bfloat16_rn(acc[part * C + e] * inv);
-        out[base + e] = *reinterpret_cast<const uint16_t*>(&b);
-      }
+      for (int e = 0; e < C; ++e) o.set(e, acc[part * C + e] * inv);
+      o.store(out + part * half + C * lane);
     }
   }
 }
@@ -266,15 +295,24 @@ bool ln(int d, const uint16_t* X, uint16_t* Y, int64_t rows, const int32_t* off,
   }
 }
 
-bool attn(int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d, int H, uint16_t* O,
-          cudaStream_t s) {
+template <int KMAX>
+bool attn_k(int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d, int H,
+            uint16_t* O, cudaStream_t s) {
   const unsigned grid = (unsigned)((n * H + kRowsPerBlock - 1) / kRowsPerBlock);
   switch (hd) {
-    case 64: attention_kernel<1, 8><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
-    case 128: attention_kernel<2, 8><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
-    case 256: attention_kernel<4, 8><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
+    case 64: attention_kernel<1, KMAX><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
+    case 128: attention_kernel<2, KMAX><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
+    case 256: attention_kernel<4, KMAX><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
     default: return false;
   }
+}
+
+// Positions held in registers: the smallest of 3, 5, 8 that covers K.
+bool attn(int K, int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d, int H,
+          uint16_t* O, cudaStream_t s) {
+  if (K <= 3) return attn_k<3>(hd, QKV, off, n, d, H, O, s);
+  if (K <= 5) return attn_k<5>(hd, QKV, off, n, d, H, O, s);
+  return attn_k<8>(hd, QKV, off, n, d, H, O, s);
 }
 
 bool ensure_rows(scone_fgram_model* m, int64_t rows) {
@@ -382,7 +420,7 @@ extern "C" int scone_fgram_precompute(scone_fgram_model* m, const int32_t* fgram
       if ((rc = gemm_bf16(m->Xn, wqkv, nullptr, m->QKV, rows, 3 * d, d, GEMM_EPI_STORE,
                           m->status, s)))
         return rc;
-      if (!attn(d / H, m->QKV, m->off, nb, d, H, m->Xn, s)) return SCONE_ERR_UNSUPPORTED;
+      if (!attn(K, d / H, m->QKV, m->off, nb, d, H, m->Xn, s)) return SCONE_ERR_UNSUPPORTED;
       if ((rc = gemm_bf16(m->Xn, wo, m->X, m->X, rows, d, d, GEMM_EPI_RESIDUAL, m->status, s)))
         return rc;
       if (!ln(d, m->X, m->Xn, rows, nullptr, s)) return SCONE_ERR_UNSUPPORTED;
