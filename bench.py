@@ -1069,6 +1069,17 @@ def bench_gemm(args, world, rank, local):
     assert int(status.item()) == 0
     ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
     flops = 2.0 * M * N * K
+    # the one-SM-per-tile kernel on the same operands, for comparison
+    for _ in range(3):
+        scone.scone_gemm_bf16(A, B, C, epilogue=scone.SCONE_GEMM_SWIGLU, status=status, variant=1)
+    ev1 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(10)]
+    for a, b in ev1:
+        a.record(stream)
+        scone.scone_gemm_bf16(A, B, C, epilogue=scone.SCONE_GEMM_SWIGLU, status=status, variant=1)
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms1 = statistics.mean(a.elapsed_time(b) for a, b in ev1)
     peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) \
         if os.path.exists(os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
     peak = float(peaks.get("bf16_tflops", 1900.0))
@@ -1090,6 +1101,8 @@ def bench_gemm(args, world, rank, local):
         "e2e": {"value": tf, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0, "what": "operands stay on the device"},
         "gpu_launches": args.steps, "clocks": clocks.summary(),
+        "variants": {"sm_pairs_256x256 (default)": tf,
+                     "one_sm_128x256": flops / (ms1 * 1e-3) / 1e12},
     }
 
 

@@ -323,6 +323,12 @@ int scone_embed_varlen(const scone_table* table, const int32_t* tok, int64_t n_t
 enum scone_gemm_epilogue { SCONE_GEMM_STORE = 0, SCONE_GEMM_RESIDUAL = 1, SCONE_GEMM_SWIGLU = 2 };
 int scone_gemm_bf16(const scone_bf16* A, const scone_bf16* B, const scone_bf16* R, scone_bf16* C,
                     int32_t M, int32_t N, int32_t K, int32_t epilogue, int* status, void* stream);
+/* The same with the kernel chosen (for tests and measurements): variant 0 =
+ * default, 1 = one SM per 128 x 256 tile, 2 = pairs of SMs per 256 x 256 tile
+ * (a 2-CTA cluster, tcgen05 cta_group::2). */
+int scone_gemm_bf16_variant(const scone_bf16* A, const scone_bf16* B, const scone_bf16* R,
+                            scone_bf16* C, int32_t M, int32_t N, int32_t K, int32_t epilogue,
+                            int32_t variant, int* status, void* stream);
 
 /*
  * Precomputing F with the f-gram model (Sec. 3.2: after training F is

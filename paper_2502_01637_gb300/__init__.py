@@ -46,7 +46,8 @@ EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noal
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
            "scone_embed_varlen", "scone_rowstore_open", "scone_rowstore_gather",
-           "scone_rowstore_get_stats", "scone_rowstore_close", "scone_gemm_bf16", "scone_fgram_model_create",
+           "scone_rowstore_get_stats", "scone_rowstore_close", "scone_gemm_bf16",
+           "scone_gemm_bf16_variant", "scone_fgram_model_create",
            "scone_fgram_model_destroy", "scone_fgram_precompute", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
            "scone_strerror", "scone_version")
 
@@ -123,6 +124,8 @@ def load_library():
     lib.scone_rowstore_get_stats.argtypes = [_vp, ctypes.POINTER(scone_rowstore_stats)]
     lib.scone_rowstore_close.argtypes = [_vp]
     lib.scone_gemm_bf16.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp]
+    lib.scone_gemm_bf16_variant.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
+                                            _vp, _vp]
     lib.scone_fgram_model_create.argtypes = [_i32, _i32, _i32, _i32, _vp, _i64,
                                              ctypes.POINTER(_vp)]
     lib.scone_fgram_model_destroy.argtypes = [_vp]
@@ -310,7 +313,7 @@ def scone_embed_varlen(table: Table, tok, cu_seqlens, out, state=None, seq_slot=
 
 
 def scone_gemm_bf16(A, B, C, R=None, epilogue: int = SCONE_GEMM_STORE, status=None,
-                    stream=None) -> None:
+                    stream=None, variant: int = 0) -> None:
     """C = epilogue(A B^T) on the tensor cores; A [M, K], B [N, K], C [M, N]
     (or [M, N/2] for SwiGLU), bf16 (or int16 raw bits) device tensors. status:
     a device int32 tensor of one element (allocated here if None; SconeError
@@ -322,8 +325,9 @@ def scone_gemm_bf16(A, B, C, R=None, epilogue: int = SCONE_GEMM_STORE, status=No
     own = status is None
     if own:
         status = torch.zeros(1, dtype=torch.int32, device=A.device)
-    _check(load_library().scone_gemm_bf16(_ptr(A), _ptr(B), _ptr(R), _ptr(C), M, N, K, epilogue,
-                                           _ptr(status), _stream(stream)), "scone_gemm_bf16")
+    _check(load_library().scone_gemm_bf16_variant(_ptr(A), _ptr(B), _ptr(R), _ptr(C), M, N, K,
+                                                   epilogue, variant, _ptr(status),
+                                                   _stream(stream)), "scone_gemm_bf16")
     if own:
         code = int(status.item())
         if code:

@@ -350,6 +350,216 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                  : "memory");
 }
 
+// ---------------------------------------------------------------- SM pairs
+// The same GEMM on pairs of SMs (a 2-CTA cluster, tcgen05 cta_group::2): a
+// pair computes a 256 x 256 tile. CTA r of the pair loads rows 128r..128r+127
+// of the tile's A slice and of its B slice (16 + 16 KB per stage, so 6
+// stages fit), both completing on the leader's (rank 0) full barrier; the
+// leader's thread issues tcgen05.mma with M = 256, which reads both CTAs'
+// halves and writes rows 128r.. of the accumulator into CTA r's tensor
+// memory. Commits are multicast to both CTAs' barriers; both CTAs' epilogue
+// warps release an accumulator on the leader's barrier. Per SM, a K-slice
+// moves 32 KB instead of 48 KB for the same MMA work.
+constexpr int kPStages = 6;
+constexpr int kPairAccs = 2;                                 // accumulators per CTA
+constexpr uint32_t kPairTmemCols = kPairAccs * kBN;
+constexpr uint32_t kPStageHalf = 128 * kBK * 2;             // 16 KB: A or B half
+constexpr uint32_t kPStageBytes = 2 * kPStageHalf;          // per CTA
+constexpr size_t kPairSmem = (size_t)kPStages * kPStageBytes + 1024 + 256;
+constexpr uint32_t kIdescPair = (1u << 4) | (1u << 7) | (1u << 10) |
+                                ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(256 >> 4) << 24);
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x,
+                                                 int y, uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::"
+      "bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void umma_bf16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                               uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n"
+      " setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(kIdescPair), "r"(accumulate)
+      : "memory");
+}
+// Arrives on the barrier at this shared offset in both CTAs of the pair.
+__device__ __forceinline__ void umma_commit_pair(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(bar),
+      "h"((uint16_t)3)
+      : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
+template <int EPI>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    gemm_bf16_pair_kernel(const __grid_constant__ CUtensorMap map_a,
+                          const __grid_constant__ CUtensorMap map_b, int M, int N, int K,
+                          const uint16_t* __restrict__ R, uint16_t* __restrict__ C, int ldc,
+                          int* status) {
+  extern __shared__ uint8_t gsm_raw[];
+  uint8_t* gsm = reinterpret_cast<uint8_t*>(((uintptr_t)gsm_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = reinterpret_cast<uint64_t*>(gsm + kPStages * kPStageBytes);
+  uint64_t* empty = full + kPStages;
+  uint64_t* tfull = empty + kPStages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  __shared__ int failed;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int num_m = (M + 255) / 256, num_n = N / kBN;
+  const int tiles = num_m * num_n;
+  const int kt_n = K / kBK;
+  const int pair = blockIdx.x >> 1, pairs = gridDim.x >> 1;
+
+  if (threadIdx.x == 0) {
+    failed = 0;
+    for (int i = 0; i < kPStages; ++i) {
+      mbar_init(saddr(&full[i]), 1);
+      mbar_init(saddr(&empty[i]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(saddr(&tfull[a]), 1);
+      mbar_init(saddr(&tempty[a]), 2 * kEpiWarps);
+    }
+    mbar_init(saddr(done), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     saddr(tmem_slot)),
+                 "r"(kPairTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  cluster_sync();   // barriers initialized and tensor memory allocated in both CTAs
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+  volatile int* vfailed = &failed;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // producer (both CTAs): this CTA's halves, completing on the leader's full barrier
+      int it = 0;
+      for (int t = pair; t < tiles && !*vfailed; t += pairs) {
+        int mt, nt;
+        tile_coords(t, num_m, num_n, &mt, &nt);
+        for (int kt = 0; kt < kt_n; ++kt, ++it) {
+          const int st = it % kPStages;
+          if (it >= kPStages && !mbar_wait(saddr(&empty[st]), ((it / kPStages) - 1) & 1)) {
+            *vfailed = 1;
+            break;
+          }
+          if (*vfailed) break;
+          const uint32_t a_dst = saddr(gsm + st * kPStageBytes);
+          const uint32_t full_leader = map_to_rank(saddr(&full[st]), 0);
+          if (leader) mbar_expect_tx(saddr(&full[st]), 2 * kPStageBytes);
+          tma_load_2d_pair(a_dst, &map_a, kt * kBK, mt * 256 + (int)rank * 128, full_leader);
+          tma_load_2d_pair(a_dst + kPStageHalf, &map_b, kt * kBK, nt * kBN + (int)rank * 128,
+                           full_leader);
+        }
+      }
+      if (leader)   // the last slices (both halves) must have landed before exit
+        for (int j = it - kPStages < 0 ? 0 : it - kPStages; j < it; ++j)
+          mbar_wait(saddr(&full[j % kPStages]), (j / kPStages) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      int it = 0, lt = 0;
+      for (int t = pair; t < tiles && !*vfailed; t += pairs, ++lt) {
+        const int acc = lt % kPairAccs;
+        if (lt >= kPairAccs && !mbar_wait(saddr(&tempty[acc]), ((lt / kPairAccs) - 1) & 1)) {
+          *vfailed = 1;
+          break;
+        }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t d_tmem = tmem + acc * kBN;
+        bool ok = true;
+        for (int kt = 0; kt < kt_n; ++kt, ++it) {
+          const int st = it % kPStages;
+          if (!mbar_wait(saddr(&full[st]), (it / kPStages) & 1) || *vfailed) {
+            *vfailed = 1;
+            ok = false;
+            break;
+          }
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t a_base = saddr(gsm + st * kPStageBytes);
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            umma_bf16_pair(d_tmem, desc_k128(a_base + 32 * k),
+                           desc_k128(a_base + kPStageHalf + 32 * k), (kt > 0 || k > 0) ? 1u : 0u);
+          umma_commit_pair(saddr(&empty[st]));
+        }
+        if (!ok) break;
+        umma_commit_pair(saddr(&tfull[acc]));
+      }
+      umma_commit_pair(saddr(done));
+    }
+  } else {
+    const int q = warp & 3;
+    const uint32_t tempty_leader0 = map_to_rank(saddr(&tempty[0]), 0);
+    const uint32_t tempty_leader1 = map_to_rank(saddr(&tempty[1]), 0);
+    int lt = 0;
+    for (int t = pair; t < tiles; t += pairs, ++lt) {
+      const int acc = lt % kPairAccs;
+      if (!mbar_wait(saddr(&tfull[acc]), (lt / kPairAccs) & 1) || *vfailed) {
+        *vfailed = 1;
+        break;
+      }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      int mt, nt;
+      tile_coords(t, num_m, num_n, &mt, &nt);
+      const int row = mt * 256 + (int)rank * 128 + q * 32 + lane;
+      const uint32_t t_row = tmem + acc * kBN + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+      for (int c0 = 0; c0 < kBN; c0 += 32) {
+        float v[32];
+        tmem_ld32(t_row + c0, v);
+        if (row < M) store_chunk<EPI>(v, row, nt * kBN + c0, R, C, ldc);
+      }
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(acc ? tempty_leader1 : tempty_leader0);
+    }
+  }
+  // every MMA of the pair has completed before either CTA frees its tensor memory
+  if (threadIdx.x == 32) mbar_wait(saddr(done), 0);
+  __syncthreads();
+  if (*vfailed && threadIdx.x == 0) atomicCAS(status, 0, (int)SCONE_ERR_CUDA);
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  cluster_sync();   // no CTA leaves while its peer may still signal its barriers
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kPairTmemCols)
+                 : "memory");
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   static std::once_flag once;
@@ -393,22 +603,65 @@ bool set_smem_attr() {
   return ok;
 }
 
+template <int EPI>
+bool set_pair_smem_attr() {
+  static std::once_flag once;
+  static bool ok = false;
+  std::call_once(once, [] {
+    ok = cudaFuncSetAttribute(gemm_bf16_pair_kernel<EPI>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)kPairSmem) == cudaSuccess;
+    if (!ok) cudaGetLastError();
+  });
+  return ok;
+}
+
+template <int EPI>
+int launch_pair(const CUtensorMap& ma, const CUtensorMap& mb, int M, int N, int K,
+                const uint16_t* R, uint16_t* C, int ldc, int* status, cudaStream_t s) {
+  if (!set_pair_smem_attr<EPI>()) return SCONE_ERR_CUDA;
+  const int64_t tiles = (int64_t)((M + 255) / 256) * (N / kBN);
+  const int64_t pairs = sm_count() / 2;
+  const unsigned grid = (unsigned)(2 * (tiles < pairs ? tiles : pairs));
+  gemm_bf16_pair_kernel<EPI><<<grid, kGemmThreads, kPairSmem, s>>>(ma, mb, M, N, K, R, C, ldc,
+                                                                   status);
+  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}
+
 }  // namespace
 
 int gemm_bf16(const uint16_t* A, const uint16_t* B, const uint16_t* R, uint16_t* C, int M, int N,
               int K, int epi, int* status, cudaStream_t s) {
+  return gemm_bf16_variant(A, B, R, C, M, N, K, epi, 0, status, s);
+}
+
+int gemm_bf16_variant(const uint16_t* A, const uint16_t* B, const uint16_t* R, uint16_t* C,
+                      int M, int N, int K, int epi, int variant, int* status, cudaStream_t s) {
   if (M < 0 || N <= 0 || K <= 0 || N % kBN || K % kBK || !A || !B || !C || !status)
     return SCONE_ERR_INVALID_ARG;
   if (epi == GEMM_EPI_RESIDUAL && !R) return SCONE_ERR_INVALID_ARG;
   if (((uintptr_t)A | (uintptr_t)B | (uintptr_t)C | (uintptr_t)R) & 15)
     return SCONE_ERR_INVALID_ARG;
   if (M == 0) return SCONE_OK;
+  if (variant < 0 || variant > 2) return SCONE_ERR_INVALID_ARG;
+  const int ldc = epi == GEMM_EPI_SWIGLU ? N / 2 : N;
+  if (variant != 1) {   // SM pairs: 128-row halves of A and B per CTA
+    CUtensorMap pa, pb;
+    if (!make_map(&pa, A, M, K, 128) || !make_map(&pb, B, N, K, 128)) return SCONE_ERR_CUDA;
+    switch (epi) {
+      case GEMM_EPI_STORE: return launch_pair<GEMM_EPI_STORE>(pa, pb, M, N, K, R, C, ldc, status, s);
+      case GEMM_EPI_RESIDUAL:
+        return launch_pair<GEMM_EPI_RESIDUAL>(pa, pb, M, N, K, R, C, ldc, status, s);
+      case GEMM_EPI_SWIGLU:
+        return launch_pair<GEMM_EPI_SWIGLU>(pa, pb, M, N, K, R, C, ldc, status, s);
+      default: return SCONE_ERR_INVALID_ARG;
+    }
+  }
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, M, K, kBM) || !make_map(&mb, B, N, K, kBN)) return SCONE_ERR_CUDA;
   const int64_t tiles = (int64_t)((M + kBM - 1) / kBM) * (N / kBN);
   const int64_t sms = sm_count();
   const dim3 grid((unsigned)(tiles < sms ? tiles : sms));
-  const int ldc = epi == GEMM_EPI_SWIGLU ? N / 2 : N;
   switch (epi) {
     case GEMM_EPI_STORE:
       if (!set_smem_attr<GEMM_EPI_STORE>()) return SCONE_ERR_CUDA;
@@ -437,4 +690,12 @@ extern "C" int scone_gemm_bf16(const scone_bf16* A, const scone_bf16* B, const s
                                scone_bf16* C, int32_t M, int32_t N, int32_t K, int32_t epilogue,
                                int* status, void* stream) {
   return scone::gemm_bf16(A, B, R, C, M, N, K, epilogue, status, (cudaStream_t)stream);
+}
+
+extern "C" int scone_gemm_bf16_variant(const scone_bf16* A, const scone_bf16* B,
+                                       const scone_bf16* R, scone_bf16* C, int32_t M, int32_t N,
+                                       int32_t K, int32_t epilogue, int32_t variant, int* status,
+                                       void* stream) {
+  return scone::gemm_bf16_variant(A, B, R, C, M, N, K, epilogue, variant, status,
+                                  (cudaStream_t)stream);
 }

@@ -21,4 +21,9 @@ enum GemmEpilogue {
 int gemm_bf16(const uint16_t* A, const uint16_t* B, const uint16_t* R, uint16_t* C, int M, int N,
               int K, int epi, int* status, cudaStream_t s);
 
+// The same with the kernel chosen: 0 = default (SM pairs), 1 = one SM per
+// 128 x 256 tile, 2 = SM pairs (256 x 256 tiles, tcgen05 cta_group::2).
+int gemm_bf16_variant(const uint16_t* A, const uint16_t* B, const uint16_t* R, uint16_t* C,
+                      int M, int N, int K, int epi, int variant, int* status, cudaStream_t s);
+
 }  // namespace scone

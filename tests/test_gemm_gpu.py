@@ -28,29 +28,35 @@ def close(got, want, what):
     assert bad == 0, f"{what}: {bad} elements off, max err {err.max().item():.3e}"
 
 
+VARIANTS = [1, 2]      # one SM per tile, SM pairs
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (200, 256, 128), (129, 512, 2048),
-                                   (1000, 768, 512)])
-def test_store(M, N, K):
+                                   (1000, 768, 512), (4099, 1024, 256)])
+def test_store(M, N, K, variant):
     A, B = rand((M, K), 1), rand((N, K), 2)
     C = torch.empty((M, N), dtype=torch.bfloat16, device=DEV)
-    scone.scone_gemm_bf16(A, B, C)
-    close(C, A.float() @ B.float().T, f"store {M}x{N}x{K}")
+    scone.scone_gemm_bf16(A, B, C, variant=variant)
+    close(C, A.float() @ B.float().T, f"store {M}x{N}x{K} variant {variant}")
 
 
+@pytest.mark.parametrize("variant", VARIANTS)
 @pytest.mark.parametrize("M,N,K", [(77, 256, 64), (300, 512, 1024)])
-def test_residual_in_place(M, N, K):
+def test_residual_in_place(M, N, K, variant):
     A, B = rand((M, K), 3), rand((N, K), 4)
     R = rand((M, N), 5, scale=4.0)
     want = R.float() + A.float() @ B.float().T
-    scone.scone_gemm_bf16(A, B, R, R=R, epilogue=scone.SCONE_GEMM_RESIDUAL)
+    scone.scone_gemm_bf16(A, B, R, R=R, epilogue=scone.SCONE_GEMM_RESIDUAL, variant=variant)
     close(R, want, "residual")
 
 
-def test_swiglu_pairs():
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_swiglu_pairs(variant):
     M, N, K = 250, 512, 256
     A, B = rand((M, K), 6, 0.5), rand((N, K), 7, 0.1)
     C = torch.empty((M, N // 2), dtype=torch.bfloat16, device=DEV)
-    scone.scone_gemm_bf16(A, B, C, epilogue=scone.SCONE_GEMM_SWIGLU)
+    scone.scone_gemm_bf16(A, B, C, epilogue=scone.SCONE_GEMM_SWIGLU, variant=variant)
     P = A.float() @ B.float().T                      # [M, N]
     P = P.view(M, N // 32, 2, 16)
     g, u = P[:, :, 0, :], P[:, :, 1, :]
