@@ -22,6 +22,7 @@
 // outstanding bulk operations before returning.
 
 #include "scone_host.h"
+#include "scone_ptx.cuh"
 
 namespace scone {
 
@@ -33,10 +34,6 @@ constexpr uint32_t kSpinLimit = 1u << 22;
 
 namespace {
 
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-
 __device__ __forceinline__ void bar_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
@@ -44,24 +41,6 @@ __device__ __forceinline__ void bar_arrive(int id, int count) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n"
-      " mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
                                           uint32_t bar) {
   asm volatile(
@@ -106,7 +85,7 @@ __global__ void __launch_bounds__(kBulkThreads)
   const int64_t n_tiles = (total + kBulkTile - 1) / kBulkTile;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < ring; ++s) mbar_init(smem_addr(&full[s]), 1);
+    for (int s = 0; s < ring; ++s) mbar_init(saddr(&full[s]), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
@@ -156,9 +135,9 @@ __global__ void __launch_bounds__(kBulkThreads)
     }
     if (lane == 0 && !failed) {
       const int s = (int)(j % ring);
-      const uint32_t bar = smem_addr(&full[s]);
+      const uint32_t bar = saddr(&full[s]);
       mbar_expect_tx(bar, row_bytes);
-      bulk_load(smem_addr(slots + (size_t)s * row_bytes),
+      bulk_load(saddr(slots + (size_t)s * row_bytes),
                 srcs[(tile & 1) * kBulkTile + (j % kBulkTile)], row_bytes, bar);
       issued = j + 1;
     }
@@ -180,7 +159,7 @@ __global__ void __launch_bounds__(kBulkThreads)
         const int s = (int)(j % ring);
         const uint32_t parity = (uint32_t)((j / ring) & 1);
         uint32_t spins = 0;
-        while (!failed && !mbar_try_wait(smem_addr(&full[s]), parity)) {
+        while (!failed && !mbar_try_wait(saddr(&full[s]), parity)) {
           if (++spins >= kSpinLimit) {
             failed = true;
             record_error(t.status, SCONE_ERR_CUDA);
@@ -188,7 +167,7 @@ __global__ void __launch_bounds__(kBulkThreads)
         }
         if (!failed) {
           waited = j + 1;
-          bulk_store(out + (lo + j) * (int64_t)row_bytes, smem_addr(slots + (size_t)s * row_bytes),
+          bulk_store(out + (lo + j) * (int64_t)row_bytes, saddr(slots + (size_t)s * row_bytes),
                      row_bytes);
         }
       }
@@ -206,7 +185,7 @@ __global__ void __launch_bounds__(kBulkThreads)
       // drain the loads still in flight into the ring before the CTA exits
       for (int64_t j = waited; j < issued; ++j) {
         uint32_t spins = 0;
-        while (!mbar_try_wait(smem_addr(&full[j % ring]), (uint32_t)((j / ring) & 1)) &&
+        while (!mbar_try_wait(saddr(&full[j % ring]), (uint32_t)((j / ring) & 1)) &&
                ++spins < kSpinLimit) {
         }
       }

@@ -111,15 +111,6 @@ DecodeFn pick_decode(int fmt, int width) {
   return width == 16 ? decode_kernel<FMT32, 16> : decode_kernel<FMT32, 0>;
 }
 
-int decode_width(const TableView& t, const void* out) {
-  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)(t.d * 2);
-  if (t.n_fgrams > 0) a |= (uintptr_t)t.F;
-  if ((a & 15) == 0) return 16;
-  if ((a & 7) == 0) return 8;
-  if ((a & 3) == 0) return 4;
-  return 2;
-}
-
 }  // namespace
 
 }  // namespace scone
@@ -169,7 +160,7 @@ extern "C" int scone_decode_step(scone_decode* st, const int32_t* new_tok, scone
     return SCONE_ERR_INVALID_ARG;
   const scone_table* tb = st->table;
   DeviceGuard g(tb->device);
-  const int width = decode_width(tb->view, out);
+  const int width = row_copy_width(tb->view, out);
   const DecodeFn fn = pick_decode(tb->fmt, width);
   const int64_t need = (st->S + kDecWarps - 1) / kDecWarps;
   const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)fn, kDecThreads, 0);

@@ -75,17 +75,6 @@ int copy_grid(const void* fn, int64_t n_tok) {
   return grid_size(fn, (n_tok + kWarps * kMinRowsPerWarp - 1) / (kWarps * kMinRowsPerWarp));
 }
 
-// Widest copy unit (16, 8, 4 or 2 bytes) that the row size and every base
-// address allow.
-int copy_width(const TableView& t, const void* out) {
-  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)(t.d * 2);
-  if (t.n_fgrams > 0) a |= (uintptr_t)t.F;
-  if ((a & 15) == 0) return 16;
-  if ((a & 7) == 0) return 8;
-  if ((a & 3) == 0) return 4;
-  return 2;
-}
-
 __device__ __forceinline__ int32_t pos_in_seq(int64_t p, int32_t L) { return (int32_t)(p % L); }
 
 template <int FMT, int KT>
@@ -243,7 +232,7 @@ extern "C" int scone_embed_gather(const scone_table* tb, const int32_t* tok, con
   if (!tok || !row || !out || misaligned(tok, 4) || misaligned(row, 4) || misaligned(out, 2))
     return SCONE_ERR_INVALID_ARG;
   DeviceGuard g(tb->device);
-  const int width = copy_width(tb->view, out);
+  const int width = row_copy_width(tb->view, out);
   const auto fn = width == 16 ? gather_kernel<16> : gather_kernel<0>;
   const int grid = copy_grid((const void*)fn, n_tok);
   fn<<<grid, kThreads, 0, (cudaStream_t)stream>>>(tb->view, tok, row, n_tok,
@@ -265,7 +254,7 @@ extern "C" int scone_embed(const scone_table* tb, const int32_t* tok, int32_t B,
     return launch_embed_bulk(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
                              (cudaStream_t)stream);
   }
-  const int width = copy_width(tb->view, out);
+  const int width = row_copy_width(tb->view, out);
   const EmbedFn fn = pick_embed(tb->fmt, tb->view.K, width);
   const int grid = copy_grid((const void*)fn, n);
   fn<<<grid, kThreads, 0, (cudaStream_t)stream>>>(tb->view, tok, n, L,

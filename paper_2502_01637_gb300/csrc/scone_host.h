@@ -45,6 +45,17 @@ bool bulk_eligible(const scone_table* tb, const void* out);
 int launch_embed_bulk(const scone_table* tb, const int32_t* tok, int64_t n, int32_t L,
                       uint8_t* out, int32_t* row, uint8_t* len, cudaStream_t stream);
 
+// Widest copy unit (16, 8, 4 or 2 bytes) that the row size, T, F, the output
+// and `extra` (another base address or size, 0 if none) all allow.
+inline int row_copy_width(const TableView& t, const void* out, uintptr_t extra = 0) {
+  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)(t.d * 2) | extra;
+  if (t.n_fgrams > 0) a |= (uintptr_t)t.F;
+  if ((a & 15) == 0) return 16;
+  if ((a & 7) == 0) return 8;
+  if ((a & 3) == 0) return 4;
+  return 2;
+}
+
 // Resident blocks per SM for a kernel at a block size (cached per function).
 int blocks_per_sm(const void* fn, int threads, size_t smem);
 int sm_count();

@@ -352,8 +352,7 @@ extern "C" int scone_rowstore_gather(scone_rowstore* st, const scone_table* tb,
   cudaStream_t s = (cudaStream_t)stream;
   if (!grow(st, n)) return SCONE_ERR_NOMEM;
   const TableView& t = tb->view;
-  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)st->cache | (uintptr_t)st->row_bytes;
-  const int width = (a & 15) == 0 ? 16 : ((a & 7) == 0 ? 8 : ((a & 3) == 0 ? 4 : 2));
+  const int width = row_copy_width(t, out, (uintptr_t)st->cache);
   const int64_t blocks_needed = (n + kStoreThreads - 1) / kStoreThreads;
   const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)lookup_kernel,
                                                           kStoreThreads, 0);

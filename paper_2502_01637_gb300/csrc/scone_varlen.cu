@@ -166,15 +166,6 @@ VarlenFn pick_varlen_w(int fmt, int K) {
   return varlen_embed_kernel<FMT32, 8, W>;
 }
 
-int varlen_width(const TableView& t, const void* out) {
-  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)(t.d * 2);
-  if (t.n_fgrams > 0) a |= (uintptr_t)t.F;
-  if ((a & 15) == 0) return 16;
-  if ((a & 7) == 0) return 8;
-  if ((a & 3) == 0) return 4;
-  return 2;
-}
-
 }  // namespace
 
 }  // namespace scone
@@ -202,7 +193,7 @@ extern "C" int scone_embed_varlen(const scone_table* tb, const int32_t* tok, int
   const int32_t S = state ? state->S : 0;
   const int32_t H = state ? state->H : 0;
   if (n_tok > 0) {
-    const int width = varlen_width(tb->view, out);
+    const int width = row_copy_width(tb->view, out);
     const VarlenFn fn = width == 16 ? pick_varlen_w<16>(tb->fmt, tb->view.K)
                                     : pick_varlen_w<0>(tb->fmt, tb->view.K);
     const int64_t want = (n_tok + kVWarps * 8 - 1) / (kVWarps * 8);
