@@ -118,3 +118,27 @@ def test_errors(case, tmp_path):
     scone.scone_rowstore_gather(store, case.table, t, row, out)
     assert scone.scone_status(case.table, raise_on_error=False) == scone.SCONE_ERR_INVALID_ARG
     store.close()
+
+
+def test_direct_io_rows(tmp_path):
+    """4 KiB rows (d = 2048): the store reads the file with O_DIRECT where the
+    filesystem allows it; bytes still equal the oracle's."""
+    w = synth.WORKLOADS["tiny"].scaled("rowstore_4k", B=2, L=300, d=2048,
+                                       quotas=((2, 1500), (3, 1000)))
+    c = SmallCase(w)
+    path = str(tmp_path / "F4k.bin")
+    c.F.tofile(path)
+    table = scone.scone_table_build(c.fg_tok, c.fg_len, w.K, w.vocab, w.d, dev_rows(c.F[:1]),
+                                    dev_rows(c.T))
+    store = scone.RowStore(path, c.F.shape[0], w.d, cache_rows=50, threads=3)
+    t = torch.from_numpy(c.tok).to(DEV)
+    row = torch.empty(t.numel(), dtype=torch.int32, device=DEV)
+    out = torch.empty((t.numel(), w.d), dtype=torch.int16, device=DEV)
+    scone.scone_match(table, t, row)
+    scone.scone_rowstore_gather(store, table, t.reshape(-1), row, out)
+    scone.scone_status(table)
+    exp = c.expected()[0].reshape(-1, w.d)
+    assert np.array_equal(out.cpu().numpy().view(np.uint16), exp)
+    assert store.stats()["rows_read"] > 0
+    store.close()
+    table.close()

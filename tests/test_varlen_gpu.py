@@ -191,3 +191,43 @@ def test_error_positions(case):
     rc = scone.scone_status(case.table, raise_on_error=False)
     assert rc in (scone.SCONE_ERR_TOKEN_RANGE, scone.SCONE_ERR_INVALID_ARG)
     st.close()
+
+
+def test_k5_ragged_and_continued():
+    """K = 5 over the stress law (4- and 5-gram matches): ragged chunks that
+    continue slots match the oracle on the whole prefixes."""
+    w5 = synth.WORKLOADS["stress_k5"].scaled("varlen_k5", B=1, L=64, d=64,
+                                             quotas=((2, 3000), (3, 3000), (4, 1500), (5, 1500)))
+    c = SmallCase(w5, tok=np.zeros((1, 1), np.int32))
+    c.table = c.build()
+    S, H = 6, w5.K - 1
+    st = scone.scone_decode_create(c.table, np.zeros((S, H), np.int32), np.zeros(S, np.int32))
+    full = [synth.zipf_tokens(w5, 900 + s, 400) for s in range(S)]
+    pos = [0] * S
+    rng = np.random.default_rng(4)
+    for rnd in range(6):
+        chunks = []
+        for s in range(S):
+            n = min(int(rng.integers(0, 120)) if rnd < 5 else 400, 400 - pos[s])
+            chunks.append(full[s][pos[s]:pos[s] + n])
+        lens = [len(x) for x in chunks]
+        cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        flat = np.concatenate(chunks).astype(np.int32) if sum(lens) else np.zeros(0, np.int32)
+        n = flat.size
+        out = torch.empty((max(n, 1), w5.d), dtype=torch.int16, device=DEV)
+        row = torch.empty(max(n, 1), dtype=torch.int32, device=DEV)
+        scone.scone_embed_varlen(c.table, torch.from_numpy(flat).to(DEV),
+                                 torch.from_numpy(cu).to(DEV), out[:n], state=st, row=row[:n])
+        torch.cuda.synchronize()
+        for s in range(S):
+            a, b = pos[s], pos[s] + lens[s]
+            exp_out, exp_row, _, rc = c.oracle.embed(np.asarray(full[s][:b], np.int32)[None, :],
+                                                     c.F, c.T)
+            assert np.array_equal(row[:n].cpu().numpy()[cu[s]:cu[s + 1]],
+                                  exp_row[0, a:b].astype(np.int32)), (rnd, s)
+            assert np.array_equal(out[:n].cpu().numpy().view(np.uint16)[cu[s]:cu[s + 1]],
+                                  exp_out[0, a:b]), (rnd, s)
+            pos[s] = b
+    assert scone.scone_status(c.table) == 0
+    st.close()
+    c.table.close()
