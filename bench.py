@@ -1196,10 +1196,14 @@ def bench_discover(args, world, rank, local):
     m = int(st["frequent"][2] + sum(st["frequent"][3:]))
     n_sel = min(S, m)
 
-    # roofline of the dominant kernel: the counting kernel of scan 2 (every window)
+    # roofline of the dominant kernel: the counting pass of scan 2 (bincount_kernel).
+    # Algorithmic bytes: each binned window's record (8-byte key + 2-byte
+    # offset) read once, the per-chunk bin offsets read once, and each distinct
+    # key's 16-byte slot brought from DRAM and written back as one 32-byte
+    # sector each way.
     ms_count = statistics.mean(s_["ms_count"][2] for s_ in stats)
-    flushes = st["flushes"][2]
-    bytes_count = 8 * n + 64 * flushes
+    n_chunks = -(-n // 16384)
+    bytes_count = 10 * st["flushes"][2] + 4 * 1025 * n_chunks + 64 * st["distinct"][2]
     hbm, peak_src = measured_peaks()
     achieved = bytes_count / (ms_count * 1e-3) / 1e9
     res = {
@@ -1229,7 +1233,9 @@ def bench_discover(args, world, rank, local):
             "traffic": None,
             "peak_source": peak_src,
             "algorithmic_bytes_per_launch": bytes_count,
-            "kernel": "count_kernel of scan 2 (8 B per window + 64 B per global table update)",
+            "kernel": ("bincount_kernel of scan 2 (10 B per binned window + 8 B per chunk and "
+                       "bin + 64 B per distinct key; bound in practice by L2 atomics on the "
+                       "resident table region, not by DRAM)"),
             "kernel_ms": ms_count,
             "kernel_share_of_step": ms_count / ms,
         },
@@ -1238,14 +1244,15 @@ def bench_discover(args, world, rank, local):
                 "d2h_bytes_per_step": n_sel * (4 * w.K + 1 + 4),
                 "what": "pinned corpus -> device, scone_fgram_discover, f-gram list -> "
                         "pinned host"},
-        # per call: count, flag, scan, assign per scan and next_id between scans;
-        # then 4 radix-select histograms (only when the cut falls inside the
-        # list), select_count, two scans and emit
-        "gpu_launches": args.steps * (5 * (w.K - 1) - 1 + (8 if S < m else 4)),
+        # per call: bin, hotflush, bincount, flagbin, unsort, scan and assign
+        # per scan; then 4 radix-select histograms (only when the cut falls
+        # inside the list), select_count, two scans and emit
+        "gpu_launches": args.steps * (7 * (w.K - 1) + (8 if S < m else 4)),
         "clocks": clocks.summary(),
         "discover": {k: st[k] for k in ("candidates", "distinct", "frequent", "flushes",
                                          "threshold", "selected_at_threshold",
-                                         "table_bytes_max", "ms_count", "ms_scan",
+                                         "table_bytes_max", "ms_bin", "ms_count", "ms_flag",
+                                         "ms_scan",
                                          "ms_select", "ms_total", "ms_alloc_host",
                                          "workspace_bytes")},
         "setup_s": setup_s,

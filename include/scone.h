@@ -226,14 +226,19 @@ int scone_match(const scone_table* table, const int32_t* tok, int32_t B, int32_t
  *  n_out        host; receives the number of f-grams written (<= S).
  *  stats        host or NULL; per length n (index n): windows counted after
  *               pruning, distinct n-grams among them, eligible n-grams,
- *               global table updates and the counting kernel's device time;
- *               the count of the S-th f-gram and how many f-grams at that
- *               count were taken; the largest counting table allocated; the
- *               device time of the call.
+ *               global table updates and the device time of each pass
+ *               (binning, counting, flagging, whole scan); the count of the
+ *               S-th f-gram and how many f-grams at that count were taken;
+ *               the largest counting table allocated; the device time of
+ *               the call.
  *
  * Synchronous: returns when the lists are written. Working memory: about
- * 9 bytes per token, a counting table of 32 bytes per counted window at the
- * largest scan, and the lists of eligible n-grams (4 (n + 1) bytes each). Errors: SCONE_ERR_INVALID_ARG (K outside [2, 8], min_count < 1,
+ * 15 bytes per token for K = 2, 19 for K = 3 and 23 for K >= 4 (binned
+ * window records and the names of the previous scan), a counting table of
+ * 64 bytes per distinct n-gram of the largest scan (see
+ * scone_discover_set_table_slack), and the lists of eligible n-grams
+ * (4 (n + 1) bytes each). Errors: SCONE_ERR_INVALID_ARG
+ * (K outside [2, 8], min_count < 1,
  * S < 0, null pointers), SCONE_ERR_UNSUPPORTED (B * L > 2^30),
  * SCONE_ERR_TOKEN_RANGE (a token outside [0, vocab); nothing is written),
  * SCONE_ERR_NOMEM, SCONE_ERR_CUDA.
@@ -242,12 +247,19 @@ typedef struct scone_discover_stats {
   int64_t candidates[9];      /* windows counted in scan n (after pruning for n >= 3) */
   int64_t distinct[9];        /* distinct n-grams among them */
   int64_t frequent[9];        /* n-grams with count >= min_count */
-  int64_t flushes[9];         /* global table updates of scan n (distinct keys per chunk) */
+  int64_t flushes[9];         /* global table updates of scan n: binned windows plus
+                                 entries of the per-block hot-key caches */
   int64_t threshold;          /* count of the last-ranked selected f-gram; 0 when all taken */
   int64_t selected_at_threshold; /* f-grams taken at that count (0 when all taken) */
   int64_t table_bytes_max;    /* largest counting table of a scan */
-  double ms_count[9];         /* device time of scan n's counting kernel (CUDA events) */
+  double ms_bin[9];           /* device time of scan n's binning pass (CUDA events) */
+  double ms_count[9];         /* ... of its counting pass */
+  double ms_flag[9];          /* ... of its flagging pass (lookups and names) */
   double ms_scan[9];          /* device time of the whole scan n */
+  int64_t estimate[9];        /* sketch estimate of the distinct n-grams of scan n, which
+                                 sizes its counting table */
+  int64_t table_rebuilds;     /* scans whose table turned out too small for the estimate
+                                 and were counted again in a worst-case table */
   double ms_select;           /* device time of the selection and the emission */
   double ms_total;            /* device time of the whole call, first launch to last */
   double ms_alloc_host;       /* host time spent in the call's allocations */
@@ -263,6 +275,17 @@ int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int32_t B, int3
 int scone_discover_create(scone_discover** out);
 /* Frees the workspace and its device buffers (NULL is a no-op). */
 int scone_discover_destroy(scone_discover* ws);
+/*
+ * Sizing of the counting tables of the calls that use ws: slots per
+ * estimated distinct n-gram (default 4, i.e. load factor 0.25). Each scan
+ * estimates its distinct n-grams with a HyperLogLog sketch (standard error
+ * 1.6%) before it counts. A table that still fills up (probe sequences past
+ * 4096 slots) is rebuilt at the worst-case size, two slots per counted
+ * window, and the scan counted again: results never depend on the setting,
+ * only memory and time do. Errors: SCONE_ERR_INVALID_ARG (ws NULL,
+ * slots_per_key not in (0, 1e6]).
+ */
+int scone_discover_set_table_slack(scone_discover* ws, double slots_per_key);
 
 /*
  * scone_embed_gather — the emission step of Algorithm 1 (Sec. 3): for each

@@ -48,7 +48,8 @@ EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noal
            "scone_embed_varlen", "scone_rowstore_open", "scone_rowstore_gather",
            "scone_rowstore_get_stats", "scone_rowstore_close", "scone_gemm_bf16",
            "scone_gemm_bf16_variant", "scone_fgram_model_create",
-           "scone_fgram_model_destroy", "scone_fgram_precompute", "scone_fgram_discover", "scone_discover_create", "scone_discover_destroy",
+           "scone_fgram_model_destroy", "scone_fgram_precompute", "scone_fgram_discover",
+           "scone_discover_create", "scone_discover_destroy", "scone_discover_set_table_slack",
            "scone_strerror", "scone_version")
 
 _lib = None
@@ -85,8 +86,10 @@ class scone_rowstore_stats(ctypes.Structure):
 class scone_discover_stats(ctypes.Structure):
     _fields_ = [("candidates", _i64 * 9), ("distinct", _i64 * 9), ("frequent", _i64 * 9),
                 ("flushes", _i64 * 9), ("threshold", _i64), ("selected_at_threshold", _i64),
-                ("table_bytes_max", _i64), ("ms_count", ctypes.c_double * 9),
-                ("ms_scan", ctypes.c_double * 9), ("ms_select", ctypes.c_double),
+                ("table_bytes_max", _i64), ("ms_bin", ctypes.c_double * 9),
+                ("ms_count", ctypes.c_double * 9), ("ms_flag", ctypes.c_double * 9),
+                ("ms_scan", ctypes.c_double * 9), ("estimate", _i64 * 9),
+                ("table_rebuilds", _i64), ("ms_select", ctypes.c_double),
                 ("ms_total", ctypes.c_double), ("ms_alloc_host", ctypes.c_double),
                 ("workspace_bytes", _i64)]
 
@@ -142,6 +145,7 @@ def load_library():
                                          ctypes.POINTER(scone_discover_stats), _vp]
     lib.scone_discover_create.argtypes = [ctypes.POINTER(_vp)]
     lib.scone_discover_destroy.argtypes = [_vp]
+    lib.scone_discover_set_table_slack.argtypes = [_vp, ctypes.c_double]
     lib.scone_strerror.argtypes = [ctypes.c_int]
     lib.scone_strerror.restype = ctypes.c_char_p
     lib.scone_version.argtypes = []
@@ -543,6 +547,11 @@ class DiscoverWorkspace:
         if self._h is None:
             raise RuntimeError("workspace was closed")
         return self._h
+
+    def set_table_slack(self, slots_per_key: float):
+        """Counting-table slots per estimated distinct n-gram (default 4)."""
+        _check(load_library().scone_discover_set_table_slack(self.handle, float(slots_per_key)),
+               "scone_discover_set_table_slack")
 
     def close(self):
         if self._h is not None:

@@ -97,6 +97,7 @@ def test_null_handles_rejected():
                                     None) == inv             # no n_out
     assert lib.scone_discover_create(None) == inv
     assert lib.scone_discover_destroy(None) == 0
+    assert lib.scone_discover_set_table_slack(None, 2.5) == inv
 
 
 def test_key_format_boundaries():

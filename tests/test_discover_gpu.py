@@ -159,3 +159,30 @@ def test_workspace_reuse():
         assert np.array_equal(a[1].cpu().numpy(), ref["len"])
         assert np.array_equal(a[0].cpu().numpy(), ref["tok"])
     ws.close()
+
+
+@pytest.mark.parametrize("slack", [0.02, 0.5, 4.0, 40.0])
+def test_table_sizing_and_rebuild(slack):
+    """The counting table is sized from a sketch of the distinct n-grams;
+    the sizing never changes the result. A table far too small for the keys
+    fills up and the scan is counted again in a worst-case table; at the
+    default and above nothing is rebuilt, and the sketch stays within a few
+    percent of the exact distinct count."""
+    V, K, mc = 3000, 4, 2
+    tok = zipf(16, 4000, V, seed=11)
+    ws = scone.scone_discover_create()
+    ws.set_table_slack(slack)
+    t = torch.from_numpy(tok).to(DEV)
+    ft, fl, fc, st = scone.scone_fgram_discover(t, V, K, 5000, mc, workspace=ws)
+    ref = oracle.discover(tok, K, V, 5000, mc)
+    assert np.array_equal(fl.cpu().numpy(), ref["len"])
+    assert np.array_equal(ft.cpu().numpy(), ref["tok"])
+    assert np.array_equal(fc.cpu().numpy().view(np.uint32), ref["count"])
+    for n in range(2, K + 1):
+        assert st["frequent"][n] == ref["frequent"][n]
+        assert abs(st["estimate"][n] - st["distinct"][n]) <= 0.06 * st["distinct"][n] + 8, n
+    if slack < 1:
+        assert st["table_rebuilds"] >= 1
+    else:
+        assert st["table_rebuilds"] == 0
+    ws.close()

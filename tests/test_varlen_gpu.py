@@ -193,41 +193,76 @@ def test_error_positions(case):
     st.close()
 
 
-def test_k5_ragged_and_continued():
-    """K = 5 over the stress law (4- and 5-gram matches): ragged chunks that
-    continue slots match the oracle on the whole prefixes."""
-    w5 = synth.WORKLOADS["stress_k5"].scaled("varlen_k5", B=1, L=64, d=64,
-                                             quotas=((2, 3000), (3, 3000), (4, 1500), (5, 1500)))
-    c = SmallCase(w5, tok=np.zeros((1, 1), np.int32))
+def ragged_continued(w, seed, rounds=6, per_seq=400):
+    """Six rounds of ragged chunks (some empty) that continue S slots, the
+    last round flushing each sequence's rest; every chunk's rows match the
+    oracle on the sequence's whole prefix."""
+    c = SmallCase(w, tok=np.zeros((1, 1), np.int32))
     c.table = c.build()
-    S, H = 6, w5.K - 1
+    S, H = 6, w.K - 1
     st = scone.scone_decode_create(c.table, np.zeros((S, H), np.int32), np.zeros(S, np.int32))
-    full = [synth.zipf_tokens(w5, 900 + s, 400) for s in range(S)]
+    full = [synth.zipf_tokens(w, seed + s, per_seq) for s in range(S)]
     pos = [0] * S
-    rng = np.random.default_rng(4)
-    for rnd in range(6):
+    rng = np.random.default_rng(seed)
+    matched = np.zeros(w.K + 1, np.int64)
+    for rnd in range(rounds):
         chunks = []
         for s in range(S):
-            n = min(int(rng.integers(0, 120)) if rnd < 5 else 400, 400 - pos[s])
+            n = min(int(rng.integers(0, 120)) if rnd < rounds - 1 else per_seq, per_seq - pos[s])
             chunks.append(full[s][pos[s]:pos[s] + n])
         lens = [len(x) for x in chunks]
         cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
         flat = np.concatenate(chunks).astype(np.int32) if sum(lens) else np.zeros(0, np.int32)
         n = flat.size
-        out = torch.empty((max(n, 1), w5.d), dtype=torch.int16, device=DEV)
+        out = torch.empty((max(n, 1), w.d), dtype=torch.int16, device=DEV)
         row = torch.empty(max(n, 1), dtype=torch.int32, device=DEV)
+        ln = torch.empty(max(n, 1), dtype=torch.uint8, device=DEV)
         scone.scone_embed_varlen(c.table, torch.from_numpy(flat).to(DEV),
-                                 torch.from_numpy(cu).to(DEV), out[:n], state=st, row=row[:n])
+                                 torch.from_numpy(cu).to(DEV), out[:n], state=st, row=row[:n],
+                                 len=ln[:n])
         torch.cuda.synchronize()
+        g_out = out[:n].cpu().numpy().view(np.uint16)
+        g_row, g_len = row[:n].cpu().numpy(), ln[:n].cpu().numpy()
         for s in range(S):
             a, b = pos[s], pos[s] + lens[s]
-            exp_out, exp_row, _, rc = c.oracle.embed(np.asarray(full[s][:b], np.int32)[None, :],
-                                                     c.F, c.T)
-            assert np.array_equal(row[:n].cpu().numpy()[cu[s]:cu[s + 1]],
-                                  exp_row[0, a:b].astype(np.int32)), (rnd, s)
-            assert np.array_equal(out[:n].cpu().numpy().view(np.uint16)[cu[s]:cu[s + 1]],
-                                  exp_out[0, a:b]), (rnd, s)
+            exp_out, exp_row, exp_len, rc = c.oracle.embed(
+                np.asarray(full[s][:b], np.int32)[None, :], c.F, c.T)
+            sl = slice(cu[s], cu[s + 1])
+            assert np.array_equal(g_row[sl], exp_row[0, a:b].astype(np.int32)), (rnd, s)
+            assert np.array_equal(g_len[sl], exp_len[0, a:b]), (rnd, s)
+            assert np.array_equal(g_out[sl], exp_out[0, a:b]), (rnd, s)
+            matched += np.bincount(exp_len[0, a:b], minlength=w.K + 1)
             pos[s] = b
+    assert pos == [per_seq] * S
     assert scone.scone_status(c.table) == 0
+    info = c.table.info()
     st.close()
     c.table.close()
+    return matched, info
+
+
+def test_k5_ragged_and_continued():
+    """K = 5 over the stress law, with phrases injected often enough that 4-
+    and 5-gram matches occur (and cross chunk boundaries)."""
+    w5 = synth.WORKLOADS["stress_k5"].scaled("varlen_k5", B=1, L=64, d=64,
+                                             quotas=((2, 3000), (3, 3000), (4, 1500), (5, 1500)),
+                                             inject_p=0.05, n_phrases=256, phrase_len=(5, 7))
+    matched, _ = ragged_continued(w5, 900)
+    assert matched[4] and matched[5]
+
+
+@pytest.mark.parametrize("name,K,vocab,slot_bytes", [
+    ("k5_fmt32", 5, 300000, 32),
+    ("k8_fmt32", 8, 1 << 20, 32),
+    ("k8_fmt16", 8, 2000, 16),
+    ("k2_fmt16", 2, 2000, 16),
+])
+def test_key_formats_ragged_and_continued(name, K, vocab, slot_bytes):
+    """Every (key format, K bound) instance of the varlen kernel: 16- and
+    32-byte slots with K up to 8, over phrase-injected streams so that long
+    matches occur across chunk boundaries."""
+    w = synth.Workload(name, 60 + K, vocab, 1.05, 1, 64, tuple((n, 1500) for n in range(2, K + 1)),
+                       K, 64, inject_p=0.05, n_phrases=256, phrase_len=(K, K + 2))
+    matched, info = ragged_continued(w, 1000 + K)
+    assert info["slot_bytes"] == slot_bytes
+    assert matched[2] and matched[K]
