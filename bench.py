@@ -144,29 +144,32 @@ def measured_peaks():
     return 6800.0, "fallback"
 
 
-def kernel_source_hash() -> str:
+EMBED_SOURCES = ("scone_embed.cu", "scone_device.cuh", "scone_host.h")
+DISCOVER_SOURCES = ("scone_discover.cu", "scone_device.cuh", "scone_host.h")
+
+
+def kernel_source_hash(files=EMBED_SOURCES) -> str:
     """Hash of the code (comments and whitespace removed) of the sources that
-    compile into the fused prefill kernel."""
+    compile into a profiled kernel (default: the fused prefill kernel)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2502_01637_gb300", "csrc")
-    files = [os.path.join(csrc, f) for f in ("scone_embed.cu", "scone_device.cuh", "scone_host.h")]
-    for f in files:
+    for f in (os.path.join(csrc, name) for name in files):
         code = re.sub(r"/\*.*?\*/", " ", open(f).read(), flags=re.S)
         code = re.sub(r"//[^\n]*", " ", code)
         h.update(" ".join(code.split()).encode())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str):
+def profiled_traffic(workload: str, kernel: str = "embed_kernel", files=EMBED_SOURCES):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
     on the current kernel sources; else None."""
-    p = os.path.join(ROOT, "profiles", f"embed_kernel_{workload}.md")
+    p = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
     if not os.path.exists(p):
         return None
     txt = open(p).read()
     m = re.search(r"dram_bytes_per_launch:\s*(\d+)", txt)
     s = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", txt)
-    if not m or not s or s.group(1) != kernel_source_hash():
+    if not m or not s or s.group(1) != kernel_source_hash(files):
         return None
     return int(m.group(1))
 
@@ -1230,7 +1233,8 @@ def bench_discover(args, world, rank, local):
             "peak": hbm,
             "unit": "GB/s",
             "frac": achieved / hbm,
-            "traffic": None,
+            "traffic": (profiled_traffic(w.name, "bincount_kernel", DISCOVER_SOURCES)
+                        if w.name == "discover" else None),
             "peak_source": peak_src,
             "algorithmic_bytes_per_launch": bytes_count,
             "kernel": ("bincount_kernel of scan 2 (10 B per binned window + 8 B per chunk and "
