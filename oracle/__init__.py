@@ -59,6 +59,8 @@ def _load():
     lib.oracle_embed.argtypes = [ctypes.c_void_p, _i32p, ctypes.c_int32, ctypes.c_int32,
                                  _u16p, ctypes.c_int64, _u16p, ctypes.c_int32, _u16p, _i64p, _u8p]
     lib.oracle_embed.restype = ctypes.c_int
+    lib.oracle_embed_threads.argtypes = lib.oracle_embed.argtypes + [ctypes.c_int32]
+    lib.oracle_embed_threads.restype = ctypes.c_int
     lib.oracle_decode.argtypes = [ctypes.c_void_p, ctypes.c_int32, _i32p, ctypes.c_int32, _i32p,
                                   ctypes.c_int32, _i32p, _u16p, ctypes.c_int64, _u16p,
                                   ctypes.c_int32, _u16p, _i64p, _u8p]
@@ -144,8 +146,9 @@ class Oracle:
             raise OracleError(rc, "oracle_select_at")
         return row, ln, rc
 
-    def embed(self, tok: np.ndarray, F: np.ndarray, T: np.ndarray):
+    def embed(self, tok: np.ndarray, F: np.ndarray, T: np.ndarray, threads: int = 1):
         """Algorithm 1 output. F [N,d], T [vocab,d] as uint16 (raw bf16 words).
+        threads > 1 splits the sequences over that many std::threads.
 
         Returns (out uint16 [B,L,d], row int64 [B,L], len uint8 [B,L], status).
         """
@@ -159,9 +162,10 @@ class Oracle:
         row = np.empty((B, L), np.int64)
         ln = np.empty((B, L), np.uint8)
         Fp = F if F.size else np.zeros((1, d), np.uint16)
-        rc = _load().oracle_embed(self._h, _ptr(tok, _i32p), B, L, _ptr(Fp, _u16p), F.shape[0],
-                                  _ptr(T, _u16p), d, _ptr(out, _u16p), _ptr(row, _i64p),
-                                  _ptr(ln, _u8p))
+        args = (self._h, _ptr(tok, _i32p), B, L, _ptr(Fp, _u16p), F.shape[0], _ptr(T, _u16p), d,
+                _ptr(out, _u16p), _ptr(row, _i64p), _ptr(ln, _u8p))
+        rc = (_load().oracle_embed_threads(*args, int(threads)) if threads > 1
+              else _load().oracle_embed(*args))
         if rc not in (OK, ERR_TOKEN_RANGE):
             raise OracleError(rc, "oracle_embed")
         return out, row, ln, rc

@@ -40,6 +40,7 @@
 #include <cstdint>
 #include <cstring>
 #include <map>
+#include <thread>
 #include <vector>
 
 namespace {
@@ -192,6 +193,35 @@ int oracle_embed(const void* tp, const int32_t* tok, int32_t B, int32_t L, const
       if (row) row[p] = r;
       if (len) len[p] = (uint8_t)(i - j + 1);
     }
+  }
+  return rc;
+}
+
+// The same definition with the sequences split over `threads` std::threads
+// (contiguous ranges; each thread runs oracle_embed on its own range, the table
+// is only read). Used to time the baseline on every host core.
+int oracle_embed_threads(const void* tp, const int32_t* tok, int32_t B, int32_t L,
+                         const uint16_t* F, int64_t n_F, const uint16_t* T, int32_t d,
+                         uint16_t* out, int64_t* row, uint8_t* len, int32_t threads) {
+  if (B < 0 || L < 0 || d <= 0) return -1;
+  if (threads < 1) threads = 1;
+  if (threads > B) threads = B > 0 ? B : 1;
+  std::vector<int> rcs((size_t)threads, 0);
+  std::vector<std::thread> pool;
+  for (int32_t k = 0; k < threads; ++k) {
+    const int64_t b0 = (int64_t)B * k / threads, b1 = (int64_t)B * (k + 1) / threads;
+    pool.emplace_back([=, &rcs] {
+      const int64_t p0 = b0 * L;
+      rcs[(size_t)k] = oracle_embed(tp, tok + p0, (int32_t)(b1 - b0), L, F, n_F, T, d,
+                                    out + p0 * d, row ? row + p0 : nullptr,
+                                    len ? len + p0 : nullptr);
+    });
+  }
+  for (std::thread& th : pool) th.join();
+  int rc = 0;
+  for (int r : rcs) {
+    if (r == -1) return -1;
+    if (r != 0) rc = r;
   }
   return rc;
 }

@@ -288,3 +288,22 @@ def test_decode_equals_prefill(K):
         assert (ln[:, s] >= 2).sum() >= steps - 1
     assert (ln[0, hl > 0] >= 2).all() and (ln[0, hl == 0] == 1).all()
     assert (ln > 2).any()
+
+
+@pytest.mark.parametrize("threads", [2, 5, 64])
+def test_threaded_embed_equals_single_thread(threads):
+    """The std::thread split over sequences (used for the multi-core CPU
+    timing) gives the single-thread result, including the status of an
+    out-of-range token in one of the ranges."""
+    w = synth.WORKLOADS["tiny"].scaled("tiny_mt", B=9, L=37)
+    ft, fl, _ = synth.fgram_set(w)
+    tok = synth.query_tokens(w)
+    tok[6, 11] = w.vocab
+    F = synth.rows_cpu(synth.F_seed(w), w.d, np.arange(len(fl)))
+    T = synth.rows_cpu(synth.T_seed(w), w.d, np.arange(w.vocab))
+    o = oracle.Oracle(ft, fl, w.K, w.vocab)
+    a = o.embed(tok, F, T)
+    b = o.embed(tok, F, T, threads=threads)
+    assert a[3] == b[3] == oracle.ERR_TOKEN_RANGE
+    for x, y in zip(a[:3], b[:3]):
+        assert np.array_equal(x, y)
