@@ -300,8 +300,12 @@ int scone_embed_gather(const scone_table* table, const int32_t* tok, const int32
 /*
  * scone_embed — Algorithm 1 end to end (Sec. 3, inference branch) in one
  * launch: match and gather fused, no intermediate row array in memory.
- * tok device [B * L]; out device [B * L * d]; row / len as in scone_match,
- * each may be NULL. Async.
+ * tok int32 [B * L], device-accessible: device memory, or page-locked host
+ * memory mapped for the device (cudaHostAlloc, cudaHostRegister,
+ * scone_host_alloc), which the kernel then reads over the host link with no
+ * staging copy; out device [B * L * d]; row / len as in scone_match, each
+ * may be NULL. Async; host tokens must stay unchanged until the call's work
+ * on the stream is done.
  */
 int scone_embed(const scone_table* table, const int32_t* tok, int32_t B, int32_t L,
                 scone_bf16* out, int32_t* row, uint8_t* len, void* stream);

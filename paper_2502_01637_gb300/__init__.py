@@ -297,10 +297,22 @@ def scone_embed_gather(table: Table, tok, row, out, stream=None) -> None:
                                              _ptr(out), _stream(stream)), "scone_embed_gather")
 
 
+def _tok_ptr(tok) -> int:
+    """Token address for the kernels: a CUDA tensor, or a pinned (page-locked,
+    device-mapped) CPU tensor that the kernel reads over the host link."""
+    if hasattr(tok, "is_cuda") and not tok.is_cuda and not tok.is_pinned():
+        raise ValueError("host tokens must be pinned (tensor.pin_memory()) to be read by "
+                         "the device")
+    if isinstance(tok, np.ndarray):
+        raise ValueError("tokens must be a CUDA or pinned CPU tensor")
+    return _ptr(tok)
+
+
 def scone_embed(table: Table, tok, out, row=None, len=None, stream=None) -> None:
-    """Fused Algorithm 1: out [B*L, d] bf16 rows; row / len optional."""
+    """Fused Algorithm 1: out [B*L, d] bf16 rows; row / len optional. tok may
+    be a pinned CPU tensor: the kernel then reads it over the host link."""
     B, L = _bl(tok)
-    _check(load_library().scone_embed(table.handle, _ptr(tok), B, L, _ptr(out), _ptr(row),
+    _check(load_library().scone_embed(table.handle, _tok_ptr(tok), B, L, _ptr(out), _ptr(row),
                                       _ptr(len), _stream(stream)), "scone_embed")
 
 

@@ -300,6 +300,20 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
     scone_table_destroy(t);
     return SCONE_ERR_NOMEM;
   }
+  // the status mirror is an optimisation: without it scone_status copies the word
+  void* mirror = nullptr;
+  if (cudaHostAlloc(&mirror, sizeof(int), cudaHostAllocMapped) == cudaSuccess) {
+    t->status_host = static_cast<int*>(mirror);
+    *t->status_host = 0;
+    void* dp = nullptr;
+    if (cudaHostGetDevicePointer(&dp, mirror, 0) == cudaSuccess) {
+      t->status_host_dev = static_cast<int*>(dp);
+    } else {
+      cudaFreeHost(mirror);
+      t->status_host = nullptr;
+    }
+  }
+  cudaGetLastError();
   t->fmt = fmt;
   TableView& v = t->view;
   v.slots = t->slots;
@@ -378,6 +392,7 @@ extern "C" int scone_table_destroy(scone_table* t) {
   if (t->slots || t->status || t->zero_row) cudaDeviceSynchronize();
   if (t->slots) cudaFree(t->slots);
   if (t->status) cudaFree(t->status);
+  if (t->status_host) cudaFreeHost(t->status_host);
   if (t->zero_row) cudaFree(t->zero_row);
   if (prev >= 0 && prev != t->device) cudaSetDevice(prev);
   delete t;
@@ -402,9 +417,30 @@ extern "C" int scone_table_set_copy_mode(scone_table* t, int32_t mode) {
   return SCONE_OK;
 }
 
+namespace scone {
+namespace {
+
+// Moves the sticky status word to the host mirror and clears it, in stream
+// order: one launch instead of a copy and a memset.
+__global__ void status_fetch_kernel(int* status, int* host_mirror) {
+  *host_mirror = *status;
+  *status = 0;
+}
+
+}  // namespace
+}  // namespace scone
+
 extern "C" int scone_status(const scone_table* t, void* stream) {
   if (!t) return SCONE_ERR_INVALID_ARG;
   cudaStream_t s = (cudaStream_t)stream;
+  if (t->status_host) {
+    scone::status_fetch_kernel<<<1, 1, 0, s>>>(t->status, t->status_host_dev);
+    if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess) {
+      cudaGetLastError();
+      return SCONE_ERR_CUDA;
+    }
+    return *static_cast<volatile int*>(t->status_host);
+  }
   int code = 0;
   if (cudaMemcpyAsync(&code, t->status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
       cudaMemsetAsync(t->status, 0, sizeof(int), s) != cudaSuccess ||

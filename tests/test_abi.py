@@ -112,3 +112,18 @@ def test_key_format_boundaries():
     assert rc == scone.SCONE_ERR_INVALID_ARG         # 8*27 = 216 <= 220: format fits
     rc = _build_rc(np.zeros((1, 8), np.int32), np.array([2], np.uint8), 8, (1 << 27) + 1)
     assert rc == scone.SCONE_ERR_UNSUPPORTED         # 8*28 = 224 > 220
+
+
+def test_host_tokens_must_be_pinned():
+    """Tokens the kernels read from host memory must be page-locked: the
+    binding refuses pageable CPU tensors and numpy arrays before any launch."""
+    import numpy as np
+    import pytest
+    import torch
+
+    import paper_2502_01637_gb300 as scone
+
+    with pytest.raises(ValueError):
+        scone._tok_ptr(torch.zeros(8, dtype=torch.int32))
+    with pytest.raises(ValueError):
+        scone._tok_ptr(np.zeros(8, np.int32))

@@ -207,6 +207,26 @@ def test_host_mapped_F():
     buf.free()
 
 
+def test_pinned_host_tokens():
+    """scone_embed reading its tokens straight from pinned host memory (the
+    zero-copy input of the end-to-end path) gives the device-token result,
+    including an out-of-range token's zero row and status."""
+    w = TINY.scaled("tiny_pinned", B=5, L=333)
+    case = SmallCase(w)
+    case.tok[3, 17] = w.vocab + 5
+    table = case.build()
+    host = torch.from_numpy(case.tok).pin_memory()
+    out = torch.empty((case.tok.size, w.d), dtype=torch.int16, device=DEV)
+    row = torch.empty(case.tok.size, dtype=torch.int32, device=DEV)
+    ln = torch.empty(case.tok.size, dtype=torch.uint8, device=DEV)
+    scone.scone_embed(table, host, out, row, ln)
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+    assert_parity(case, out.cpu().numpy().view(np.uint16), row.cpu().numpy(), ln.cpu().numpy())
+    with pytest.raises(ValueError):
+        scone.scone_embed(table, torch.from_numpy(case.tok), out)   # pageable: refused
+    table.close()
+
+
 # ------------------------------------------------------------------ decode
 def _decode_case(K, S, steps, vocab=2000, d=96, seed=0):
     rng = np.random.default_rng(seed)
