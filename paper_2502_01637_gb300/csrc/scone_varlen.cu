@@ -11,12 +11,15 @@
 //
 // varlen_embed_kernel is the fused kernel's scheme (persistent grid, an even
 // split of positions over warps, a lane per position, then a warp-wide row
-// copy) with two changes per lane: the sequence of position p is found by a
-// binary search of cu (the last b with cu[b] <= p, so empty sequences are
-// skipped), and window tokens left of the chunk come from the history.
-// varlen_hist_kernel then replaces each continued slot's history with the
-// last K-1 tokens of history ++ chunk; it is a separate launch because the
-// embedding kernel's lanes read the old history.
+// copy) with two changes per lane: the sequence of position p is found in cu
+// (the last b with cu[b] <= p, so empty sequences are skipped) by a galloping
+// search that starts at the sequence of the warp's previous tile, and window
+// tokens left of the chunk come from the history. varlen_hist_kernel then
+// replaces each continued slot's history with the last K-1 tokens of
+// history ++ chunk; it is a separate launch because the embedding kernel's
+// lanes read the old history, made with programmatic dependent launch: it is
+// scheduled while the embedding kernel runs and waits on the device
+// (griddepcontrol.wait) until that grid has finished.
 
 #include "scone_host.h"
 
@@ -27,10 +30,23 @@ namespace {
 constexpr int kVThreads = 256;
 constexpr int kVWarps = kVThreads / 32;
 
-// Last b in [0, n_seq) with cu[b] <= p (cu[0] = 0 <= p).
-__device__ __forceinline__ int32_t seq_of(const int32_t* __restrict__ cu, int32_t n_seq,
-                                          int64_t p) {
-  int32_t lo = 0, hi = n_seq - 1;
+// Last b in [b0, n_seq) with cu[b] <= p, given cu[b0] <= p (b0 = 0, or the
+// sequence of an earlier position): steps of 1, 2, 4, .. from b0 until one
+// overshoots, then a binary search below it. A position in the sequence of
+// the previous one costs one read; indices stay in [b0, n_seq).
+__device__ __forceinline__ int32_t seq_from(const int32_t* __restrict__ cu, int32_t n_seq,
+                                            int64_t p, int32_t b0) {
+  int32_t lo = b0, hi = n_seq - 1, step = 1;
+  while (lo < hi) {
+    const int32_t probe = hi - lo > step ? lo + step : hi;
+    if ((int64_t)__ldg(cu + probe) <= p) {
+      lo = probe;
+      step <<= 1;
+    } else {
+      hi = probe - 1;
+      break;
+    }
+  }
   while (lo < hi) {
     const int32_t mid = (lo + hi + 1) >> 1;
     if ((int64_t)__ldg(cu + mid) <= p) lo = mid;
@@ -44,7 +60,7 @@ __device__ __forceinline__ int32_t seq_of(const int32_t* __restrict__ cu, int32_
 template <int FMT, int KT>
 __device__ __forceinline__ int32_t match_varlen(const TableView& t,
                                                 const int32_t* __restrict__ tok,
-                                                const int32_t* __restrict__ cu, int32_t n_seq,
+                                                const int32_t* __restrict__ cu, int32_t b,
                                                 const int32_t* __restrict__ hist,
                                                 const int32_t* __restrict__ hist_len,
                                                 const int32_t* __restrict__ slot, int32_t S,
@@ -55,7 +71,6 @@ __device__ __forceinline__ int32_t match_varlen(const TableView& t,
     *len = 0;
     return -1;
   }
-  const int32_t b = seq_of(cu, n_seq, p);
   const int32_t c0 = __ldg(cu + b);
   const int64_t i = p - (c0 > 0 ? c0 : 0);   // offset in the chunk, never left of tok[0]
   int32_t h = 0;
@@ -97,17 +112,22 @@ __global__ void __launch_bounds__(kVThreads, VarlenTuning<KT>::kMinBlocks)
   __shared__ const void* src_s[kVWarps][32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int row_bytes = t.d * 2;
+  // the history kernel that follows may be scheduled now; it waits for this grid
+  asm volatile("griddepcontrol.launch_dependents;");
   const int64_t nw = (int64_t)gridDim.x * kVWarps, w = (int64_t)blockIdx.x * kVWarps + warp;
   const int64_t lo = n_tok * w / nw, hi = n_tok * (w + 1) / nw;
+  int32_t bq = 0;   // sequence of the warp's previous position (positions only increase)
   for (int64_t base = lo; base < hi; base += 32) {
     const int nrows = (int)(hi - base < 32 ? hi - base : 32);
     const int64_t p = base + lane;
     const void* src = nullptr;
+    const int32_t b = lane < nrows ? seq_from(cu, n_seq, p, bq) : bq;
+    bq = __shfl_sync(0xFFFFFFFFu, b, nrows - 1);
     if (lane < nrows) {
       const int32_t x = __ldg(tok + p);
       int len = 0, err = 0;
-      const int32_t r = match_varlen<FMT, KT>(t, tok, cu, n_seq, hist, hist_len, slot, S, H, p,
-                                              x, &len, &err);
+      const int32_t r = match_varlen<FMT, KT>(t, tok, cu, b, hist, hist_len, slot, S, H, p, x,
+                                              &len, &err);
       if (err) {
         record_error(t.status, err);
       } else {
@@ -132,6 +152,9 @@ __global__ void __launch_bounds__(256)
                        const int32_t* __restrict__ cu, int32_t n_seq, int32_t* __restrict__ hist,
                        int32_t* __restrict__ hist_len, const int32_t* __restrict__ slot,
                        int32_t S, int32_t H) {
+  // launched as a programmatic dependent of the embedding kernel, whose lanes
+  // read the histories this kernel rewrites: wait until that grid is done
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int32_t b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= n_seq || H == 0) return;
   const int32_t s = slot ? slot[b] : b;
@@ -204,10 +227,21 @@ extern "C" int scone_embed_varlen(const scone_table* tb, const int32_t* tok, int
     if (cudaGetLastError() != cudaSuccess) return SCONE_ERR_CUDA;
   }
   if (state && H > 0) {
-    varlen_hist_kernel<<<(n_seq + 255) / 256, 256, 0, s>>>(tok, n_tok, cu_seqlens, n_seq,
-                                                         state->hist, state->hist_len, slot, S,
-                                                         H);
-    if (cudaGetLastError() != cudaSuccess) return SCONE_ERR_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((n_seq + 255) / 256));
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, varlen_hist_kernel, tok, n_tok, cu_seqlens, n_seq, state->hist,
+                           state->hist_len, slot, S, H) != cudaSuccess) {
+      cudaGetLastError();
+      return SCONE_ERR_CUDA;
+    }
   }
   return SCONE_OK;
 }
