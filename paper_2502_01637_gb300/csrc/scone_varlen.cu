@@ -82,7 +82,8 @@ __device__ __forceinline__ int32_t match_varlen(const TableView& t,
       *len = 0;
       return -1;
     }
-    h = hist_len[s];
+    // only the chunk's first K-1 windows reach into the history
+    if (i < t.K - 1) h = hist_len[s];
     hrow = hist + (int64_t)s * H;
   }
   const int64_t known = i + 1 + h;        // tokens of the sequence up to p
