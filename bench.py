@@ -1271,7 +1271,7 @@ def bench_discover(args, world, rank, local):
                         if w.name == "discover" else None),
             "peak_source": peak_src,
             "algorithmic_bytes_per_launch": bytes_count,
-            "kernel": ("bincount_kernel of scan 2 (10 B per binned window + 8 B per chunk and "
+            "kernel": ("bincount_kernel of scan 2 (10 B per binned window + 4 B per chunk and "
                        "bin + 64 B per distinct key; bound in practice by L2 atomics on the "
                        "resident table region, not by DRAM)"),
             "kernel_ms": ms_count,
