@@ -41,8 +41,8 @@ SCONE_GEMM_RESIDUAL = 1
 SCONE_GEMM_SWIGLU = 2
 
 EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noalloc",
-           "scone_table_get_info",
-           "scone_table_set_probe_limit", "scone_table_set_copy_mode", "scone_match", "scone_embed_gather", "scone_embed",
+           "scone_table_get_info", "scone_table_set_probe_limit", "scone_table_set_copy_mode",
+           "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
            "scone_embed_varlen", "scone_rowstore_open", "scone_rowstore_gather",
@@ -388,8 +388,8 @@ def scone_fgram_model_destroy(model: FgramModel) -> None:
     model.close()
 
 
-def scone_fgram_precompute(model: FgramModel, fgram_tok, fgram_len, T, F, vocab: Optional[int] = None,
-                           stream=None) -> None:
+def scone_fgram_precompute(model: FgramModel, fgram_tok, fgram_len, T, F,
+                           vocab: Optional[int] = None, stream=None) -> None:
     """F rows of the f-grams: fgram_tok [n, K] int32 and fgram_len [n] uint8 device
     tensors, T [vocab, d] device, F [n, d] device tensor (or host-mapped address)."""
     n, K = fgram_tok.shape

@@ -960,8 +960,9 @@ extern "C" int scone_discover_destroy(scone_discover* ws) {
   return SCONE_OK;
 }
 
-extern "C" int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int32_t B, int32_t L, int32_t vocab,
-                                    int32_t K, int64_t S, int32_t min_count, int32_t* fgram_tok,
+extern "C" int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int32_t B, int32_t L,
+                                    int32_t vocab, int32_t K, int64_t S, int32_t min_count,
+                                    int32_t* fgram_tok,
                                     uint8_t* fgram_len, uint32_t* fgram_count, int64_t* n_out,
                                     scone_discover_stats* stats, void* stream) {
   if (B < 0 || L < 0 || vocab < 1 || K < 2 || K > 8 || S < 0 || min_count < 1 || !n_out)
@@ -976,7 +977,6 @@ extern "C" int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int3
   if (stats) *stats = st;
   if (N == 0) return SCONE_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-
 
   Events evs;
   cudaEvent_t ev_begin = evs.make(), ev_end = evs.make();

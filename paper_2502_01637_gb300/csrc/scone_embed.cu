@@ -52,7 +52,8 @@ int blocks_per_sm(const void* fn, int threads, size_t smem) {
   auto it = cache.find(key);
   if (it != cache.end()) return it->second;
   int n = 1;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, smem) != cudaSuccess || n < 1) {
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, smem) != cudaSuccess ||
+      n < 1) {
     cudaGetLastError();
     n = 1;
   }

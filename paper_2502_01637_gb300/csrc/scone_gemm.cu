@@ -603,7 +603,8 @@ int gemm_bf16_variant(const uint16_t* A, const uint16_t* B, const uint16_t* R, u
     CUtensorMap pa, pb;
     if (!make_map(&pa, A, M, K, 128) || !make_map(&pb, B, N, K, 128)) return SCONE_ERR_CUDA;
     switch (epi) {
-      case GEMM_EPI_STORE: return launch_pair<GEMM_EPI_STORE>(pa, pb, M, N, K, R, C, ldc, status, s);
+      case GEMM_EPI_STORE:
+        return launch_pair<GEMM_EPI_STORE>(pa, pb, M, N, K, R, C, ldc, status, s);
       case GEMM_EPI_RESIDUAL:
         return launch_pair<GEMM_EPI_RESIDUAL>(pa, pb, M, N, K, R, C, ldc, status, s);
       case GEMM_EPI_SWIGLU:

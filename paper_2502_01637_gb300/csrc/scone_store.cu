@@ -422,8 +422,8 @@ extern "C" int scone_rowstore_gather(scone_rowstore* st, const scone_table* tb,
   const int64_t warps = (int64_t)n_miss + n_fill;
   fill_kernel<<<(unsigned)((warps + kStoreWarps - 1) / kStoreWarps), kStoreThreads, 0, s>>>(
       st->d_stage, st->row_bytes, st->d_miss_pos, st->d_miss_src, n_miss, st->d_fill,
-      st->d_fill + st->stage_cap, st->d_fill_src, (int)n_fill, reinterpret_cast<uint8_t*>(out), reinterpret_cast<uint8_t*>(st->cache),
-      st->tag);
+      st->d_fill + st->stage_cap, st->d_fill_src, (int)n_fill, reinterpret_cast<uint8_t*>(out),
+      reinterpret_cast<uint8_t*>(st->cache), st->tag);
   if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
     return SCONE_ERR_CUDA;
   st->stats.rows_read += nu;

@@ -176,7 +176,8 @@ uint64_t synth_mix64(uint64_t z) { return mix64(z); }
 uint64_t synth_draw(uint64_t seed, uint64_t ctr) { return draw(seed, ctr); }
 
 // Seed of sub-stream `sub` of stream `stream_id` of workload `workload_id`.
-uint64_t synth_stream_seed(uint64_t master, uint32_t workload_id, uint32_t stream_id, uint64_t sub) {
+uint64_t synth_stream_seed(uint64_t master, uint32_t workload_id, uint32_t stream_id,
+                           uint64_t sub) {
   const uint64_t s = mix64(master ^ (((uint64_t)workload_id << 32) | stream_id));
   return mix64(s ^ mix64(sub + kGamma));
 }
