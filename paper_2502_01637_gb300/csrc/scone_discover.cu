@@ -847,6 +847,15 @@ double elapsed_ms(cudaEvent_t a, cudaEvent_t b) {
   return ms;
 }
 
+// Pinned host memory that the call's small device-to-host reads land in (a
+// copy into pageable memory is staged and synchronous in the driver).
+struct HostStage {
+  uint32_t hll[kHllRegs];
+  unsigned long long counters[16];
+  DiscoverErr err;
+  unsigned int hist[256];
+};
+
 // Named buffers of a workspace.
 enum Buf {
   kBufNames, kBufNamesNext, kBufRecKey, kBufRecLoc, kBufRecOff, kBufRecRes, kBufHot, kBufFlags,
@@ -863,6 +872,7 @@ enum Buf {
 // Reusable device workspace: grow-only buffers, kept between calls.
 struct scone_discover {
   int device = 0;
+  scone::HostStage* stage = nullptr;   // pinned, allocated on first use
   // counting-table slots per estimated distinct key: load factor 0.25. On the
   // 1.07e9-token corpus 4 beat 2.5 (longer probe chains) and 8 to 16 (more
   // table to clear and to miss in L2) by 2 to 4 ms per call.
@@ -896,9 +906,21 @@ struct scone_discover {
     for (size_t b : bytes) t += b;
     return t;
   }
+  scone::HostStage* host_stage() {
+    if (!stage) {
+      void* p = nullptr;
+      if (cudaHostAlloc(&p, sizeof(scone::HostStage), cudaHostAllocDefault) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+      }
+      stage = static_cast<scone::HostStage*>(p);
+    }
+    return stage;
+  }
   ~scone_discover() {
     for (void* p : ptr)
       if (p) cudaFree(p);
+    if (stage) cudaFreeHost(stage);
   }
 };
 
@@ -908,13 +930,13 @@ namespace {
 // HyperLogLog estimate of the number of distinct keys from the sketch
 // registers (Flajolet, Fusy, Gandouet, Meunier 2007), with linear counting
 // for small cardinalities; 64-bit hashes need no large-range correction.
-double hll_estimate(const std::vector<uint32_t>& reg) {
-  const double m = (double)reg.size();
+double hll_estimate(const uint32_t* reg, int n_regs) {
+  const double m = (double)n_regs;
   double sum = 0.0;
   int zeros = 0;
-  for (uint32_t r : reg) {
-    sum += std::ldexp(1.0, -(int)r);
-    zeros += r == 0;
+  for (int j = 0; j < n_regs; ++j) {
+    sum += std::ldexp(1.0, -(int)reg[j]);
+    zeros += reg[j] == 0;
   }
   double e = 0.7213 / (1.0 + 1.079 / m) * m * m / sum;
   if (e <= 2.5 * m && zeros > 0) e = m * std::log(m / zeros);
@@ -1035,7 +1057,8 @@ extern "C" int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int3
   auto* counters = static_cast<unsigned long long*>(get(kBufCounters, kCounters * 8));
   auto* d_err = static_cast<DiscoverErr*>(get(kBufErr, sizeof(DiscoverErr)));
   auto* hll = static_cast<uint32_t*>(get(kBufHll, kHllRegs * sizeof(uint32_t)));
-  if (nomem) return SCONE_ERR_NOMEM;
+  HostStage* hs = ws->host_stage();
+  if (nomem || !hs) return SCONE_ERR_NOMEM;
   if (cudaMemsetAsync(d_err, 0, sizeof(DiscoverErr), s) != cudaSuccess) return SCONE_ERR_CUDA;
   if (cudaFuncSetAttribute((const void*)bin_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)kBinSmem) != cudaSuccess)
@@ -1083,15 +1106,14 @@ extern "C" int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int3
     if (ev_b1[n]) cudaEventRecord(ev_b1[n], s);
     if (cudaGetLastError() != cudaSuccess) return SCONE_ERR_CUDA;
     // size the table from the sketch of the distinct keys
-    std::vector<uint32_t> reg(kHllRegs);
-    unsigned long long n_cand = 0;
-    if (cudaMemcpyAsync(reg.data(), hll, kHllRegs * sizeof(uint32_t), cudaMemcpyDeviceToHost,
-                        s) != cudaSuccess ||
-        cudaMemcpyAsync(&n_cand, counters, sizeof(n_cand), cudaMemcpyDeviceToHost, s) !=
+    if (cudaMemcpyAsync(hs->hll, hll, kHllRegs * sizeof(uint32_t), cudaMemcpyDeviceToHost, s) !=
             cudaSuccess ||
+        cudaMemcpyAsync(hs->counters, counters, sizeof(unsigned long long),
+                        cudaMemcpyDeviceToHost, s) != cudaSuccess ||
         cudaStreamSynchronize(s) != cudaSuccess)
       return SCONE_ERR_CUDA;
-    const double est = hll_estimate(reg);
+    const unsigned long long n_cand = hs->counters[0];
+    const double est = hll_estimate(hs->hll, kHllRegs);
     // at most one distinct n-gram per counted window: load factor <= 0.5
     const uint64_t worst = 2 * n_cand > 64 ? 2 * n_cand : 64;
     const double want = std::ceil(ws->table_slack * est);
@@ -1120,11 +1142,14 @@ extern "C" int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int3
       if (ev_f1[n]) cudaEventRecord(ev_f1[n], s);
       scan_kernel<<<1, kScanThreads, 0, s>>>(chunk_cnt, chunk_off, n_wchunks, counters + 2);
       if (cudaGetLastError() != cudaSuccess) return SCONE_ERR_CUDA;
-      if (cudaMemcpyAsync(h, counters, sizeof(h), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
-          cudaMemcpyAsync(&herr, d_err, sizeof(herr), cudaMemcpyDeviceToHost, s) !=
+      if (cudaMemcpyAsync(hs->counters, counters, sizeof(h), cudaMemcpyDeviceToHost, s) !=
+              cudaSuccess ||
+          cudaMemcpyAsync(&hs->err, d_err, sizeof(herr), cudaMemcpyDeviceToHost, s) !=
               cudaSuccess ||
           cudaStreamSynchronize(s) != cudaSuccess)
         return SCONE_ERR_CUDA;
+      std::memcpy(h, hs->counters, sizeof(h));
+      herr = hs->err;
       if (herr.token_range) return SCONE_ERR_TOKEN_RANGE;
       if (!herr.table_full) break;
       if (cap >= worst) return SCONE_ERR_TABLE_FULL;
@@ -1202,12 +1227,13 @@ extern "C" int scone_fgram_discover(scone_discover* ws, const int32_t* tok, int3
     const dim3 hg((unsigned)grid_for((const void*)hist_kernel, 256, 0, (max_size + 255) / 256),
                   (unsigned)ls.n_lists);
     for (int shift = 24; shift >= 0; shift -= 8) {
-      unsigned int hh[256];
+      const unsigned int* hh = hs->hist;
       if (cudaMemsetAsync(hist, 0, 256 * sizeof(unsigned int), s) != cudaSuccess)
         return SCONE_ERR_CUDA;
       hist_kernel<<<hg, 256, 0, s>>>(ls, shift, mask, prefix, hist);
       if (cudaGetLastError() != cudaSuccess ||
-          cudaMemcpyAsync(hh, hist, sizeof(hh), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+          cudaMemcpyAsync(hs->hist, hist, 256 * sizeof(unsigned int), cudaMemcpyDeviceToHost,
+                          s) != cudaSuccess ||
           cudaStreamSynchronize(s) != cudaSuccess)
         return SCONE_ERR_CUDA;
       int b = 255;

@@ -33,6 +33,7 @@ struct scone_fgram_model {
   int64_t cap_rows = 0;                  // workspace rows (tokens)
   int32_t* off = nullptr;                // [batch + 1] token offsets
   int* status = nullptr;                 // sticky device error
+  int* h_words = nullptr;                // pinned [2]: a batch's token count, the status
   uint16_t *X = nullptr, *Xn = nullptr, *QKV = nullptr, *Act = nullptr;
 };
 
@@ -362,7 +363,8 @@ extern "C" int scone_fgram_model_create(int32_t d, int32_t n_heads, int32_t ffw,
   m->batch = batch > 0 ? batch : 16384;
   if (cudaMalloc(&m->off, (size_t)(m->batch + 1) * sizeof(int32_t)) != cudaSuccess ||
       cudaMalloc(&m->status, sizeof(int)) != cudaSuccess ||
-      cudaMemset(m->status, 0, sizeof(int)) != cudaSuccess) {
+      cudaMemset(m->status, 0, sizeof(int)) != cudaSuccess ||
+      cudaHostAlloc(&m->h_words, 2 * sizeof(int), cudaHostAllocDefault) != cudaSuccess) {
     cudaGetLastError();
     scone_fgram_model_destroy(m);
     return SCONE_ERR_NOMEM;
@@ -378,6 +380,7 @@ extern "C" int scone_fgram_model_destroy(scone_fgram_model* m) {
   for (void* p : {(void*)m->off, (void*)m->status, (void*)m->X, (void*)m->Xn, (void*)m->QKV,
                   (void*)m->Act})
     if (p) cudaFree(p);
+  if (m->h_words) cudaFreeHost(m->h_words);
   delete m;
   return SCONE_OK;
 }
@@ -399,12 +402,12 @@ extern "C" int scone_fgram_precompute(scone_fgram_model* m, const int32_t* fgram
   for (int64_t f0 = 0; f0 < n; f0 += m->batch) {
     const int64_t nb = n - f0 < m->batch ? n - f0 : m->batch;
     offsets_kernel<<<1, 1024, 0, s>>>(fgram_len + f0, nb, K, m->off, m->status);
-    int32_t rows = 0;
     if (cudaGetLastError() != cudaSuccess ||
-        cudaMemcpyAsync(&rows, m->off + nb, sizeof(rows), cudaMemcpyDeviceToHost, s) !=
+        cudaMemcpyAsync(m->h_words, m->off + nb, sizeof(int32_t), cudaMemcpyDeviceToHost, s) !=
             cudaSuccess ||
         cudaStreamSynchronize(s) != cudaSuccess)
       return SCONE_ERR_CUDA;
+    const int32_t rows = m->h_words[0];
     if (!ensure_rows(m, rows)) return SCONE_ERR_NOMEM;
     const unsigned gw = (unsigned)((nb + kRowsPerBlock - 1) / kRowsPerBlock);
     gather_rows_kernel<<<gw, 256, 0, s>>>(fgram_tok + f0 * K, fgram_len + f0, m->off, nb, K, T,
@@ -435,10 +438,10 @@ extern "C" int scone_fgram_precompute(scone_fgram_model* m, const int32_t* fgram
     if (!ln(d, m->X, F + f0 * d, nb, m->off, s)) return SCONE_ERR_UNSUPPORTED;
     if (cudaGetLastError() != cudaSuccess) return SCONE_ERR_CUDA;
   }
-  int st = 0;
-  if (cudaMemcpyAsync(&st, m->status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+  if (cudaMemcpyAsync(m->h_words + 1, m->status, sizeof(int), cudaMemcpyDeviceToHost, s) !=
+          cudaSuccess ||
       cudaMemsetAsync(m->status, 0, sizeof(int), s) != cudaSuccess ||
       cudaStreamSynchronize(s) != cudaSuccess)
     return SCONE_ERR_CUDA;
-  return st;
+  return m->h_words[1];
 }

@@ -201,6 +201,7 @@ struct scone_rowstore {
   int64_t cap = 0;                     // positions
   int32_t *d_miss_pos = nullptr, *d_miss_row = nullptr, *d_miss_src = nullptr;
   int* d_miss_count = nullptr;
+  int* h_miss_count = nullptr;         // pinned
   int32_t *h_miss_row = nullptr, *h_miss_src = nullptr;
   int64_t stage_cap = 0;               // staged rows
   uint8_t* h_stage = nullptr;          // pinned, 4096-aligned
@@ -219,9 +220,10 @@ void free_call_buffers(scone_rowstore* st) {
                   (void*)st->d_miss_count, (void*)st->d_stage, (void*)st->d_fill,
                   (void*)st->d_fill_src})
     if (p) cudaFree(p);
-  for (void* p : {(void*)st->h_miss_row, (void*)st->h_miss_src,
+  for (void* p : {(void*)st->h_miss_count, (void*)st->h_miss_row, (void*)st->h_miss_src,
                   (void*)st->h_stage, (void*)st->h_fill, (void*)st->h_fill_src})
     if (p) cudaFreeHost(p);
+  st->h_miss_count = nullptr;
   st->d_fill_src = st->h_fill_src = nullptr;
   st->d_miss_pos = st->d_miss_row = st->d_miss_src = nullptr;
   st->d_miss_count = nullptr;
@@ -245,6 +247,7 @@ bool grow(scone_rowstore* st, int64_t n) {
       cudaMalloc(&st->d_stage, c * rb) != cudaSuccess ||
       cudaMalloc(&st->d_fill, 2 * c * sizeof(int64_t)) != cudaSuccess ||
       cudaMalloc(&st->d_fill_src, c * 4) != cudaSuccess ||
+      cudaHostAlloc(&st->h_miss_count, sizeof(int), cudaHostAllocDefault) != cudaSuccess ||
       cudaHostAlloc(&st->h_miss_row, c * 4, cudaHostAllocDefault) != cudaSuccess ||
       cudaHostAlloc(&st->h_miss_src, c * 4, cudaHostAllocDefault) != cudaSuccess ||
       cudaHostAlloc(&st->h_stage, c * rb, cudaHostAllocDefault) != cudaSuccess ||
@@ -357,17 +360,17 @@ extern "C" int scone_rowstore_gather(scone_rowstore* st, const scone_table* tb,
   const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)lookup_kernel,
                                                           kStoreThreads, 0);
   const int grid = (int)(blocks_needed < cap ? blocks_needed : cap);
-  int n_miss = 0;
   if (cudaMemsetAsync(st->d_miss_count, 0, sizeof(int), s) != cudaSuccess) return SCONE_ERR_CUDA;
   lookup_kernel<<<grid, kStoreThreads, 0, s>>>(t, tok, row, n, st->cache, st->tag,
                                                st->cache_rows, st->n_rows,
                                                reinterpret_cast<uint8_t*>(out), st->d_miss_pos,
                                                st->d_miss_row, st->d_miss_count, width);
   if (cudaGetLastError() != cudaSuccess ||
-      cudaMemcpyAsync(&n_miss, st->d_miss_count, sizeof(int), cudaMemcpyDeviceToHost, s) !=
-          cudaSuccess ||
+      cudaMemcpyAsync(st->h_miss_count, st->d_miss_count, sizeof(int), cudaMemcpyDeviceToHost,
+                      s) != cudaSuccess ||
       cudaStreamSynchronize(s) != cudaSuccess)
     return SCONE_ERR_CUDA;
+  const int n_miss = *st->h_miss_count;
   st->stats.positions += n;
   st->stats.misses += n_miss;
   if (n_miss == 0) return SCONE_OK;
