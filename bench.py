@@ -547,21 +547,26 @@ def bench_decode(args, world, rank, local):
     ms_step = statistics.mean(per_replay) / steps
 
     # end to end through the public API, one step at a time: the step's new
-    # tokens copied from pinned host memory, scone_decode_step, scone_status
-    # (sync + status word read)
+    # tokens from pinned host memory (read by the kernel; "staged": copied to
+    # the device first), scone_decode_step, scone_status (sync + status word)
     host_new = torch.from_numpy(new).pin_memory()
     tok_d = torch.empty(S, dtype=torch.int32, device=dev)
     e2e_n = min(steps, 64)
-    e2e_t = []
-    for k in range(e2e_n + 3):
-        torch.cuda.synchronize()
-        t1 = time.perf_counter()
-        tok_d.copy_(host_new[k % steps], non_blocking=True)
-        scone.scone_decode_step(st, tok_d, out)
-        scone.scone_status(table)
-        if k >= 3:
-            e2e_t.append(time.perf_counter() - t1)
-    e2e_ms = max_over_ranks(1e3 * statistics.mean(e2e_t), world)
+    e2e_ms = {}
+    for staged in (False, True):
+        e2e_t = []
+        for k in range(e2e_n + 3):
+            torch.cuda.synchronize()
+            t1 = time.perf_counter()
+            if staged:
+                tok_d.copy_(host_new[k % steps], non_blocking=True)
+                scone.scone_decode_step(st, tok_d, out)
+            else:
+                scone.scone_decode_step(st, host_new[k % steps], out)
+            scone.scone_status(table)
+            if k >= 3:
+                e2e_t.append(time.perf_counter() - t1)
+        e2e_ms[staged] = max_over_ranks(1e3 * statistics.mean(e2e_t), world)
     host_bytes_step = matched / steps * 2 * w.d
     hbm_bytes_step = (S * (4 + 32 * (w.K - 1)) + (S - matched / steps) * 2 * w.d + S * 2 * w.d)
     achieved = host_bytes_step / (ms_step * 1e-3) / 1e9
@@ -601,11 +606,13 @@ def bench_decode(args, world, rank, local):
             "hbm_bytes_per_step": hbm_bytes_step,
             "kernel": "decode_kernel (one warp per sequence)",
         },
-        "e2e": {"value": world * S / (e2e_ms * 1e-3), "unit": "tokens/s",
+        "e2e": {"value": world * S / (e2e_ms[False] * 1e-3), "unit": "tokens/s",
                 "h2d_bytes_per_step": 4 * S, "d2h_bytes_per_step": 4,
-                "what": "each step: new tokens from pinned host memory, scone_decode_step, "
-                        "scone_status (sync + status word read); no graph, one step at a "
-                        "time as a serving loop issues them"},
+                "what": "each step: new tokens read by the decode kernel from pinned host "
+                        "memory, scone_decode_step, scone_status (sync + status word read); "
+                        "no graph, one step at a time as a serving loop issues them",
+                "staged": {"value": world * S / (e2e_ms[True] * 1e-3), "unit": "tokens/s",
+                           "what": "the same with a cudaMemcpyAsync of the tokens first"}},
         "gpu_launches": replays * steps,
         "clocks": clocks.summary(),
         "match_len_hist": {str(i): int(c) for i, c in enumerate(hist_counts)},

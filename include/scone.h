@@ -441,12 +441,14 @@ int scone_decode_create(const scone_table* table, int32_t S, const int32_t* hist
                         const int32_t* hist_len, scone_decode** out);
 
 /*
- * scone_decode_step: appends new_tok[s] (device int32 [S]) to sequence s,
- * embeds it by Algorithm 1 over the sequence so far, and writes
- * out device [S * d]; row device int32 [S] and len device uint8 [S] may be
- * NULL. out may be NULL when row is given: the step then only selects (for
- * rows gathered from a row store, scone_rowstore_gather). Async; steps on
- * one state must be ordered on one stream.
+ * scone_decode_step: appends new_tok[s] (int32 [S], device memory or
+ * page-locked host memory mapped for the device, which the kernel then reads
+ * over the host link) to sequence s, embeds it by Algorithm 1 over the
+ * sequence so far, and writes out device [S * d]; row device int32 [S] and
+ * len device uint8 [S] may be NULL. out may be NULL when row is given: the
+ * step then only selects (for rows gathered from a row store,
+ * scone_rowstore_gather). Async; steps on one state must be ordered on one
+ * stream, and host tokens must stay unchanged until the step is done.
  */
 int scone_decode_step(scone_decode* state, const int32_t* new_tok, scone_bf16* out, int32_t* row,
                       uint8_t* len, void* stream);

@@ -488,8 +488,11 @@ def scone_decode_create(table: Table, hist: np.ndarray, hist_len: np.ndarray) ->
 
 
 def scone_decode_step(state: DecodeState, new_tok, out, row=None, len=None, stream=None) -> None:
-    _check(load_library().scone_decode_step(state.handle, _ptr(new_tok), _ptr(out), _ptr(row),
-                                            _ptr(len), _stream(stream)), "scone_decode_step")
+    """One decode step; new_tok [S] int32, a CUDA tensor or a pinned CPU tensor
+    (read by the kernel over the host link)."""
+    _check(load_library().scone_decode_step(state.handle, _tok_ptr(new_tok), _ptr(out),
+                                            _ptr(row), _ptr(len), _stream(stream)),
+           "scone_decode_step")
 
 
 def scone_decode_get_history(state: DecodeState):

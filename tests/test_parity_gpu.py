@@ -289,6 +289,31 @@ def test_decode_steps_match_oracle(K, S, vocab):
     assert set(np.unique(o_len)) >= {0, 1, 2}
 
 
+def test_decode_pinned_host_tokens():
+    """Decode steps reading their new tokens from pinned host memory give the
+    oracle's rows, as with device tokens (the zero-copy input of the serving
+    loop)."""
+    K, S, steps, d = 3, 64, 8, 96
+    ft, fl, hist, hl, new, F, T = _decode_case(K, S, steps, 2000, d, seed=21)
+    o = oracle.Oracle(ft, fl, K, 2000)
+    o_out, o_row, o_len, _ = o.decode(hist, hl, new, F, T)
+    table = scone.scone_table_build(ft, fl, K, 2000, d, dev_rows(F), dev_rows(T))
+    st = scone.scone_decode_create(table, hist, hl)
+    host_new = torch.from_numpy(np.ascontiguousarray(new)).pin_memory()
+    out = torch.empty((S, d), dtype=torch.int16, device=DEV)
+    row = torch.empty(S, dtype=torch.int32, device=DEV)
+    for k in range(steps):
+        scone.scone_decode_step(st, host_new[k], out, row)
+        torch.cuda.synchronize()
+        assert np.array_equal(row.cpu().numpy(), o_row[k].astype(np.int32)), k
+        assert np.array_equal(out.cpu().numpy().view(np.uint16), o_out[k]), k
+    assert scone.scone_status(table) == 0
+    with pytest.raises(ValueError):
+        scone.scone_decode_step(st, torch.from_numpy(np.ascontiguousarray(new[0])), out)
+    st.close()
+    table.close()
+
+
 def test_decode_equals_prefill_on_device():
     K, S, steps, vocab, d = 3, 64, 20, 2000, 64
     ft, fl, hist, hl, new, F, T = _decode_case(K, S, steps, vocab, d, seed=11)
