@@ -1,0 +1,42 @@
+"""The bench's reference arm and its JSON line (CPU): `bench.py --impl
+reference` times the oracle on the measured arm's workload config, metric and
+unit and prints one line with the keys the measurement contract asks for."""
+
+import json
+import os
+import subprocess
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def run_bench(*args):
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), *args],
+                         cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [l for l in out.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, out.stdout[-2000:]
+    return json.loads(lines[0])
+
+
+def test_reference_line_keys():
+    import bench
+
+    d = run_bench("--impl", "reference", "--steps", "2", "--warmup", "1")
+    assert d["impl"] == "reference"
+    assert d["metric"] == bench.METRIC and d["unit"] == "tokens/s"
+    assert d["higher_is_better"] is True and d["value"] > 0
+    assert d["warmup"] >= 3 and d["steps"] == 2
+    import synth
+
+    w = synth.WORKLOADS["prefill_1b"]
+    assert d["config"]["workload"] == bench.prefill_config(w, 1)["workload"]
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] == d["value"]
+    assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
+
+
+def test_reference_line_other_workload_is_explicit():
+    d = run_bench("--impl", "reference", "--workload", "discover", "--steps", "1")
+    assert d["impl"] == "reference" and "unavailable" in d
