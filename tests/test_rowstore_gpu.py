@@ -142,3 +142,31 @@ def test_direct_io_rows(tmp_path):
     assert store.stats()["rows_read"] > 0
     store.close()
     table.close()
+
+
+def test_long_keys_and_k8(tmp_path):
+    """A table with 32-byte slots (K = 8 over a 2^20-token vocabulary): rows
+    selected by the long-key matcher and served by the store equal the
+    oracle's bytes."""
+    w = synth.Workload("rowstore_k8", 88, 1 << 20, 1.05, 3, 600,
+                       tuple((n, 1200) for n in range(2, 9)), 8, 64, inject_p=0.05,
+                       n_phrases=256, phrase_len=(8, 10))
+    c = SmallCase(w)
+    path = str(tmp_path / "F8.bin")
+    c.F.tofile(path)
+    table = scone.scone_table_build(c.fg_tok, c.fg_len, w.K, w.vocab, w.d, dev_rows(c.F[:1]),
+                                    dev_rows(c.T))
+    assert table.info()["slot_bytes"] == 32
+    store = scone.RowStore(path, c.F.shape[0], w.d, cache_rows=61, threads=2)
+    t = torch.from_numpy(c.tok).to(DEV)
+    row = torch.empty(t.numel(), dtype=torch.int32, device=DEV)
+    out = torch.empty((t.numel(), w.d), dtype=torch.int16, device=DEV)
+    scone.scone_match(table, t, row)
+    scone.scone_rowstore_gather(store, table, t.reshape(-1), row, out)
+    scone.scone_status(table)
+    exp_out, exp_row, exp_len, _ = c.expected()
+    assert np.array_equal(row.cpu().numpy(), exp_row.reshape(-1).astype(np.int32))
+    assert np.array_equal(out.cpu().numpy().view(np.uint16), exp_out.reshape(-1, w.d))
+    assert (exp_len == 8).any()
+    store.close()
+    table.close()
