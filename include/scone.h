@@ -213,9 +213,10 @@ int scone_match(const scone_table* table, const int32_t* tok, int32_t B, int32_t
  * r gets row r). If fewer than S n-grams are eligible, all are returned.
  *
  *  ws           a workspace from scone_discover_create, or NULL. The call's
- *               device buffers are taken from it and stay allocated there
- *               (grown as needed, never shrunk) until scone_discover_destroy,
- *               so repeated calls allocate nothing; with NULL they are
+ *               device buffers (and a small pinned host area for its reads of
+ *               counters) are taken from it and stay allocated there (grown as
+ *               needed, never shrunk) until scone_discover_destroy, so
+ *               repeated calls allocate nothing; with NULL they are
  *               allocated and freed inside the call.
  *  tok          int32 [B * L], device-accessible (device memory, or host
  *               memory from scone_host_alloc read over the host link);
@@ -237,11 +238,12 @@ int scone_match(const scone_table* table, const int32_t* tok, int32_t B, int32_t
  * window records and the names of the previous scan), a counting table of
  * 64 bytes per distinct n-gram of the largest scan (see
  * scone_discover_set_table_slack), and the lists of eligible n-grams
- * (4 (n + 1) bytes each). Errors: SCONE_ERR_INVALID_ARG
- * (K outside [2, 8], min_count < 1,
- * S < 0, null pointers), SCONE_ERR_UNSUPPORTED (B * L > 2^30),
+ * (4 (n + 1) bytes each). Errors: SCONE_ERR_INVALID_ARG (K outside [2, 8],
+ * min_count < 1, S < 0, null pointers), SCONE_ERR_UNSUPPORTED (B * L > 2^30),
  * SCONE_ERR_TOKEN_RANGE (a token outside [0, vocab); nothing is written),
- * SCONE_ERR_NOMEM, SCONE_ERR_CUDA.
+ * SCONE_ERR_TABLE_FULL (a worst-case counting table filled up, which only a
+ * corpus built to collide in the hash can cause), SCONE_ERR_NOMEM,
+ * SCONE_ERR_CUDA.
  */
 typedef struct scone_discover_stats {
   int64_t candidates[9];      /* windows counted in scan n (after pruning for n >= 3) */
