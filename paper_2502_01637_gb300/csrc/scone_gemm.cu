@@ -41,7 +41,12 @@ constexpr int kBM = 128, kBN = 256, kBK = 64;
 constexpr int kStages = 4;
 constexpr int kEpiWarps = 4;
 constexpr int kGemmThreads = 32 * (2 + kEpiWarps);   // loader, MMA issuer, 4 epilogue warps
-constexpr int kGroupM = 8;                            // row tiles per group of the tile order
+// Rows per group of the tile order (kGroupRows / tile height row tiles at a
+// time). On M = N = 16384, K = 2048, groups of 8, 16, 32 and 64 row tiles
+// gave the SM-pair kernel (256-row tiles) 1704, 1714, 1722 and 1681-1688
+// TFLOP/s, and the one-SM kernel (128-row tiles) 1607, 1668, 1697 and 1741:
+// both are best near 8192 rows.
+constexpr int kGroupRows = 8192;
 constexpr uint32_t kStageA = kBM * kBK * 2;   // 16 KB
 constexpr uint32_t kStageB = kBN * kBK * 2;   // 32 KB
 constexpr uint32_t kStageBytes = kStageA + kStageB;
@@ -121,14 +126,15 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// Tile t of the grouped order: kGroupM row tiles at a time sweep all column
-// tiles, so the CTAs running at once share a few A tiles and a few B tiles in
-// L2 instead of each streaming its own A.
+// Tile t of the grouped order: G row tiles at a time sweep all column tiles,
+// so the CTAs running at once share a few A tiles and a few B tiles in L2
+// instead of each streaming its own A.
+template <int G>
 __device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int* m_tile,
                                             int* n_tile) {
-  const int per_group = kGroupM * num_n;
-  const int first_m = (t / per_group) * kGroupM;
-  const int gm = num_m - first_m < kGroupM ? num_m - first_m : kGroupM;
+  const int per_group = G * num_n;
+  const int first_m = (t / per_group) * G;
+  const int gm = num_m - first_m < G ? num_m - first_m : G;
   const int local = t % per_group;
   *m_tile = first_m + local % gm;
   *n_tile = local / gm;
@@ -235,7 +241,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       int it = 0;
       for (int t = blockIdx.x; t < tiles && !*vfailed; t += gridDim.x) {
         int mt, nt;
-        tile_coords(t, num_m, num_n, &mt, &nt);
+        tile_coords<kGroupRows / kBM>(t, num_m, num_n, &mt, &nt);
         for (int kt = 0; kt < kt_n; ++kt, ++it) {
           const int s = it % kStages;
           if (it >= kStages && !mbar_wait(saddr(&empty[s]), ((it / kStages) - 1) & 1)) {
@@ -300,7 +306,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       int mt, nt;
-      tile_coords(t, num_m, num_n, &mt, &nt);
+      tile_coords<kGroupRows / kBM>(t, num_m, num_n, &mt, &nt);
       const int row = mt * kBM + q * 32 + lane;
       const uint32_t t_row = tmem + acc * kBN + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
@@ -423,7 +429,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       int it = 0;
       for (int t = pair; t < tiles && !*vfailed; t += pairs) {
         int mt, nt;
-        tile_coords(t, num_m, num_n, &mt, &nt);
+        tile_coords<kGroupRows / 256>(t, num_m, num_n, &mt, &nt);
         for (int kt = 0; kt < kt_n; ++kt, ++it) {
           const int st = it % kPStages;
           if (it >= kPStages && !mbar_wait(saddr(&empty[st]), ((it / kPStages) - 1) & 1)) {
@@ -488,7 +494,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       }
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       int mt, nt;
-      tile_coords(t, num_m, num_n, &mt, &nt);
+      tile_coords<kGroupRows / 256>(t, num_m, num_n, &mt, &nt);
       const int row = mt * 256 + (int)rank * 128 + q * 32 + lane;
       const uint32_t t_row = tmem + acc * kBN + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
