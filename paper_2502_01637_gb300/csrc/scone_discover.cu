@@ -13,13 +13,17 @@
 //
 // Per scan, over the flattened B x L corpus (positions i, window ending at i):
 //   1a. bin_kernel: every window's key; windows whose key sits in their
-//      block's shared-memory cache of hot keys are counted there (the cache
-//      is added to the global table {key, count, ~first} once per block).
-//      Every other window becomes a record, grouped per chunk of kChunk
-//      windows by the region of the table its key hashes to.
+//      block's shared-memory cache of hot keys are counted there (each
+//      block's cache goes to a hot list). Every other window becomes a
+//      record, grouped per chunk of kChunk windows by the region of the table
+//      its key hashes to. Every key also enters a HyperLogLog sketch.
+//   The host sizes the counting table {key, count, ~first} from the sketch's
+//   estimate of the distinct keys and zeroes it; hotflush_kernel adds the hot
+//   lists to it.
 //   1b. bincount_kernel: the records, region by region, add themselves to the
-//      table with atomics. All warps work on one or two regions at a time, so
-//      the updates hit L2 instead of random DRAM sectors.
+//      table with atomics. All blocks work on one or two regions at a time, so
+//      the updates hit L2 instead of random DRAM sectors. (If the table fills
+//      up, it is rebuilt at the worst-case size and 1b to 2b run again.)
 //   2a. flagbin_kernel: the records, region by region again, look their keys
 //      up in the finished table (L2 hits). A window is the first occurrence
 //      of a frequent n-gram when its start equals the slot's first occurrence
