@@ -4,8 +4,9 @@
 // tensor memory.
 //
 // Tiles of 128 x 256, persistent (one CTA per SM walks its share of the
-// tiles in a grouped order: 8 row tiles at a time sweep every column tile, so
-// the tiles in flight share their A and B slices in L2), warp-specialized:
+// tiles in a grouped order: 8192 rows of row tiles at a time sweep every column
+// tile, so the tiles in flight share their A and B slices in L2),
+// warp-specialized:
 //   * warp 0 streams K-slices of 64 (A: 128 x 64, B: 256 x 64, 48 KB) into a
 //     ring of kStages shared-memory stages with TMA (cp.async.bulk.tensor,
 //     128-byte swizzle), each stage completed on an mbarrier by byte count;
