@@ -120,21 +120,39 @@ int scone_table_destroy(scone_table* table);
  * location stay those of the original build. The build kernels' scratch (a
  * device copy of the list plus three flags) lives in one file-scope device
  * array of SCONE_REBUILD_SCRATCH_BYTES, which every GPU that loads the library
- * holds until the process exits; a list needs 64 + n_fgrams * (4 K + 1)
- * bytes of it, rounded up to 256, and a larger list is rejected with
- * SCONE_ERR_INVALID_ARG before any device work. The first call on a device
- * looks the array's address up (once per device); make that first call
- * before any stream capture begins.
+ * holds until the process exits. A list of n f-grams needs
+ *     256 + round256(n) + round256(4 * K * n)
+ * bytes of it (round256 rounds up to a multiple of 256; a list of
+ * SCONE_REBUILD_MAX_FGRAMS(K) f-grams always fits: 1,290,496 at K = 3), and a
+ * larger list is rejected with SCONE_ERR_INVALID_ARG before any device work.
+ * The first call on a device looks the array's address up (once per device);
+ * make that first call before any stream capture begins.
  *
  * All calls share that array and it keeps the last call's contents; the
  * flags are cleared by each call. Calls whose device work overlaps (other
  * streams, other threads) race on it, and so do lookups on this table from
  * other streams during the call. Synchronous: it synchronizes `stream`.
+ *
+ * Launches take the table's state (F, row count, hash seed) by value when
+ * they are enqueued. Work enqueued or captured before this call (a CUDA graph
+ * of embed or decode launches, in particular) keeps the old state and would
+ * read the new slots against the old F: capture such graphs again after the
+ * call returns.
+ *
  * Errors: INVALID_ARG (table NULL, list too large for the table or the
- * scratch, bad list or F), DUPLICATE_FGRAM or TABLE_FULL (the table is then
- * left empty: every position falls back to T), CUDA.
+ * scratch, bad list or F; the table is unchanged), DUPLICATE_FGRAM or
+ * TABLE_FULL (the table is then left empty: every position falls back to T),
+ * CUDA (one attempt is made to leave the table empty; if scone_table_get_info
+ * then still reports the old n_fgrams the table is inconsistent and must be
+ * destroyed).
  */
 #define SCONE_REBUILD_SCRATCH_BYTES (16u << 20)
+/* A list size that always fits the scratch: since each rounding adds at most
+ * 255 bytes, n = floor((SCONE_REBUILD_SCRATCH_BYTES - 768) / (4*K + 1)) satisfies
+ * 256 + round256(n) + round256(4*K*n) <= SCONE_REBUILD_SCRATCH_BYTES, and the
+ * exact limit exceeds it by fewer than 510 / (4*K + 1) + 1 f-grams. */
+#define SCONE_REBUILD_MAX_FGRAMS(K) \
+  ((int64_t)(((int64_t)SCONE_REBUILD_SCRATCH_BYTES - 768) / (4 * (int64_t)(K) + 1)))
 int scone_table_rebuild_noalloc(scone_table* table, const int32_t* fgram_tok,
                                 const uint8_t* fgram_len, int64_t n_fgrams, const scone_bf16* F,
                                 void* stream);

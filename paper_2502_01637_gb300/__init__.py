@@ -248,6 +248,14 @@ def scone_table_rebuild_noalloc(table: Table, fgram_tok: np.ndarray, fgram_len: 
     list must fit the table (at most 0.85 of its slots) and the library's
     fixed device scratch (SCONE_REBUILD_SCRATCH_BYTES); calls that overlap on
     the GPU race on that scratch. Synchronizes the stream.
+
+    Work captured before the call (a CUDA graph of embed or decode launches)
+    still holds the old list's F, row count and hash seed: capture it again
+    after the call.
+
+    The table keeps referencing the F it reads: the new F after a successful
+    call with a non-empty list, the old F after a refused call (the table is
+    unchanged then), and both after a CUDA error.
     """
     K = table.info()["K"]
     ft = np.ascontiguousarray(fgram_tok, dtype=np.int32).reshape(-1)
@@ -258,7 +266,11 @@ def scone_table_rebuild_noalloc(table: Table, fgram_tok: np.ndarray, fgram_len: 
     rc = load_library().scone_table_rebuild_noalloc(table.handle, _ptr(ft) if n else None,
                                                     _ptr(fl) if n else None, n, _ptr(F),
                                                     _stream(stream))
-    table._keep = (F, table._keep[1] if table._keep else None)
+    old_F, T = table._keep if table._keep else (None, None)
+    if rc == SCONE_OK and n > 0:
+        table._keep = (F, T)
+    elif rc == SCONE_ERR_CUDA:
+        table._keep = ((old_F, F), T)
     _check(rc, "scone_table_rebuild_noalloc")
 
 

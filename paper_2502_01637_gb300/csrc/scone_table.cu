@@ -676,6 +676,18 @@ extern "C" int scone_table_rebuild_noalloc(scone_table* t, const int32_t* fgram_
   // flags (which must start at zero) before every attempt
   rc = build_slots(t, d_tok, d_len, d_flags, n_fgrams, s, &flags);
   if (rc == SCONE_ERR_CUDA) {
+    // the slot array may hold part of the new list while view.F, n_fgrams and
+    // the hash seed still describe the old one: one best-effort attempt to
+    // leave the table empty (every position falls back to T), as the other
+    // failure paths do. If even that fails the table must be destroyed.
+    cudaGetLastError();
+    if (cudaMemsetAsync(t->slots, 0xFF, (size_t)t->info.table_bytes, s) == cudaSuccess &&
+        cudaStreamSynchronize(s) == cudaSuccess) {
+      t->view.n_fgrams = 0;
+      t->info.n_fgrams = 0;
+      t->info.max_insert_probe = 0;
+      t->info.F_bytes = 0;
+    }
     cudaGetLastError();
     return rc;
   }

@@ -13,12 +13,11 @@ This file is collected last so that a run stopping at the first failure has
 already run every other test; it also passes when run on its own.
 """
 
-import ctypes
-
 import numpy as np
 import pytest
 import torch
 
+import oracle
 import synth
 import paper_2502_01637_gb300 as scone
 from gpu_cases import DEV, dev_rows, run_embed
@@ -58,21 +57,163 @@ def _same_as_fresh_build(table, fg_tok, fg_len, F, T, tok):
     return a
 
 
+def _same_as_oracle(got, fg_tok, fg_len, F_host, T_host, tok, K=BASE.K, vocab=BASE.vocab):
+    """Element-wise equality of (out, row, len) with the oracle of Algorithm 1."""
+    o_out, o_row, o_len, rc = oracle.Oracle(fg_tok, fg_len, K, vocab).embed(tok, F_host, T_host)
+    assert rc == oracle.OK
+    out, row, ln = got
+    assert np.array_equal(row, o_row.reshape(-1).astype(np.int32))
+    assert np.array_equal(ln, o_len.reshape(-1))
+    assert np.array_equal(out, o_out.reshape(out.shape))
+
+
+def _no_alloc_call(table, fg_tok, fg_len, F):
+    """One call with the device's free memory and torch's allocation counters
+    read on both sides: neither may move."""
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    n0 = torch.cuda.memory_stats().get("allocation.all.allocated", 0)
+    rc = _rebuild_via_c_abi(table, fg_tok, fg_len, F)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    n1 = torch.cuda.memory_stats().get("allocation.all.allocated", 0)
+    assert free1 == free0, f"device free memory moved by {free0 - free1} bytes"
+    assert n1 == n0
+    return rc
+
+
 def test_rebuild_noalloc_matches_build_on_two_calls_in_a_row():
     fg1_tok, fg1_len, _ = synth.fgram_set(BASE)
     fg2_tok, fg2_len, _ = synth.fgram_set(OTHER)
-    T = dev_rows(synth.rows_cpu(synth.T_seed(BASE), BASE.d, np.arange(BASE.vocab)))
-    F1 = _rows(BASE, BASE.n_fgrams)
-    F2 = _rows(OTHER, OTHER.n_fgrams)
+    T_host = synth.rows_cpu(synth.T_seed(BASE), BASE.d, np.arange(BASE.vocab))
+    F1_host = synth.rows_cpu(synth.F_seed(BASE), BASE.d, np.arange(BASE.n_fgrams))
+    F2_host = synth.rows_cpu(synth.F_seed(OTHER), OTHER.d, np.arange(OTHER.n_fgrams))
+    T, F1, F2 = dev_rows(T_host), dev_rows(F1_host), dev_rows(F2_host)
     tok = synth.query_tokens(BASE)
     table = scone.scone_table_build(fg1_tok, fg1_len, BASE.K, BASE.vocab, BASE.d, F1, T)
     assert OTHER.n_fgrams <= 0.85 * table.info()["n_slots"]
     # two calls in a row, each compared with a table built the ordinary way
-    for fg_tok, fg_len, F in ((fg2_tok, fg2_len, F2), (fg1_tok, fg1_len, F1)):
-        assert _rebuild_via_c_abi(table, fg_tok, fg_len, F) == scone.SCONE_OK
-        out, row, ln = _same_as_fresh_build(table, fg_tok, fg_len, F, T, tok)
+    # and with the oracle; the second call must not move the device's free
+    # memory (the first may load the library's module on a fresh device)
+    calls = ((fg2_tok, fg2_len, F2, F2_host), (fg1_tok, fg1_len, F1, F1_host))
+    for k, (fg_tok, fg_len, F, F_host) in enumerate(calls):
+        if k == 0:
+            assert _rebuild_via_c_abi(table, fg_tok, fg_len, F) == scone.SCONE_OK
+        else:
+            assert _no_alloc_call(table, fg_tok, fg_len, F) == scone.SCONE_OK
+        got = _same_as_fresh_build(table, fg_tok, fg_len, F, T, tok)
+        _same_as_oracle(got, fg_tok, fg_len, F_host, T_host, tok)
         assert table.info()["n_fgrams"] == fg_len.shape[0]
-        assert (ln >= 2).any() and (ln == 1).any()
+        assert (got[2] >= 2).any() and (got[2] == 1).any()
+    assert scone.scone_status(table) == scone.SCONE_OK
+    table.close()
+
+
+def test_rebuild_noalloc_host_mapped_F():
+    """F in pinned, device-mapped host memory (the offloaded tier): the new
+    list's rows are read through the mapped address of the new buffer."""
+    fg1_tok, fg1_len, _ = synth.fgram_set(BASE)
+    fg2_tok, fg2_len, _ = synth.fgram_set(OTHER)
+    T_host = synth.rows_cpu(synth.T_seed(BASE), BASE.d, np.arange(BASE.vocab))
+    T = dev_rows(T_host)
+    tok = synth.query_tokens(BASE)
+    bufs, hosts = [], []
+    for w in (BASE, OTHER):
+        h = synth.rows_cpu(synth.F_seed(w), w.d, np.arange(w.n_fgrams))
+        b = scone.scone_host_alloc(h.nbytes)
+        b.numpy(np.uint16)[:h.size] = h.reshape(-1)
+        bufs.append(b)
+        hosts.append(h)
+    table = scone.scone_table_build(fg1_tok, fg1_len, BASE.K, BASE.vocab, BASE.d, bufs[0].ptr,
+                                    T, F_location=scone.SCONE_ROWS_HOST_MAPPED)
+    calls = ((fg2_tok, fg2_len, bufs[1], hosts[1]), (fg1_tok, fg1_len, bufs[0], hosts[0]))
+    for fg_tok, fg_len, b, h in calls:
+        lib = scone.load_library()
+        rc = lib.scone_table_rebuild_noalloc(
+            table.handle, np.ascontiguousarray(fg_tok, np.int32).ctypes.data,
+            np.ascontiguousarray(fg_len, np.uint8).ctypes.data, fg_len.shape[0], b.ptr,
+            torch.cuda.current_stream().cuda_stream)
+        assert rc == scone.SCONE_OK
+        assert table.info()["F_location"] == scone.SCONE_ROWS_HOST_MAPPED
+        _same_as_oracle(run_embed(table, tok, BASE.d), fg_tok, fg_len, h, T_host, tok)
+    assert scone.scone_status(table) == scone.SCONE_OK
+    table.close()
+    for b in bufs:
+        b.free()
+
+
+def test_wrapper_keeps_the_old_F_after_a_refused_call():
+    """A refused call leaves the table on its old list and old F; the Python
+    wrapper must keep that F alive even when the caller drops it."""
+    fg_tok, fg_len, _ = synth.fgram_set(BASE)
+    T_host = synth.rows_cpu(synth.T_seed(BASE), BASE.d, np.arange(BASE.vocab))
+    F_host = synth.rows_cpu(synth.F_seed(BASE), BASE.d, np.arange(BASE.n_fgrams))
+    T, F = dev_rows(T_host), dev_rows(F_host)
+    tok = synth.query_tokens(BASE)
+    table = scone.scone_table_build(fg_tok, fg_len, BASE.K, BASE.vocab, BASE.d, F, T)
+    n_slots = table.info()["n_slots"]
+    big = int(0.85 * n_slots) + 1
+    F_big = torch.zeros((big, BASE.d), dtype=torch.int16, device=DEV)
+    with pytest.raises(scone.SconeError) as e:
+        scone.scone_table_rebuild_noalloc(table, np.zeros((big, BASE.K), np.int32),
+                                          np.full(big, 2, np.uint8), F_big)
+    assert e.value.code == scone.SCONE_ERR_INVALID_ARG
+    # drop the caller's references; a same-sized allocation would take the old
+    # F's block from torch's cache if the wrapper had released it
+    nbytes = F.numel()
+    del F, F_big
+    junk = torch.full((nbytes,), -1, dtype=torch.int16, device=DEV)
+    _same_as_oracle(run_embed(table, tok, BASE.d), fg_tok, fg_len, F_host, T_host, tok)
+    del junk
+    table.close()
+
+
+def test_graphs_captured_again_after_a_rebuild():
+    """A graph captured before the call keeps the old list's state; captured
+    again after it, it gives the new list's result, bit for bit."""
+    fg1_tok, fg1_len, _ = synth.fgram_set(BASE)
+    fg2_tok, fg2_len, _ = synth.fgram_set(OTHER)
+    T_host = synth.rows_cpu(synth.T_seed(BASE), BASE.d, np.arange(BASE.vocab))
+    F1_host = synth.rows_cpu(synth.F_seed(BASE), BASE.d, np.arange(BASE.n_fgrams))
+    F2_host = synth.rows_cpu(synth.F_seed(OTHER), OTHER.d, np.arange(OTHER.n_fgrams))
+    T, F1, F2 = dev_rows(T_host), dev_rows(F1_host), dev_rows(F2_host)
+    tok = synth.query_tokens(BASE)
+    tok_d = torch.from_numpy(tok).to(DEV)
+    n = tok.size
+    out = torch.empty((n, BASE.d), dtype=torch.int16, device=DEV)
+    row = torch.empty(n, dtype=torch.int32, device=DEV)
+    ln = torch.empty(n, dtype=torch.uint8, device=DEV)
+    table = scone.scone_table_build(fg1_tok, fg1_len, BASE.K, BASE.vocab, BASE.d, F1, T)
+
+    def capture():
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            scone.scone_embed(table, tok_d, out, row, ln)      # warm-up outside capture
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            scone.scone_embed(table, tok_d, out, row, ln)
+        return g
+
+    def replay(g):
+        out.fill_(0)
+        g.replay()
+        torch.cuda.synchronize()
+        return (out.cpu().numpy().view(np.uint16), row.cpu().numpy(), ln.cpu().numpy())
+
+    g1 = capture()
+    _same_as_oracle(replay(g1), fg1_tok, fg1_len, F1_host, T_host, tok)
+    scone.scone_table_rebuild_noalloc(table, fg2_tok, fg2_len, F2)
+    g2 = capture()
+    got = replay(g2)
+    _same_as_oracle(got, fg2_tok, fg2_len, F2_host, T_host, tok)
+    fresh = scone.scone_table_build(fg2_tok, fg2_len, BASE.K, BASE.vocab, BASE.d, F2, T)
+    for x, y in zip(got, run_embed(fresh, tok, BASE.d)):
+        assert np.array_equal(x, y)
+    fresh.close()
+    del g1, g2
     assert scone.scone_status(table) == scone.SCONE_OK
     table.close()
 
@@ -114,8 +255,11 @@ def test_rebuild_noalloc_scratch_limit():
     error before any device work, and the table keeps its previous list."""
     K, vocab, d = 3, 1000, 8
     scratch = 16 << 20                                  # SCONE_REBUILD_SCRATCH_BYTES
-    n_under, n_over = 1_200_000, 1_300_000
     need = lambda n: 256 + -(-n // 256) * 256 + -(-(n * 4 * K) // 256) * 256
+    n_under = (scratch - 768) // (4 * K + 1)            # SCONE_REBUILD_MAX_FGRAMS(3)
+    n_over = n_under + 1
+    while need(n_over) <= scratch:                      # the first size the header's rule refuses
+        n_over += 1
     assert need(n_under) <= scratch < need(n_over)
     T = dev_rows(np.zeros((vocab, d), np.uint16))
     ft0, fl0 = _distinct_trigrams(100_000, vocab)
