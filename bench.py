@@ -5,11 +5,16 @@
 
 One step is one pass of the whole path (match + gather, fused in one launch)
 over one batch of the workload's seeded synthetic tokens; the default
-workload is the 1B-model prefill configuration (32 x 2048 tokens, 1e6
-f-grams, K = 3, d = 2048, Zipf(1.1) over a 100k vocabulary). Steps rotate
-over 4 distinct batches and L2 is flushed (256 MB written, then read) between timed
-steps; each step is timed with CUDA events on its stream. Prints one JSON
-line (see the keys below). ``--impl reference`` times the CPU oracle (the
+workload is the largest configuration that fits one GPU, the large
+HBM-resident table (64 x 4096 tokens, 1e7 f-grams (41 GB of F), K = 3,
+d = 2048, Zipf(1.1) over a 100k vocabulary). Steps rotate over 4 distinct
+batches and L2 is flushed (256 MB written, then read) between timed steps;
+each step is timed with CUDA events on its stream. Prints one JSON line (see
+the keys below). Without --workload, the same process also measures the
+1B-model prefill (32 x 2048 tokens, 1e6 f-grams) and the offloaded decode
+tier (2e7 f-grams, 82 GB of F in host memory read over the host link, 512
+sequences x 256 steps) and reports them under "extra" with their own
+roofline, clocks and e2e. ``--impl reference`` times the CPU oracle (the
 plain statement of Algorithm 1) on the host cores instead.
 
 Under torchrun (N > 1) every rank embeds its own batches (independent
@@ -56,11 +61,17 @@ def workload(name):
         # the offloaded-decode law with 2e6 f-grams (8 GB of host rows) for ncu captures
         return synth.WORKLOADS["offload_decode"].scaled(
             "decode_profile", quotas=((2, 1_200_000), (3, 800_000)))
+    if name == "offload_decode_first_seen":
+        # the offloaded decode with F's rows in first-seen order instead of by count
+        return synth.WORKLOADS["offload_decode"].scaled("offload_decode_first_seen",
+                                                        row_order="first_seen")
     return synth.WORKLOADS[name]
 
 
 N_BATCHES = 4
 FLUSH_BYTES = 256 << 20
+# the largest configuration that fits one GPU (41 GB of F in HBM)
+DEFAULT_WORKLOAD = "large_hbm"
 
 
 def flush_l2(buf):
@@ -81,7 +92,7 @@ class ClockSampler:
                0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
                0x100: "display_clock_setting"}
 
-    def __init__(self, index: int, period_s: float = 0.005):
+    def __init__(self, index: int, period_s: float = 0.001):
         self.ok = False
         self.samples = []
         self.reasons = 0
@@ -388,6 +399,40 @@ def prefill_config(w, world: int) -> dict:
     }
 
 
+def host_F_for(o, batches, w, F_dev=None):
+    """A host array [n_fgrams, d] holding the F rows that the oracle selects
+    on these batches (untimed set-up of the CPU legs). It spans every row, but
+    only the pages of the selected rows are ever written, so a 41 GB F
+    commits a few GB at most. The rows come from the device copy when one is
+    given, else from the host-side generator."""
+    sel = np.unique(np.concatenate([o.select(b)[0].reshape(-1) for b in batches]))
+    sel = sel[sel >= 0]
+    Fh = np.zeros((max(w.n_fgrams, 1), w.d), np.uint16)     # lazily committed pages
+    if sel.size == 0:
+        return Fh
+    if F_dev is not None:
+        import torch
+
+        for a in range(0, sel.size, 1 << 16):
+            part = sel[a:a + (1 << 16)]
+            idx = torch.from_numpy(part).to(F_dev.device)
+            Fh[part] = F_dev.index_select(0, idx).cpu().numpy().view(np.uint16)
+        return Fh
+    import concurrent.futures as cf
+
+    import synth
+
+    chunks = np.array_split(sel, max(1, min(16, os.cpu_count() or 1) * 4))
+
+    def fill(part):
+        if part.size:
+            Fh[part] = synth.rows_cpu(synth.F_seed(w), w.d, part)
+
+    with cf.ThreadPoolExecutor(min(16, os.cpu_count() or 1)) as ex:
+        list(ex.map(fill, chunks))
+    return Fh
+
+
 def cpu_baseline(w, fg_tok, fg_len, tok, F, T, budget_s: float = 10.0):
     """The oracle as it stands (single thread, std::map) on a bounded sample:
     whole passes over one batch until budget_s of CPU work is done. Beside it,
@@ -396,7 +441,7 @@ def cpu_baseline(w, fg_tok, fg_len, tok, F, T, budget_s: float = 10.0):
     import oracle
 
     o = oracle.Oracle(fg_tok, fg_len, w.K, w.vocab)
-    Fh = F.cpu().numpy().view(np.uint16)
+    Fh = host_F_for(o, [tok], w, F_dev=F)
     Th = T.cpu().numpy().view(np.uint16)
 
     def timed(seqs, threads, budget):
@@ -528,7 +573,7 @@ def bench_decode(args, world, rank, local):
     with torch.cuda.graph(g):
         for k in range(steps):
             scone.scone_decode_step(st, new_d[k], out)
-    replays = max(1, args.steps // steps)
+    replays = max(10, args.steps // steps)
     for _ in range(max(1, args.warmup // steps) + 1):
         g.replay()
     torch.cuda.synchronize()
@@ -570,6 +615,7 @@ def bench_decode(args, world, rank, local):
     host_bytes_step = matched / steps * 2 * w.d
     hbm_bytes_step = (S * (4 + 32 * (w.K - 1)) + (S - matched / steps) * 2 * w.d + S * 2 * w.d)
     achieved = host_bytes_step / (ms_step * 1e-3) / 1e9
+    fracs = [host_bytes_step * steps / (t * 1e-3) / 1e9 / link["peak_gbs"] for t in per_replay]
     res = {
         "metric": METRIC,
         "value": S / (ms_step * 1e-3),
@@ -586,7 +632,8 @@ def bench_decode(args, world, rank, local):
         "config": {
             "workload": (f"{w.name}: {S} live sequences x {steps} decode steps, "
                          f"{w.n_fgrams} f-grams (n=2..{w.K}), d={w.d}, vocab {w.vocab}, "
-                         f"F ({w.n_fgrams * w.d * 2 / 1e9:.1f} GB) host-pinned, device-mapped"),
+                         f"F ({w.n_fgrams * w.d * 2 / 1e9:.1f} GB) host-pinned, device-mapped, "
+                         f"rows in {w.row_order.replace('_', '-')} order"),
             "timing": f"{steps} steps captured in one CUDA graph, {replays} replays, "
                       "CUDA events per replay",
             "l2": "working set per replay (~%d MB of rows) exceeds L2" %
@@ -617,6 +664,9 @@ def bench_decode(args, world, rank, local):
         "clocks": clocks.summary(),
         "match_len_hist": {str(i): int(c) for i, c in enumerate(hist_counts)},
         "match_rate": matched / (S * steps),
+        "replay_frac": {"median": statistics.median(fracs), "min": min(fracs),
+                        "max": max(fracs), "replays": replays,
+                        "what": "host-link fraction of each graph replay (256 steps)"},
         "setup_s": setup_s,
     }
     st.close()
@@ -1353,9 +1403,10 @@ PREFILL_WORKLOADS = ("tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_pr
 
 
 def bench_reference(args, world, rank):
-    """The reference arm: the CPU oracle (the plain definition of Algorithm 1)
-    on the host cores, on the prefill workloads' config, metric and unit. Each
-    step is a bounded sample of the workload (one sequence)."""
+    """The reference arm: the CPU oracle (the plain definition of Algorithm 1,
+    single-threaded) on the host cores, on the measured arm's config, metric
+    and unit. Each step embeds one whole batch of the workload (B x L
+    tokens), rotating over the same batches the measured arm times."""
     import synth
     import oracle
 
@@ -1364,35 +1415,62 @@ def bench_reference(args, world, rank):
         return {"impl": "reference", "unavailable": (
             f"the reference arm times the embedding oracle on the prefill workloads; "
             f"{args.workload} reports its CPU oracle under cpu_baseline of its own line")}
+    t0 = time.time()
     fg_tok, fg_len, _ = synth.fgram_set(w)
-    tok = synth.query_tokens(w, range(0, 8))
+    # batch k of rank r is the one the measured arm's rank r embeds at step k
+    batches = [[synth.query_tokens(w, range((r * N_BATCHES + k) * w.B,
+                                            (r * N_BATCHES + k + 1) * w.B))
+                for k in range(N_BATCHES)] for r in range(world)]
     o = oracle.Oracle(fg_tok, fg_len, w.K, w.vocab)
-    # rows the sample can select: T in full, F rows generated on the host
-    F = synth.rows_range_cpu(synth.F_seed(w), w.d, 0, w.n_fgrams)
+    # rows the batches select, generated on the host; T in full
+    F = host_F_for(o, [b for per_rank in batches for b in per_rank], w)
     T = synth.rows_range_cpu(synth.T_seed(w), w.d, 0, w.vocab)
-    seqs = 1
+    setup_s = time.time() - t0
+
+    def step(k):
+        for per_rank in batches:                     # the whole job's batch of step k
+            o.embed(per_rank[k % N_BATCHES], F, T)
+
     for k in range(args.warmup):
-        o.embed(tok[k % 8:k % 8 + seqs], F, T)
+        step(k)
     times = []
     for k in range(args.steps):
         t1 = time.perf_counter()
-        o.embed(tok[k % 8:k % 8 + seqs], F, T)
+        step(k)
         times.append(time.perf_counter() - t1)
     ms = 1e3 * statistics.mean(times)
-    val = seqs * w.L / (ms * 1e-3)
-    sample = f"each step: oracle over {seqs} x {w.L} tokens of {w.name} (map build untimed)"
+    n_tok = world * w.B * w.L
+    val = n_tok / (ms * 1e-3)
+    sample = (f"each step: the oracle over the whole job's batch of {w.name} ({world} x "
+              f"{w.B} x {w.L} = {n_tok} tokens; {N_BATCHES} batches per rank in rotation; "
+              f"map build untimed)")
     return {
         "impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded Zipf token streams and f-gram sets, N(0,0.02)-like bf16 rows)",
         "config": {**prefill_config(w, world),
-                   "timing": "host clock around each oracle call, one sequence per step"},
+                   "timing": "host clock around the oracle calls of one step (the whole "
+                             "job's batch)"},
         "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
+        "setup_s": setup_s,
     }
+
+
+EXTRA_KEYS = ("value", "unit", "ms_per_step", "steps", "warmup", "config", "roofline", "e2e",
+              "gpu_launches", "clocks", "match_rate", "match_len_hist", "kernel_ms_median",
+              "replay_frac")
+
+
+def extra_summary(res: dict) -> dict:
+    """The keys of another workload's line that go under 'extra' of the main one."""
+    out = {k: res[k] for k in EXTRA_KEYS if k in res}
+    if "roofline" in out:
+        out["roofline"] = {k: v for k, v in out["roofline"].items()}
+    return out
 
 
 def main():
@@ -1401,16 +1479,23 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="scone", choices=["scone", "reference"])
-    ap.add_argument("--workload", default="prefill_1b",
+    ap.add_argument("--workload", default=None,
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
-                             "offload_decode", "decode_profile", "prescan", "discover",
-                             "discover_k5", "discover_profile", "mixed_serving", "precompute",
-                             "gemm_profile", "store_decode"])
+                             "offload_decode", "offload_decode_first_seen", "decode_profile",
+                             "prescan", "discover", "discover_k5", "discover_profile",
+                             "mixed_serving", "precompute", "gemm_profile", "store_decode"],
+                    help="default: large_hbm, plus prefill_1b and offload_decode under "
+                         "'extra' (single GPU)")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="without --workload: measure large_hbm only")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk"],
                     help="row copy method of the fused kernel (results are identical)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
+    extras = args.workload is None and not args.no_extras
+    if args.workload is None:
+        args.workload = DEFAULT_WORKLOAD
     world, rank, local = dist_setup()
     if args.impl == "reference":
         if rank == 0:
@@ -1421,7 +1506,7 @@ def main():
     if rank == 0:
         __graft_entry__.build()
     barrier(world)
-    if args.workload in ("offload_decode", "decode_profile"):
+    if args.workload in ("offload_decode", "offload_decode_first_seen", "decode_profile"):
         res = bench_decode(args, world, rank, local)
     elif args.workload == "prescan":
         res = bench_prescan(args, world, rank, local)
@@ -1437,6 +1522,23 @@ def main():
         res = bench_discover(args, world, rank, local)
     else:
         res = bench_prefill(args, world, rank, local)
+    if extras and world == 1:
+        # the other two configurations measured in the same process: the
+        # 1B-model prefill and the offloaded tier (F in host memory, read over
+        # the host link), each with its own roofline, clocks and e2e
+        import torch
+
+        res["extra"] = {}
+        for name, fn in (("prefill_1b", bench_prefill), ("offload_decode", bench_decode)):
+            torch.cuda.empty_cache()
+            sub = argparse.Namespace(**vars(args))
+            sub.workload = name
+            sub.no_cpu_baseline = True
+            sub.steps = max(args.steps, 200)
+            sub.warmup = max(args.warmup, 10)
+            res["extra"][name] = extra_summary(fn(sub, world, rank, local))
+            res["gpu_launches_extra"] = res.get("gpu_launches_extra", 0) + \
+                res["extra"][name]["gpu_launches"]
     if rank == 0:
         print(json.dumps(res), flush=True)
     if world > 1:

@@ -75,7 +75,7 @@ def _load():
     lib.synth_phrase_pool.argtypes = [u64, i32, dbl, i32, i32, i32, _i32p, _i32p]
     lib.synth_phrase_pool.restype = ctypes.c_int
     lib.synth_fgram_set.argtypes = [u64, i32, dbl, i32, _i64p, dbl, _i32p, _i32p, i32, i32, i64,
-                                    _i32p, _u8p, _i64p]
+                                    _i32p, _u8p, _i64p, _i64p]
     lib.synth_fgram_set.restype = i64
     lib.synth_rows_cpu.argtypes = [u64, i32, _i64p, i64, _u16p]
     lib.synth_rows_cpu.restype = None
@@ -111,6 +111,10 @@ class Workload:
     dec_hist: int = 0                    # decode: history tokens per sequence
     dec_steps: int = 0                   # decode: steps
     min_count: int = 5                   # f-gram discovery: eligibility threshold (Sec. 3.2)
+    # order of the f-gram list (row r of F belongs to f-gram r): "first_seen" in
+    # the source stream, or "count": by descending count in the source stream
+    # (ties in first-seen order), the order a top-S-by-count selection yields
+    row_order: str = "first_seen"
 
     @property
     def n_fgrams(self) -> int:
@@ -143,7 +147,8 @@ WORKLOADS: Dict[str, Workload] = {
                           _split(10_000_000, {2: 0.6, 3: 0.4}), 3, 2048),
     "offload_decode": Workload("offload_decode", 4, 100000, 1.1, 0, 0,
                                _split(20_000_000, {2: 0.6, 3: 0.4}), 3, 2048,
-                               location="host_mapped", dec_S=512, dec_hist=2, dec_steps=256),
+                               location="host_mapped", dec_S=512, dec_hist=2, dec_steps=256,
+                               row_order="count"),
     "stress_k5": Workload("stress_k5", 5, 100000, 1.05, 16, 8192,
                           ((2, 1_666_666), (3, 1_666_666), (4, 833_334), (5, 833_334)), 5, 1536,
                           inject_p=0.05 / 6, n_phrases=4096),
@@ -223,19 +228,17 @@ def query_tokens(w: Workload, seqs: Optional[range] = None, out: Optional[np.nda
     return out
 
 
-_FGRAM_CACHE: Dict[Workload, Tuple[np.ndarray, np.ndarray, int]] = {}
+_FGRAM_CACHE: Dict[Workload, tuple] = {}
 
 
-def fgram_set(w: Workload, max_stream: int = 4_000_000_000):
-    """(fgram_tok [N, K] int32 padded with -1, fgram_len [N] uint8, stream tokens used)."""
-    if w in _FGRAM_CACHE:
-        return _FGRAM_CACHE[w]
+def _fgram_set_first_seen(w: Workload, max_stream: int, with_counts: bool):
     quota = np.zeros(w.K + 1, np.int64)
     for n, c in w.quotas:
         quota[n] = c
     N = int(quota.sum())
     tok = np.empty((N, w.K), np.int32)
     ln = np.empty(N, np.uint8)
+    counts = np.empty(N, np.int64) if with_counts else None
     used = ctypes.c_int64(0)
     pt, pl = phrase_pool(w)
     n_ph = 0 if pt is None else pt.shape[0]
@@ -243,14 +246,40 @@ def fgram_set(w: Workload, max_stream: int = 4_000_000_000):
     got = _load().synth_fgram_set(stream_seed(w, S_SOURCE), w.vocab, w.zipf_s, w.K,
                                   _p(quota, _i64p), w.inject_p if n_ph else 0.0, _p(pt, _i32p),
                                   _p(pl, _i32p), n_ph, stride, max_stream, _p(tok, _i32p),
-                                  _p(ln, _u8p), ctypes.byref(used))
+                                  _p(ln, _u8p), ctypes.byref(used), _p(counts, _i64p))
     if got != N:
         raise RuntimeError(f"f-gram generation for {w.name} failed ({got})")
-    res = (tok, ln, int(used.value))
+    return tok, ln, int(used.value), counts
+
+
+def fgram_set(w: Workload, max_stream: int = 4_000_000_000):
+    """(fgram_tok [N, K] int32 padded with -1, fgram_len [N] uint8, stream tokens used),
+    listed in the workload's row order."""
+    return _fgram_entry(w, max_stream)[:3]
+
+
+def fgram_counts(w: Workload, max_stream: int = 4_000_000_000) -> np.ndarray:
+    """Count of each f-gram of fgram_set(w) (same order) in the source stream."""
+    e = _fgram_entry(w, max_stream, with_counts=True)
+    return e[3]
+
+
+def _fgram_entry(w: Workload, max_stream: int, with_counts: bool = False):
+    e = _FGRAM_CACHE.get(w)
+    if e is not None and (e[3] is not None or not with_counts):
+        return e
+    need_counts = with_counts or w.row_order == "count"
+    tok, ln, used, counts = _fgram_set_first_seen(w, max_stream, need_counts)
+    if w.row_order == "count":
+        order = np.argsort(-counts, kind="stable")
+        tok, ln, counts = tok[order], ln[order], counts[order]
+    elif w.row_order != "first_seen":
+        raise ValueError(f"unknown row order {w.row_order}")
+    e = (tok, ln, used, counts)
     if len(_FGRAM_CACHE) >= 4:
         _FGRAM_CACHE.pop(next(iter(_FGRAM_CACHE)))
-    _FGRAM_CACHE[w] = res
-    return res
+    _FGRAM_CACHE[w] = e
+    return e
 
 
 def rows_cpu(seed: int, d: int, row_ids) -> np.ndarray:

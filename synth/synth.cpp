@@ -118,6 +118,16 @@ struct WindowSet {
   std::vector<int64_t> slots;
   size_t used = 0;
   WindowSet(const std::vector<int32_t>& s, int n_) : src(s), n(n_), slots(1 << 16, -1) {}
+  // Slot of the stored window equal to the window at p, or -1.
+  int64_t find(int64_t p) const {
+    const size_t mask = slots.size() - 1;
+    size_t i = hash_at(p) & mask;
+    while (slots[i] >= 0) {
+      if (same(slots[i], p)) return (int64_t)i;
+      i = (i + 1) & mask;
+    }
+    return -1;
+  }
   uint64_t hash_at(int64_t p) const {
     uint64_t h = 0x51ED270B27FA1C3Dull ^ (uint64_t)n;
     for (int j = 0; j < n; ++j) h = mix64(h ^ (uint64_t)(uint32_t)src[p + j]);
@@ -248,11 +258,13 @@ int synth_phrase_pool(uint64_t seed, int32_t vocab, double s, int32_t n_ph, int3
 // is not full, the window src[p .. p+n-1] is appended if it was not seen
 // before. The stream is extended until every quota is full or max_stream
 // tokens were used. Outputs are fgram_tok[N * K] (row-padded with -1) and
-// fgram_len[N], N = sum of quotas. Returns N, or -1 (bad args), -2 (cap hit).
+// fgram_len[N], N = sum of quotas. If counts is not NULL, counts[r] receives
+// the number of windows equal to f-gram r in the whole stream that was
+// generated (stream_used tokens). Returns N, or -1 (bad args), -2 (cap hit).
 int64_t synth_fgram_set(uint64_t seed, int32_t vocab, double s, int32_t K, const int64_t* quota,
                         double inject_p, const int32_t* ph_tok, const int32_t* ph_len,
                         int32_t n_ph, int32_t ph_stride, int64_t max_stream, int32_t* fgram_tok,
-                        uint8_t* fgram_len, int64_t* stream_used) {
+                        uint8_t* fgram_len, int64_t* stream_used, int64_t* counts) {
   if (vocab <= 0 || K < 2 || K > 16 || !quota || !fgram_tok || !fgram_len) return -1;
   int64_t total = 0;
   for (int n = 2; n <= K; ++n) {
@@ -286,6 +298,42 @@ int64_t synth_fgram_set(uint64_t seed, int32_t vocab, double s, int32_t K, const
     }
   }
   if (stream_used) *stream_used = (int64_t)src.size();
+  if (counts && rc == 0) {
+    // row of each stored window: the f-grams of length n were appended in
+    // increasing first position, so row r of length n pairs with the r-th
+    // smallest stored position of that length
+    std::vector<std::vector<int64_t>> slot_row(K + 1);
+    for (int n = 2; n <= K; ++n) {
+      std::vector<int64_t> rows;
+      for (int64_t r = 0; r < filled; ++r)
+        if (fgram_len[r] == n) rows.push_back(r);
+      std::vector<std::pair<int64_t, int64_t>> by_pos;  // (stored position, slot)
+      const auto& sl = sets[n]->slots;
+      for (size_t i = 0; i < sl.size(); ++i)
+        if (sl[i] >= 0) by_pos.emplace_back(sl[i], (int64_t)i);
+      std::sort(by_pos.begin(), by_pos.end());
+      slot_row[n].assign(sl.size(), -1);
+      for (size_t k = 0; k < by_pos.size(); ++k) slot_row[n][by_pos[k].second] = rows[k];
+    }
+    for (int64_t r = 0; r < filled; ++r) counts[r] = 0;
+    // every window of the stream, split over threads; counts are atomic adds
+    const int64_t end = (int64_t)src.size();
+    const int threads = std::max(1u, std::min(16u, std::thread::hardware_concurrency()));
+    std::vector<std::thread> pool;
+    const int64_t per = (end + threads - 1) / threads;
+    for (int t = 0; t < threads; ++t) {
+      const int64_t a = t * per, b = std::min<int64_t>(end, a + per);
+      if (a >= b) break;
+      pool.emplace_back([&, a, b] {
+        for (int n = 2; n <= K; ++n)
+          for (int64_t p = a; p < b && p + n <= end; ++p) {
+            const int64_t i = sets[n]->find(p);
+            if (i >= 0) __atomic_fetch_add(&counts[slot_row[n][i]], 1, __ATOMIC_RELAXED);
+          }
+      });
+    }
+    for (auto& th : pool) th.join();
+  }
   for (int n = 2; n <= K; ++n) delete sets[n];
   return rc ? rc : filled;
 }

@@ -19,18 +19,33 @@ def run_bench(*args):
     return json.loads(lines[0])
 
 
+def test_default_workload_is_the_largest_single_gpu_config():
+    import bench
+    import synth
+
+    w = synth.WORKLOADS[bench.DEFAULT_WORKLOAD]
+    hbm = [x for x in synth.WORKLOADS.values()
+           if x.location == "device" and x.B * x.L > 0 and x.d > 8]
+    assert w.n_fgrams * w.d == max(x.n_fgrams * x.d for x in hbm)
+
+
 def test_reference_line_keys():
     import bench
 
-    d = run_bench("--impl", "reference", "--steps", "2", "--warmup", "1")
+    # the tiny workload keeps this CPU test short; the default (large_hbm)
+    # runs the same code on a larger batch
+    d = run_bench("--impl", "reference", "--workload", "tiny", "--steps", "2", "--warmup", "1")
     assert d["impl"] == "reference"
     assert d["metric"] == bench.METRIC and d["unit"] == "tokens/s"
     assert d["higher_is_better"] is True and d["value"] > 0
     assert d["warmup"] >= 3 and d["steps"] == 2
     import synth
 
-    w = synth.WORKLOADS["prefill_1b"]
+    w = synth.WORKLOADS["tiny"]
+    # the arm times what its config names: one whole B x L batch per step
     assert d["config"]["workload"] == bench.prefill_config(w, 1)["workload"]
+    assert d["config"]["global_batch_tokens"] == w.B * w.L
+    assert f"{w.B} x {w.L}" in d["cpu_baseline"]["sample"]
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,

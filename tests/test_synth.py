@@ -88,3 +88,31 @@ def test_query_batch_equals_per_sequence_streams():
         for k, b in enumerate(range(3, 8)):
             one = synth.zipf_tokens(w, synth.stream_seed(w, synth.S_QUERY, b), w.L)
             assert np.array_equal(batch[k], one)
+
+
+def test_fgram_counts_and_count_order():
+    """Counts are the number of windows equal to each f-gram in the whole
+    generated source stream (checked by a plain dictionary count); the count
+    order lists the same set by descending count, ties in first-seen order."""
+    base = synth.WORKLOADS["tiny"].scaled("tiny_cnt", quotas=((2, 400), (3, 300)))
+    tok, ln, used = synth.fgram_set(base)
+    cnt = synth.fgram_counts(base)
+    src = synth.zipf_tokens(base, synth.stream_seed(base, synth.S_SOURCE), used)
+    ref = {}
+    for n in (2, 3):
+        for p in range(used - n + 1):
+            g = tuple(int(x) for x in src[p:p + n])
+            ref[g] = ref.get(g, 0) + 1
+    grams = [tuple(int(x) for x in tok[r, :ln[r]]) for r in range(ln.shape[0])]
+    assert [ref[g] for g in grams] == cnt.tolist()
+    assert (cnt >= 1).all()
+    w = base.scaled("tiny_cnt_order", row_order="count")
+    tok2, ln2, used2 = synth.fgram_set(w)
+    cnt2 = synth.fgram_counts(w)
+    assert used2 == used
+    grams2 = [tuple(int(x) for x in tok2[r, :ln2[r]]) for r in range(ln2.shape[0])]
+    first = {g: r for r, g in enumerate(grams)}
+    assert sorted(grams2) == sorted(grams)
+    keys = [(-ref[g], first[g]) for g in grams2]
+    assert keys == sorted(keys)
+    assert cnt2.tolist() == [ref[g] for g in grams2]
