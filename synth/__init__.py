@@ -328,8 +328,10 @@ class FgramModel:
     The packed weight buffer holds, per layer, four row-major bf16 matrices:
     qkv [3d x d] (query, key, value rows), o [d x d], gu [2 ffw x d] (gate and
     up rows interleaved in groups of 16: rows 32g..32g+15 are the gates of
-    features 16g..16g+15, the next 16 rows their ups), down [d x ffw]. Every
-    entry is an independent draw of the bf16 row generator (std 0.02).
+    features 16g..16g+15, the next 16 rows their ups), down [d x ffw]. With
+    absolute positions (the paper's scheme, Appendix F) the buffer ends with
+    the position table P [max_pos x d] after the last layer. Every entry is an
+    independent draw of the bf16 row generator (std 0.02).
     """
     name: str
     mid: int          # model id, mixed into every seed
@@ -337,6 +339,8 @@ class FgramModel:
     n_heads: int
     ffw: int
     n_layers: int
+    max_pos: int = 8              # positions of P: the longest f-gram the model takes
+    position: str = "absolute"    # "absolute" (P added to the input) or "rotary"
 
     def shapes(self):
         d, f = self.d, self.ffw
@@ -347,8 +351,17 @@ class FgramModel:
         return sum(r * c for _, r, c in self.shapes())
 
     @property
-    def n_elems(self) -> int:
+    def pos_offset(self) -> int:
+        """Element offset of P (after the last layer)."""
         return self.n_layers * self.layer_elems
+
+    @property
+    def pos_elems(self) -> int:
+        return self.max_pos * self.d if self.position == "absolute" else 0
+
+    @property
+    def n_elems(self) -> int:
+        return self.n_layers * self.layer_elems + self.pos_elems
 
     def offset(self, layer: int, which: str) -> int:
         off = layer * self.layer_elems
@@ -363,8 +376,9 @@ MODELS: Dict[str, FgramModel] = {
     # small enough for the fp64 oracle on every f-gram of a test
     "tiny": FgramModel("tiny", 20, 256, 4, 512, 2),
     # the 711M OLMo shape the paper uses for its smaller f-gram model
-    # (d_model 2048, ffw 8192, 12 layers; 16 heads of 128)
-    "olmo_711m": FgramModel("olmo_711m", 21, 2048, 16, 8192, 12),
+    # (d_model 2048, ffw 8192, 12 layers; 16 heads of 128); 3 positions, the
+    # longest f-gram of the lists it precomputes (K = 3)
+    "olmo_711m": FgramModel("olmo_711m", 21, 2048, 16, 8192, 12, max_pos=3),
 }
 
 
@@ -379,6 +393,9 @@ def model_weights_cpu(m: FgramModel) -> np.ndarray:
         for k, (name, r, c) in enumerate(m.shapes()):
             off = m.offset(layer, name)
             out[off:off + r * c] = rows_range_cpu(model_seed(m, layer, k), c, 0, r).reshape(-1)
+    if m.pos_elems:
+        out[m.pos_offset:] = rows_range_cpu(model_seed(m, m.n_layers, 0), m.d, 0,
+                                            m.max_pos).reshape(-1)
     return out
 
 
@@ -388,3 +405,6 @@ def model_weights_gpu(m: FgramModel, out_ptr: int, stream_ptr: int) -> None:
         for k, (name, r, c) in enumerate(m.shapes()):
             rows_gpu(model_seed(m, layer, k), c, 0, r, out_ptr + 2 * m.offset(layer, name),
                      stream_ptr)
+    if m.pos_elems:
+        rows_gpu(model_seed(m, m.n_layers, 0), m.d, 0, m.max_pos, out_ptr + 2 * m.pos_offset,
+                 stream_ptr)

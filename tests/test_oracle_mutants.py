@@ -6,7 +6,9 @@ handling, gather source, decode history alignment) and for Algorithm 3
 (window bound, length range, first occurrence, threshold, sort direction, tie
 order, the top-S cut, sequence boundary), and in the f-gram model oracle
 (rotation direction and base, causal mask, score scale, layer-norm epsilon,
-gate/up swap, a dropped residual, the output position, bf16 tie rounding).
+gate/up swap, a dropped residual, the output position, bf16 tie rounding,
+and the absolute positions dropped, counted from the end, or added after the
+first layer norm).
 The copy is compiled (C++) or loaded (Python) on the CPU and the pin tests
 run against it in a subprocess; they must fail.
 """
@@ -36,6 +38,13 @@ MODEL_MUTANTS = {
     "m_attention_residual_dropped": ('x = r(x + o @ L["o"].T)', 'x = r(o @ L["o"].T)'),
     "m_first_position": ("f = layer_norm(x[-1:])[0]", "f = layer_norm(x[:1])[0]"),
     "m_round_half_up": ("np.round(m * 256.0)", "np.floor(m * 256.0 + 0.5)"),
+    # the absolute position scheme of Appendix F
+    "m_pos_dropped": ("    x0 = x0 + position_rows(W, idx.shape[0])\n", "    x0 = x0\n"),
+    "m_pos_from_end": ("    return W.P[:n]\n", "    return W.P[:n][::-1]\n"),
+    "m_pos_after_first_ln": [
+        ("    x0 = x0 + position_rows(W, idx.shape[0])\n", "    x0 = x0\n"),
+        ("        xn = r(layer_norm(x))\n        q, k, v",
+         "        xn = r(layer_norm(x) + position_rows(W, x.shape[0]))\n        q, k, v")],
 }
 
 SCAN = """  for (int64_t jp = first; jp < i; ++jp) {
@@ -137,11 +146,13 @@ def test_unmutated_copy_passes(tmp_path):
 
 @pytest.mark.parametrize("name", sorted(MODEL_MUTANTS))
 def test_model_mutant_is_caught(name, tmp_path):
-    old, new = MODEL_MUTANTS[name]
+    edits = MODEL_MUTANTS[name]
     src = open(MODEL_SRC).read()
-    assert old in src, f"mutation site for {name} not found"
+    for old, new in ([edits] if isinstance(edits, tuple) else edits):
+        assert src.count(old) == 1, f"mutation site for {name} not found once"
+        src = src.replace(old, new)
     path = tmp_path / "fgram_model_mut.py"
-    path.write_text(src.replace(old, new))
+    path.write_text(src)
     env = dict(os.environ, SCONE_FGRAM_ORACLE_FILE=str(path))
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
                         MODEL_PINS], cwd=ROOT, env=env, capture_output=True, text=True,
