@@ -1052,7 +1052,8 @@ def bench_precompute(args, world, rank, local):
     tok_d = torch.from_numpy(fg_tok).to(dev)
     len_d = torch.from_numpy(fg_len).to(dev)
     F = torch.empty((n_f, m.d), dtype=torch.int16, device=dev)
-    model = scone.FgramModel(m.d, m.n_heads, m.ffw, m.n_layers, weights, batch=16384)
+    model = scone.FgramModel(m.d, m.n_heads, m.ffw, m.n_layers, weights, batch=16384,
+                             max_pos=m.max_pos)
     setup_s = time.time() - t0
     tokens = int(fg_len.astype(np.int64).sum())
     flops = model_flops_per_token(m) * tokens

@@ -380,24 +380,32 @@ int scone_gemm_bf16_variant(const scone_bf16* A, const scone_bf16* B, const scon
 /*
  * Precomputing F with the f-gram model (Sec. 3.2: after training F is
  * precomputed and stored; Algorithm 1 embeds an f-gram by A_fgram(T(s_j), ..,
- * T(s_i)) in training). The model is a pre-LN transformer: per layer
- * h = x + Attn(LN(x)), x = h + MLP(LN(h)); LN is the non-parametric layer norm
- * (eps 1e-5); Attn is causal multi-head attention with rotary positions
- * (rotate-half pairs (i, i + hd/2), angle pos * 10000^(-2i/hd)), scaled by
- * 1/sqrt(hd); MLP is SwiGLU. F(w) = LN of the last position's final state.
+ * T(s_i)) in training). The model is a pre-LN transformer over the f-gram's
+ * token rows plus absolute position embeddings: x_0[j] = T(s_j) + P[j],
+ * j = 0..n-1 from the f-gram's first token (Appendix F, Implementation
+ * Details: an absolute position embedding layer whose size is the longest
+ * f-gram). Per layer h = x + Attn(LN(x)), x = h + MLP(LN(h)); LN is the
+ * non-parametric layer norm (eps 1e-5); Attn is causal multi-head attention
+ * scaled by 1/sqrt(hd); MLP is SwiGLU. F(w) = LN of the last position's final
+ * state. A model created with SCONE_FGRAM_POS_ROTARY has no P and applies
+ * rotary embeddings to q and k instead (rotate-half pairs (i, i + hd/2),
+ * angle pos * 10000^(-2i/hd)); that option is not the paper's scheme.
  *
  * scone_fgram_model_create: d (multiple of 256, d/256 a power of two up to
  * 16), n_heads (head size d/n_heads in {64, 128, 256}), ffw (multiple of 128),
- * n_layers; weights: device bf16, packed per layer as qkv [3d x d] (query,
- * key, value rows), o [d x d], gu [2 ffw x d] (rows 32g..32g+15 are the gates
- * of features 16g..16g+15, the next 16 rows their ups), down [d x ffw],
- * row-major; borrowed, must outlive the model. batch: f-grams per internal
- * batch (0 = 16384); the workspace grows with the tokens of a batch.
- * Synchronous.
+ * n_layers, max_pos (rows of P, 1..8; ignored for rotary), position;
+ * weights: device bf16, packed per layer as qkv [3d x d] (query, key, value
+ * rows), o [d x d], gu [2 ffw x d] (rows 32g..32g+15 are the gates of
+ * features 16g..16g+15, the next 16 rows their ups), down [d x ffw],
+ * row-major, followed (absolute positions) by P [max_pos x d]; borrowed, must
+ * outlive the model. batch: f-grams per internal batch (0 = 16384); the
+ * workspace grows with the tokens of a batch. Synchronous.
  */
+enum scone_fgram_position { SCONE_FGRAM_POS_ABSOLUTE = 0, SCONE_FGRAM_POS_ROTARY = 1 };
 typedef struct scone_fgram_model scone_fgram_model;
 int scone_fgram_model_create(int32_t d, int32_t n_heads, int32_t ffw, int32_t n_layers,
-                             const scone_bf16* weights, int64_t batch, scone_fgram_model** out);
+                             int32_t max_pos, int32_t position, const scone_bf16* weights,
+                             int64_t batch, scone_fgram_model** out);
 int scone_fgram_model_destroy(scone_fgram_model* model);
 
 /*
@@ -406,8 +414,11 @@ int scone_fgram_model_destroy(scone_fgram_model* model);
  * [2, K] (lengths outside [1, K] are read as 1 and reported), T device
  * [vocab * d], F device or host-mapped [n * d] (16-byte aligned). The f-grams
  * of a batch are packed without padding and every dense layer is a
- * tensor-core GEMM over all their tokens. Synchronous; returns SCONE_OK or
- * the first device-detected error (TOKEN_RANGE: that token's row is zero;
+ * tensor-core GEMM over all their tokens (f-grams are not padded: with the
+ * padding of Appendix F after the last token and causal attention, the last
+ * token's output is the same). K above max_pos (absolute positions) is
+ * INVALID_ARG before any device work. Synchronous; returns SCONE_OK or the
+ * first device-detected error (TOKEN_RANGE: that token's input row is zero;
  * INVALID_ARG: a length outside [1, K]; CUDA: a GEMM pipeline timed out).
  */
 int scone_fgram_precompute(scone_fgram_model* model, const int32_t* fgram_tok,

@@ -39,6 +39,8 @@ SCONE_COPY_BULK = 2
 SCONE_GEMM_STORE = 0
 SCONE_GEMM_RESIDUAL = 1
 SCONE_GEMM_SWIGLU = 2
+SCONE_FGRAM_POS_ABSOLUTE = 0
+SCONE_FGRAM_POS_ROTARY = 1
 
 EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noalloc",
            "scone_table_get_info", "scone_table_set_probe_limit", "scone_table_set_copy_mode",
@@ -129,7 +131,7 @@ def load_library():
     lib.scone_gemm_bf16.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp]
     lib.scone_gemm_bf16_variant.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                                             _vp, _vp]
-    lib.scone_fgram_model_create.argtypes = [_i32, _i32, _i32, _i32, _vp, _i64,
+    lib.scone_fgram_model_create.argtypes = [_i32, _i32, _i32, _i32, _i32, _i32, _vp, _i64,
                                              ctypes.POINTER(_vp)]
     lib.scone_fgram_model_destroy.argtypes = [_vp]
     lib.scone_fgram_precompute.argtypes = [_vp, _vp, _vp, _i64, _i32, _vp, _i32, _vp, _vp]
@@ -363,12 +365,15 @@ def scone_gemm_bf16(A, B, C, R=None, epilogue: int = SCONE_GEMM_STORE, status=No
 
 
 class FgramModel:
-    """The f-gram model on the device (borrows its packed weights)."""
+    """The f-gram model on the device (borrows its packed weights). With
+    absolute positions (the default) the weights end with P [max_pos, d]."""
 
-    def __init__(self, d: int, n_heads: int, ffw: int, n_layers: int, weights, batch: int = 0):
+    def __init__(self, d: int, n_heads: int, ffw: int, n_layers: int, weights, batch: int = 0,
+                 max_pos: int = 8, position: int = SCONE_FGRAM_POS_ABSOLUTE):
         h = _vp()
-        _check(load_library().scone_fgram_model_create(d, n_heads, ffw, n_layers, _ptr(weights),
-                                                       batch, ctypes.byref(h)),
+        _check(load_library().scone_fgram_model_create(d, n_heads, ffw, n_layers, max_pos,
+                                                       position, _ptr(weights), batch,
+                                                       ctypes.byref(h)),
                "scone_fgram_model_create")
         self._h = h
         self._keep = weights
@@ -392,8 +397,9 @@ class FgramModel:
             pass
 
 
-def scone_fgram_model_create(d, n_heads, ffw, n_layers, weights, batch=0) -> FgramModel:
-    return FgramModel(d, n_heads, ffw, n_layers, weights, batch)
+def scone_fgram_model_create(d, n_heads, ffw, n_layers, max_pos, position, weights,
+                             batch=0) -> FgramModel:
+    return FgramModel(d, n_heads, ffw, n_layers, weights, batch, max_pos, position)
 
 
 def scone_fgram_model_destroy(model: FgramModel) -> None:

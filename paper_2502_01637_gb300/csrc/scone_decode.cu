@@ -5,11 +5,17 @@
 // keeps, per sequence, a device ring of its last K-1 tokens (right-aligned,
 // oldest first) and how many of them are known. One warp serves one
 // sequence: lane j looks up the window of length j + 2 ending at the new
-// token (its first cuckoo bucket, and the second only when the first is full
-// without the key), a warp ballot keeps the longest hit,
-// the lanes shift the new token into the history, and the warp copies the
-// selected row (F over the host link in the offloaded tier, or T from HBM)
-// with every lane's loads issued at once.
+// token, a warp ballot keeps the longest hit, the lanes shift the new token
+// into the history, and the warp copies the selected row (F over the host
+// link in the offloaded tier, or T from HBM) with every lane's loads issued
+// at once.
+//
+// A step is a chain of dependent reads, so its reads are issued as early as
+// their addresses are known: the new token, the history length and the
+// history entries in one round trip (lane j reads entry j and the window
+// tokens reach the other lanes by shuffles), then both candidate buckets of
+// every length in one round trip (a second 32-byte sector per lookup instead
+// of a second dependent read), then the row.
 //
 // Steps are launched with programmatic dependent launch: each step lets the
 // next one be scheduled at once (griddepcontrol.launch_dependents) and every
@@ -44,26 +50,30 @@ __global__ void __launch_bounds__(kDecThreads)
   asm volatile("griddepcontrol.launch_dependents;");
   for (int64_t s = (int64_t)blockIdx.x * kDecWarps + warp; s < S;
        s += (int64_t)gridDim.x * kDecWarps) {
+    int32_t* hs = hist + s * H;
+    // one round trip: the new token, the history length, history entry `lane`
     const int32_t x = __ldg(new_tok + s);
     const int32_t h = hist_len[s];
-    int32_t* hs = hist + s * H;
+    const int32_t hv = lane < H ? hs[lane] : 0;
     const bool xvalid = valid_token(x, t.vocab);
     const int n = lane + 2;
     int32_t r_lane = -1;
     int err = 0;
-    if (xvalid && n <= t.K && n <= h + 1) {
-      KeyBits<NW> k;
+    KeyBits<NW> k;
 #pragma unroll
-      for (int q = 0; q < NW; ++q) k.w[q] = 0;
-      k.w[0] = (uint32_t)x;
-      bool ok = true;
-      for (int m = 1; m < n; ++m) {
-        const int32_t y = hs[H - m];
+    for (int q = 0; q < NW; ++q) k.w[q] = 0;
+    k.w[0] = (uint32_t)x;
+    bool ok = true;
+    for (int m = 1; m < H + 1; ++m) {     // every lane joins each shuffle
+      const int32_t y = __shfl_sync(0xFFFFFFFFu, hv, H - m);
+      if (m < n) {
         ok = ok && valid_token(y, t.vocab);
         put_field<NW>(k, m * t.bits, (uint32_t)y, t.bits);
       }
+    }
+    if (xvalid && ok && n <= t.K && n <= h + 1) {
       put_len<FMT>(k, n);
-      if (ok) r_lane = cuckoo_lookup<FMT>(t, k, &err);
+      r_lane = cuckoo_lookup_eager<FMT>(t, k, &err);
     }
     const unsigned hits = __ballot_sync(0xFFFFFFFFu, r_lane >= 0);
     const unsigned errs = __ballot_sync(0xFFFFFFFFu, err != 0);
@@ -83,11 +93,9 @@ __global__ void __launch_bounds__(kDecThreads)
       src = r >= 0 ? static_cast<const void*>(t.F + (int64_t)r * t.d)
                    : static_cast<const void*>(t.T + (int64_t)x * t.d);
     }
-    // shift the new token into the history (all lanes have read it above)
-    int32_t keep = 0;
-    if (lane < H) keep = lane + 1 < H ? hs[lane + 1] : x;
-    __syncwarp();
-    if (lane < H) hs[lane] = keep;
+    // shift the new token into the history (entry j takes entry j + 1)
+    const int32_t next = __shfl_down_sync(0xFFFFFFFFu, hv, 1);
+    if (lane < H) hs[lane] = lane + 1 < H ? next : x;
     if (lane == 0) {
       hist_len[s] = h + 1 < H ? h + 1 : H;
       if (row_out) row_out[s] = r;

@@ -202,6 +202,27 @@ __device__ __forceinline__ int32_t cuckoo_lookup(const TableView& t,
   return find_in_bucket<FMT>(ld_bucket_data<FMT>(t, b2), k);
 }
 
+// The same result as cuckoo_lookup with both candidate buckets loaded in one
+// round trip: for latency-bound callers (a decode step) that can spend a
+// second 32-byte sector per lookup to save a dependent read. The second
+// bucket is used only where cuckoo_lookup would read it.
+template <int FMT>
+__device__ __forceinline__ int32_t cuckoo_lookup_eager(const TableView& t,
+                                                       const KeyBits<Fmt<FMT>::kWords>& k,
+                                                       int* err) {
+  uint64_t b1, b2;
+  cuckoo_buckets(key_hash<FMT>(k, t.hash_seed), t.n_buckets, &b1, &b2);
+  const BucketData<FMT> v1 = ld_bucket_data<FMT>(t, b1);
+  const BucketData<FMT> v2 = ld_bucket_data<FMT>(t, b2);
+  const int32_t r = find_in_bucket<FMT>(v1, k);
+  if (r >= 0 || !bucket_full<FMT>(v1)) return r;
+  if (t.probe_limit < 2) {
+    *err = SCONE_ERR_PROBE_LIMIT;
+    return -1;
+  }
+  return find_in_bucket<FMT>(v2, k);
+}
+
 __device__ __forceinline__ void record_error(int* status, int code) {
   if (*reinterpret_cast<volatile int*>(status) == 0) atomicCAS(status, 0, code);
 }

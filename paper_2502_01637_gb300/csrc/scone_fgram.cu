@@ -3,10 +3,18 @@
 // At inference F(w) is the f-gram model's output for w, computed once and
 // stored (Sec. 3.2; Algorithm 1 uses A_fgram(T(s_j), .., T(s_i)) in training
 // and the stored F(s_j, .., s_i) at inference). The model is a pre-LN
-// transformer: per layer h = x + Attn(LN(x)), x = h + MLP(LN(h)), with
-// non-parametric layer norm (eps 1e-5), causal multi-head attention with
-// rotary positions (rotate-half pairs, base 10000) and a SwiGLU MLP; F(w) is
-// the layer norm of the last position's final state.
+// transformer: its input is the f-gram's token rows plus absolute position
+// embeddings P[0..n-1] (Appendix F: an absolute position embedding layer
+// with as many positions as the longest f-gram); per layer
+// h = x + Attn(LN(x)), x = h + MLP(LN(h)), with non-parametric layer norm
+// (eps 1e-5), causal multi-head attention and a SwiGLU MLP; F(w) is the layer
+// norm of the last position's final state. Rotary positions on q and k
+// (rotate-half pairs, base 10000) replace P when a model is created with
+// SCONE_FGRAM_POS_ROTARY; that option is not the paper's scheme.
+//
+// Appendix F pads the f-grams of a batch to the longest one; the padding
+// follows the last token and the attention is causal, so the last token's
+// output does not depend on it, and the f-grams are packed here without it.
 //
 // The f-grams of a batch are packed token after token (no padding) into one
 // [M x d] activation matrix, M = sum of their lengths, so every dense layer
@@ -28,7 +36,10 @@
 struct scone_fgram_model {
   int device = 0;
   int32_t d = 0, n_heads = 0, ffw = 0, n_layers = 0;
+  int32_t max_pos = 0;                   // rows of P (absolute positions)
+  int32_t position = 0;                  // SCONE_FGRAM_POS_ABSOLUTE or _ROTARY
   const uint16_t* weights = nullptr;     // borrowed, packed layout
+  const uint16_t* P = nullptr;           // [max_pos x d] inside weights; null for rotary
   int64_t batch = 0;                     // f-grams per batch
   int64_t cap_rows = 0;                  // workspace rows (tokens)
   int32_t* off = nullptr;                // [batch + 1] token offsets
@@ -91,12 +102,20 @@ __global__ void __launch_bounds__(1024)
   }
 }
 
-// X[off[f] + j] = T[tok[f * K + j]]: one warp per f-gram.
+__device__ __forceinline__ uint32_t add2(uint32_t a, uint32_t b) {
+  return pack2(lo_f(a) + lo_f(b), hi_f(a) + hi_f(b));
+}
+
+// The model input: X[off[f] + j] = bf16(T[tok[f * K + j]] + P[j]) (fp32 sum,
+// rounded to nearest even), or T's row alone when P is null; one warp per
+// f-gram. Position j counts from the f-gram's first token; j < K <= max_pos
+// is checked on the host, and rows past a length outside [1, K] are not
+// read (offsets_kernel counts such an f-gram as one token).
 __global__ void __launch_bounds__(256)
     gather_rows_kernel(const int32_t* __restrict__ tok, const uint8_t* __restrict__ len,
                        const int32_t* __restrict__ off, int64_t n, int32_t K,
                        const uint16_t* __restrict__ T, int32_t vocab, int32_t d,
-                       uint16_t* __restrict__ X, int* status) {
+                       const uint16_t* __restrict__ P, uint16_t* __restrict__ X, int* status) {
   const int lane = threadIdx.x & 31;
   const int64_t f = (int64_t)blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
   if (f >= n) return;
@@ -111,7 +130,15 @@ __global__ void __launch_bounds__(256)
       continue;
     }
     const uint4* src = reinterpret_cast<const uint4*>(T + (int64_t)t * d);
-    for (int c = lane; c < chunks; c += 32) dst[c] = __ldg(src + c);
+    if (!P) {
+      for (int c = lane; c < chunks; c += 32) dst[c] = __ldg(src + c);
+      continue;
+    }
+    const uint4* pos = reinterpret_cast<const uint4*>(P + (int64_t)j * d);
+    for (int c = lane; c < chunks; c += 32) {
+      const uint4 a = __ldg(src + c), b = __ldg(pos + c);
+      dst[c] = make_uint4(add2(a.x, b.x), add2(a.y, b.y), add2(a.z, b.z), add2(a.w, b.w));
+    }
   }
 }
 
@@ -192,8 +219,8 @@ struct Lanes {
 // Causal attention of one (f-gram, head) per warp over at most KMAX
 // positions. Lane l holds dims C*l .. C*l+C-1 of the head's first half and the
 // same offsets of its second half (C = hd / 64), so each rotate-half pair of
-// the rotary embedding stays in one lane.
-template <int C, int KMAX>
+// the rotary embedding (applied when ROTARY) stays in one lane.
+template <int C, int KMAX, bool ROTARY>
 __global__ void __launch_bounds__(256)
     attention_kernel(const uint16_t* __restrict__ QKV, const int32_t* __restrict__ off, int64_t n,
                      int32_t d, int32_t H, uint16_t* __restrict__ O) {
@@ -209,7 +236,7 @@ __global__ void __launch_bounds__(256)
   float theta[C];
 #pragma unroll
   for (int e = 0; e < C; ++e)
-    theta[e] = powf(10000.f, -2.f * (float)(C * lane + e) / (float)hd);
+    theta[e] = ROTARY ? powf(10000.f, -2.f * (float)(C * lane + e) / (float)hd) : 0.f;
 #pragma unroll
   for (int j = 0; j < KMAX; ++j) {
     if (j >= nl) break;
@@ -229,7 +256,7 @@ __global__ void __launch_bounds__(256)
     }
     // rotary embedding at position j: (a, b) -> (a cos - b sin, b cos + a sin)
 #pragma unroll
-    for (int e = 0; e < C; ++e) {
+    for (int e = 0; e < (ROTARY ? C : 0); ++e) {
       float s, c;
       sincosf((float)j * theta[e], &s, &c);
       const float qa = q[j][e], qb = q[j][C + e], ka = k[j][e], kb = k[j][C + e];
@@ -296,24 +323,37 @@ bool ln(int d, const uint16_t* X, uint16_t* Y, int64_t rows, const int32_t* off,
   }
 }
 
-template <int KMAX>
+template <int KMAX, bool ROTARY>
 bool attn_k(int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d, int H,
             uint16_t* O, cudaStream_t s) {
   const unsigned grid = (unsigned)((n * H + kRowsPerBlock - 1) / kRowsPerBlock);
   switch (hd) {
-    case 64: attention_kernel<1, KMAX><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
-    case 128: attention_kernel<2, KMAX><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
-    case 256: attention_kernel<4, KMAX><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O); return true;
+    case 64:
+      attention_kernel<1, KMAX, ROTARY><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O);
+      return true;
+    case 128:
+      attention_kernel<2, KMAX, ROTARY><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O);
+      return true;
+    case 256:
+      attention_kernel<4, KMAX, ROTARY><<<grid, 256, 0, s>>>(QKV, off, n, d, H, O);
+      return true;
     default: return false;
   }
 }
 
 // Positions held in registers: the smallest of 3, 5, 8 that covers K.
-bool attn(int K, int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d, int H,
-          uint16_t* O, cudaStream_t s) {
-  if (K <= 3) return attn_k<3>(hd, QKV, off, n, d, H, O, s);
-  if (K <= 5) return attn_k<5>(hd, QKV, off, n, d, H, O, s);
-  return attn_k<8>(hd, QKV, off, n, d, H, O, s);
+template <bool ROTARY>
+bool attn_r(int K, int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d, int H,
+            uint16_t* O, cudaStream_t s) {
+  if (K <= 3) return attn_k<3, ROTARY>(hd, QKV, off, n, d, H, O, s);
+  if (K <= 5) return attn_k<5, ROTARY>(hd, QKV, off, n, d, H, O, s);
+  return attn_k<8, ROTARY>(hd, QKV, off, n, d, H, O, s);
+}
+
+bool attn(bool rotary, int K, int hd, const uint16_t* QKV, const int32_t* off, int64_t n, int d,
+          int H, uint16_t* O, cudaStream_t s) {
+  return rotary ? attn_r<true>(K, hd, QKV, off, n, d, H, O, s)
+                : attn_r<false>(K, hd, QKV, off, n, d, H, O, s);
 }
 
 bool ensure_rows(scone_fgram_model* m, int64_t rows) {
@@ -342,13 +382,17 @@ bool ensure_rows(scone_fgram_model* m, int64_t rows) {
 using namespace scone;
 
 extern "C" int scone_fgram_model_create(int32_t d, int32_t n_heads, int32_t ffw, int32_t n_layers,
+                                        int32_t max_pos, int32_t position,
                                         const scone_bf16* weights, int64_t batch,
                                         scone_fgram_model** out) {
   if (!out) return SCONE_ERR_INVALID_ARG;
   *out = nullptr;
+  const bool absolute = position == SCONE_FGRAM_POS_ABSOLUTE;
+  if (!absolute && position != SCONE_FGRAM_POS_ROTARY) return SCONE_ERR_INVALID_ARG;
   if (d <= 0 || d % 256 || d / 256 > 16 || (d / 256) & (d / 256 - 1) || n_heads <= 0 ||
-      d % n_heads || ffw <= 0 || ffw % 128 || n_layers < 0 || (n_layers > 0 && !weights) ||
-      ((uintptr_t)weights & 15) || batch < 0)
+      d % n_heads || ffw <= 0 || ffw % 128 || n_layers < 0 ||
+      ((n_layers > 0 || absolute) && !weights) || ((uintptr_t)weights & 15) || batch < 0 ||
+      (absolute && (max_pos < 1 || max_pos > 8)))
     return SCONE_ERR_INVALID_ARG;
   const int hd = d / n_heads;
   if (hd != 64 && hd != 128 && hd != 256) return SCONE_ERR_UNSUPPORTED;
@@ -360,6 +404,12 @@ extern "C" int scone_fgram_model_create(int32_t d, int32_t n_heads, int32_t ffw,
   m->ffw = ffw;
   m->n_layers = n_layers;
   m->weights = weights;
+  m->position = position;
+  m->max_pos = absolute ? max_pos : 0;
+  // P follows the last layer in the packed buffer
+  const int64_t layer_elems = (int64_t)3 * d * d + (int64_t)d * d + (int64_t)2 * ffw * d +
+                              (int64_t)d * ffw;
+  m->P = absolute ? weights + n_layers * layer_elems : nullptr;
   m->batch = batch > 0 ? batch : 16384;
   if (cudaMalloc(&m->off, (size_t)(m->batch + 1) * sizeof(int32_t)) != cudaSuccess ||
       cudaMalloc(&m->status, sizeof(int)) != cudaSuccess ||
@@ -390,6 +440,8 @@ extern "C" int scone_fgram_precompute(scone_fgram_model* m, const int32_t* fgram
                                       const scone_bf16* T, int32_t vocab, scone_bf16* F,
                                       void* stream) {
   if (!m || n < 0 || K < 2 || K > 8 || vocab < 1) return SCONE_ERR_INVALID_ARG;
+  // every position of an f-gram needs a row of P
+  if (m->position == SCONE_FGRAM_POS_ABSOLUTE && K > m->max_pos) return SCONE_ERR_INVALID_ARG;
   if (n == 0) return SCONE_OK;
   if (!fgram_tok || !fgram_len || !T || !F || ((uintptr_t)T & 15) || ((uintptr_t)F & 15) ||
       ((uintptr_t)fgram_tok & 3))
@@ -411,7 +463,7 @@ extern "C" int scone_fgram_precompute(scone_fgram_model* m, const int32_t* fgram
     if (!ensure_rows(m, rows)) return SCONE_ERR_NOMEM;
     const unsigned gw = (unsigned)((nb + kRowsPerBlock - 1) / kRowsPerBlock);
     gather_rows_kernel<<<gw, 256, 0, s>>>(fgram_tok + f0 * K, fgram_len + f0, m->off, nb, K, T,
-                                          vocab, d, m->X, m->status);
+                                          vocab, d, m->P, m->X, m->status);
     for (int l = 0; l < m->n_layers; ++l) {
       const uint16_t* w = m->weights + l * layer_elems;
       const uint16_t* wqkv = w;
@@ -423,7 +475,9 @@ extern "C" int scone_fgram_precompute(scone_fgram_model* m, const int32_t* fgram
       if ((rc = gemm_bf16(m->Xn, wqkv, nullptr, m->QKV, rows, 3 * d, d, GEMM_EPI_STORE,
                           m->status, s)))
         return rc;
-      if (!attn(K, d / H, m->QKV, m->off, nb, d, H, m->Xn, s)) return SCONE_ERR_UNSUPPORTED;
+      if (!attn(m->position == SCONE_FGRAM_POS_ROTARY, K, d / H, m->QKV, m->off, nb, d, H,
+                m->Xn, s))
+        return SCONE_ERR_UNSUPPORTED;
       if ((rc = gemm_bf16(m->Xn, wo, m->X, m->X, rows, d, d, GEMM_EPI_RESIDUAL, m->status, s)))
         return rc;
       if (!ln(d, m->X, m->Xn, rows, nullptr, s)) return SCONE_ERR_UNSUPPORTED;

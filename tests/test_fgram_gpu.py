@@ -1,5 +1,6 @@
 """Precomputing F with the f-gram model on the GPU against the float64 oracle
-(GPU).
+(GPU). The model takes absolute position embeddings (Appendix F), and the
+rotary option is checked against the oracle's rotary scheme.
 
 The oracle rounds to bf16 at the points where the GPU stores bf16 (residual
 stream, layer-norm outputs, q/k/v, attention output, MLP activation, F), so
@@ -12,6 +13,8 @@ f-grams for each of K = 2, 5, 8): max |diff| 0.031 (one bf16 unit at |F| near
 exact float64 as the emulating oracle is (both about 0.0038 mean). Bound used
 here: max |diff| <= 0.08, row mean <= 6e-3, more than 75% of entries equal.
 """
+
+import dataclasses
 
 import numpy as np
 import pytest
@@ -35,6 +38,11 @@ def tiny_model():
     w_d = torch.from_numpy(packed.view(np.int16)).to(DEV)
     T_d = torch.from_numpy(T.view(np.int16)).to(DEV)
     return packed, W, T, w_d, T_d
+
+
+def tiny_dev_model(w_d, **kw):
+    return scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d,
+                            max_pos=TINY.max_pos, **kw)
 
 
 def fgram_list(n, K, seed):
@@ -66,7 +74,7 @@ def check(got_bits, tok, ln, W, T):
 
 def test_matches_oracle_all_lengths(tiny_model):
     packed, W, T, w_d, T_d = tiny_model
-    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
+    model = tiny_dev_model(w_d)
     for K in (2, 5, 8):
         tok, ln = fgram_list(150, K, seed=K)
         check(run(model, tok, ln, T_d), tok, ln, W, T)
@@ -78,8 +86,8 @@ def test_batches_equal_one_batch(tiny_model):
     ragged ends) gives the same bytes as one batch."""
     packed, W, T, w_d, T_d = tiny_model
     tok, ln = fgram_list(700, 5, seed=11)
-    one = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
-    many = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d, batch=37)
+    one = tiny_dev_model(w_d)
+    many = tiny_dev_model(w_d, batch=37)
     a, b = run(one, tok, ln, T_d), run(many, tok, ln, T_d)
     assert np.array_equal(a, b)
     check(a[::7], tok[::7], ln[::7], W, T)
@@ -88,19 +96,42 @@ def test_batches_equal_one_batch(tiny_model):
 
 
 def test_zero_layers_is_layer_norm(tiny_model):
+    """No layers: F = LN(T[last] + P[n-1]) (the buffer holds only P)."""
     packed, W, T, w_d, T_d = tiny_model
-    m0 = synth.FgramModel("none", 99, TINY.d, TINY.n_heads, TINY.ffw, 0)
-    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, 0, w_d)
-    tok, ln = fgram_list(40, 3, seed=2)
+    m0 = synth.FgramModel("none", 99, TINY.d, TINY.n_heads, TINY.ffw, 0, max_pos=5)
+    p0 = synth.model_weights_cpu(m0)
+    p0_d = torch.from_numpy(p0.view(np.int16)).to(DEV)
+    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, 0, p0_d, max_pos=5)
+    tok, ln = fgram_list(40, 5, seed=2)
     got = fm.bf16_to_f64(run(model, tok, ln, T_d))
-    want = fm.precompute(tok, ln, T, fm.Weights(np.zeros(0, np.uint16), m0), emulate_bf16=True)
+    want = fm.precompute(tok, ln, T, fm.Weights(p0, m0), emulate_bf16=True)
     assert np.abs(got - want).max() <= 2 ** -7 * 4          # one bf16 rounding of |F| <= ~4
+    assert (got == want).mean() > 0.95
+    # a list longer than the model's positions is refused before any device work
+    tok8, ln8 = fgram_list(10, 8, seed=4)
+    with pytest.raises(scone.SconeError) as e:
+        run(model, tok8, ln8, T_d)
+    assert e.value.code == scone.SCONE_ERR_INVALID_ARG
+    model.close()
+
+
+def test_rotary_option_matches_rotary_oracle(tiny_model):
+    """The non-default rotary scheme (no P in the buffer) against the oracle's."""
+    mr = dataclasses.replace(TINY, name="tiny_rotary", position="rotary")
+    pr = synth.model_weights_cpu(mr)
+    pr_d = torch.from_numpy(pr.view(np.int16)).to(DEV)
+    _, _, T, _, T_d = tiny_model
+    model = scone.FgramModel(mr.d, mr.n_heads, mr.ffw, mr.n_layers, pr_d,
+                             position=scone.SCONE_FGRAM_POS_ROTARY)
+    for K in (3, 8):
+        tok, ln = fgram_list(100, K, seed=20 + K)
+        check(run(model, tok, ln, T_d), tok, ln, fm.Weights(pr, mr), T)
     model.close()
 
 
 def test_errors(tiny_model):
     packed, W, T, w_d, T_d = tiny_model
-    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
+    model = tiny_dev_model(w_d)
     tok, ln = fgram_list(20, 3, seed=3)
     tok[4, 1] = VOCAB + 3
     with pytest.raises(scone.SconeError) as e:
@@ -114,6 +145,8 @@ def test_errors(tiny_model):
     model.close()
     with pytest.raises(scone.SconeError):
         scone.FgramModel(200, 4, 512, 2, w_d)                 # d not a multiple of 256
+    with pytest.raises(scone.SconeError):
+        scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d, max_pos=9)
 
 
 def test_discover_precompute_embed_pipeline(tiny_model):
@@ -126,7 +159,7 @@ def test_discover_precompute_embed_pipeline(tiny_model):
                                                 2000, 3)
     n = fl.shape[0]
     assert n > 100
-    model = scone.FgramModel(TINY.d, TINY.n_heads, TINY.ffw, TINY.n_layers, w_d)
+    model = tiny_dev_model(w_d)
     F = torch.empty((n, TINY.d), dtype=torch.int16, device=DEV)
     scone.scone_fgram_precompute(model, ft.contiguous(), fl.contiguous(), T_d, F)
     table = scone.scone_table_build(ft.cpu().numpy(), fl.cpu().numpy(), 3, VOCAB, TINY.d, F, T_d)
