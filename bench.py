@@ -61,6 +61,17 @@ def workload(name):
         # the offloaded-decode law with 2e6 f-grams (8 GB of host rows) for ncu captures
         return synth.WORKLOADS["offload_decode"].scaled(
             "decode_profile", quotas=((2, 1_200_000), (3, 800_000)))
+    if name == "large_hbm_profile":
+        # large_hbm's law (K = 3, d = 2048, Zipf(1.1), 64 x 4096 batches cut to 16) with
+        # 7.5e5 f-grams: F 3.1 GB + T 0.4 GB on the device, for counter captures
+        return synth.WORKLOADS["large_hbm"].scaled("large_hbm_profile", B=16,
+                                                   quotas=((2, 450_000), (3, 300_000)))
+    if name == "stress_profile":
+        # stress_k5's law (K = 5, d = 1536, phrases injected) with 8 x 8192 tokens and
+        # 1e6 f-grams in the same length split: F 3.1 GB + T 0.3 GB on the device
+        return synth.WORKLOADS["stress_k5"].scaled(
+            "stress_profile", B=8, quotas=((2, 333_333), (3, 333_333), (4, 166_667),
+                                           (5, 166_667)))
     if name == "offload_decode_first_seen":
         # the offloaded decode with F's rows in first-seen order instead of by count
         return synth.WORKLOADS["offload_decode"].scaled("offload_decode_first_seen",
@@ -171,18 +182,24 @@ def kernel_source_hash(files=EMBED_SOURCES) -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str, kernel: str = "embed_kernel", files=EMBED_SOURCES):
+def profiled_traffic(workload: str, kernel: str = "embed_kernel", files=EMBED_SOURCES,
+                     with_note: bool = False):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel sources; else None."""
+    on the current kernel sources; else None. With ``with_note``, also the
+    summary's one-line note on how the figure was obtained (a capture of a
+    smaller case scaled to a full launch, for instance)."""
     p = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
     if not os.path.exists(p):
-        return None
+        return (None, None) if with_note else None
     txt = open(p).read()
     m = re.search(r"dram_bytes_per_launch:\s*(\d+)", txt)
     s = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", txt)
-    if not m or not s or s.group(1) != kernel_source_hash(files):
-        return None
-    return int(m.group(1))
+    n = re.search(r"traffic_note:\s*([^\n]+)", txt)
+    ok = bool(m and s and s.group(1) == kernel_source_hash(files))
+    val = int(m.group(1)) if ok else None
+    if with_note:
+        return val, (n.group(1).strip() if (ok and n) else None)
+    return val
 
 
 def algorithmic_bytes_per_token(K: int, d: int) -> int:
@@ -354,6 +371,7 @@ def bench_prefill(args, world, rank, local):
             "unit": "GB/s",
             "frac": achieved / hbm,
             "traffic": profiled_traffic(w.name),
+            "traffic_note": profiled_traffic(w.name, with_note=True)[1],
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
             "algorithmic_bytes_per_launch": bytes_launch,
             "kernel": "embed_bulk_kernel (fused match + TMA bulk gather)" if args.copy == "bulk"
@@ -530,6 +548,50 @@ def host_link_bandwidth(dev, table, F_rows: int, d: int, zero_copy: bool = True)
             "d2h_copy_gbs": best_d2h}
 
 
+def decode_row_ceiling(table, new_d, rows, host_bytes, d):
+    """What the host link gives for the rows the decode steps select, without
+    the steps' dependent match: every step's rows gathered in one launch
+    (best of 5), and gathered one step per launch in a CUDA graph (best of 5
+    replays; the per-step time left to the match is the decode step's time
+    minus this one)."""
+    import torch
+
+    import paper_2502_01637_gb300 as scone
+
+    steps, S = rows.shape
+    big = torch.empty((steps * S, d), dtype=torch.int16, device=new_d.device)
+    one = torch.empty((S, d), dtype=torch.int16, device=new_d.device)
+    flat_tok, flat_row = new_d.reshape(-1).contiguous(), rows.reshape(-1).contiguous()
+
+    def best(fn, n=5):
+        t = []
+        for _ in range(n):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            t.append(a.elapsed_time(b))
+        return min(t)
+
+    scone.scone_embed_gather(table, flat_tok, flat_row, big)
+    all_ms = best(lambda: scone.scone_embed_gather(table, flat_tok, flat_row, big))
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for k in range(steps):
+            scone.scone_embed_gather(table, new_d[k], rows[k], one)
+    g.replay()
+    step_ms = best(g.replay) / steps
+    scone.scone_status(table)
+    del big, g
+    return {"all_steps_one_launch_gbs": host_bytes / (all_ms * 1e-3) / 1e9,
+            "per_step_gather_us": step_ms * 1e3,
+            "per_step_gather_gbs": host_bytes / steps / (step_ms * 1e-3) / 1e9,
+            "what": "the host rows the decode selects, gathered by gather_kernel without "
+                    "the match: all steps in one launch, and one launch per step (graph)"}
+
+
 def bench_decode(args, world, rank, local):
     import torch
 
@@ -555,15 +617,17 @@ def bench_decode(args, world, rank, local):
     new_d = torch.from_numpy(new).to(dev)
     out = torch.empty((S, w.d), dtype=torch.int16, device=dev)
     lens = torch.empty((steps, S), dtype=torch.uint8, device=dev)
+    rows = torch.empty((steps, S), dtype=torch.int32, device=dev)
     # one eager pass: match lengths of every step (host bytes = matched rows)
     st = scone.scone_decode_create(table, hist, hl)
     for k in range(steps):
-        scone.scone_decode_step(st, new_d[k], out, None, lens[k])
+        scone.scone_decode_step(st, new_d[k], out, rows[k], lens[k])
     scone.scone_status(table)
     ln = lens.cpu().numpy()
     matched = int((ln >= 2).sum())
     hist_counts = np.bincount(ln.reshape(-1), minlength=w.K + 1)
     st.close()
+    step_rows = decode_row_ceiling(table, new_d, rows, matched * 2 * w.d, w.d)
     # timed: the 256-step loop captured once in a CUDA graph, replayed
     st = scone.scone_decode_create(table, hist, hl)
     for k in range(3):
@@ -649,6 +713,7 @@ def bench_decode(args, world, rank, local):
             "peak_source": "measured in this run: max(pinned 1 GiB H2D copy, zero-copy "
                            "streaming read by the gather kernel)",
             "host_link": link,
+            "decode_rows": step_rows,
             "host_bytes_per_step": host_bytes_step,
             "hbm_bytes_per_step": hbm_bytes_step,
             "kernel": "decode_kernel (one warp per sequence)",
@@ -1400,7 +1465,8 @@ def cpu_baseline_discover(w, tok, budget_s: float = 10.0):
 
 
 # ----------------------------------------------------------- reference arm
-PREFILL_WORKLOADS = ("tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile")
+PREFILL_WORKLOADS = ("tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
+                     "large_hbm_profile", "stress_profile")
 
 
 def bench_reference(args, world, rank):
@@ -1482,6 +1548,7 @@ def main():
     ap.add_argument("--impl", default="scone", choices=["scone", "reference"])
     ap.add_argument("--workload", default=None,
                     choices=["tiny", "prefill_1b", "large_hbm", "stress_k5", "prefill_profile",
+                             "large_hbm_profile", "stress_profile",
                              "offload_decode", "offload_decode_first_seen", "decode_profile",
                              "prescan", "discover", "discover_k5", "discover_profile",
                              "mixed_serving", "precompute", "gemm_profile", "store_decode"],
