@@ -189,9 +189,11 @@ int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
 enum scone_copy_mode {
   SCONE_COPY_AUTO = 0,       /* the library picks per call */
   SCONE_COPY_REGISTERS = 1,  /* 16-byte loads and streaming stores through registers */
-  SCONE_COPY_BULK = 2        /* cp.async.bulk (TMA) through a shared-memory ring; needs rows of a
+  SCONE_COPY_BULK = 2,       /* cp.async.bulk (TMA) through a shared-memory ring; needs rows of a
                                 multiple of 16 bytes, 16-byte aligned F, T and out, and F in
                                 device memory, else scone_embed returns SCONE_ERR_UNSUPPORTED */
+  SCONE_COPY_SPLIT = 3       /* register copies by warps that only copy, fed through a
+                                shared-memory ring by warps that only match */
 };
 
 int scone_table_set_copy_mode(scone_table* table, int32_t mode);

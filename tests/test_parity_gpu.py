@@ -377,3 +377,48 @@ def test_bulk_copy_refuses_ineligible_calls():
     scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_REGISTERS)
     out, row, ln = run_embed(table, case.tok, w.d, out_offset=1)
     assert_parity(case, out, row, ln)
+
+
+# ------------------------------------------- separate match and copy warps
+SPLIT_CASES = [
+    ("split_k3", 3, 32000, 256, 4, 512, ((2, 60000), (3, 40000)), 0.0),
+    ("split_k5_d1536", 5, 100000, 1536, 3, 1001, ((2, 9000), (3, 9000), (4, 4000), (5, 4000)),
+     0.05 / 6),
+    ("split_k5_fmt32", 5, 300000, 128, 3, 700, ((2, 5000), (3, 5000), (4, 5000), (5, 5000)), 0.05),
+    ("split_k8_fmt32", 8, 1 << 20, 64, 3, 700, tuple((n, 2000) for n in range(2, 9)), 0.05),
+    ("split_k7_fmt16", 7, 8192, 64, 2, 333, tuple((n, 2000) for n in range(2, 8)), 0.05),
+    ("split_one_row", 5, 1000, 2048, 1, 1, ((2, 10), (3, 10), (4, 10), (5, 10)), 0.0),
+    ("split_ragged_tail", 5, 100000, 1536, 1, 33 * 8 * 40 + 7,
+     ((2, 6000), (3, 6000), (4, 3000), (5, 3000)), 0.05 / 6),
+]
+
+
+@pytest.mark.parametrize("name,K,vocab,d,B,L,quotas,inject", SPLIT_CASES)
+def test_split_copy_parity(name, K, vocab, d, B, L, quotas, inject):
+    """SCONE_COPY_SPLIT (match warps hand row addresses to copy warps through
+    a shared-memory ring): bit-exact against the oracle, for both key
+    formats, ragged tile tails and a single-row batch."""
+    w = synth.Workload(name, 80 + K, vocab, 1.05, B, L, quotas, K, d, inject_p=inject,
+                       n_phrases=512 if inject else 0, phrase_len=(K, K + 2))
+    case = SmallCase(w)
+    table = case.build()
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_SPLIT)
+    for offset in (0, 1):                    # 16-byte and 2-byte copy widths
+        out, row, ln = run_embed(table, case.tok, d, out_offset=offset)
+        assert_parity(case, out, row, ln)
+    out2, _, _ = run_embed(table, case.tok, d, mode="fused_noaux")
+    assert np.array_equal(out, out2)
+    assert scone.scone_status(table) == 0
+
+
+def test_split_copy_error_positions_get_zero_rows():
+    w = TINY.scaled("split_bad", B=3, L=300, quotas=((2, 3000), (3, 2000)))
+    tok = synth.query_tokens(w)
+    tok[0, 3] = -1
+    tok[2, 299] = w.vocab + 5
+    case = SmallCase(w, tok=tok)
+    table = case.build()
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_SPLIT)
+    out, row, ln = run_embed(table, case.tok, w.d)
+    assert_parity(case, out, row, ln)
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
