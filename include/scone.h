@@ -459,6 +459,18 @@ int scone_rowstore_gather(scone_rowstore* store, const scone_table* table, const
                           const int32_t* row, int64_t n, scone_bf16* out, void* stream);
 int scone_rowstore_get_stats(const scone_rowstore* store, scone_rowstore_stats* out);
 int scone_rowstore_close(scone_rowstore* store);
+/*
+ * scone_rowstore_probe_reads — the storage device's own rate for this store:
+ * n_reads rows drawn uniformly (a counter hash of `seed`) from the store's
+ * file, read with the store's reader threads and I/O mode (O_DIRECT where the
+ * gather uses it) into host buffers that are then discarded; no GPU work and
+ * no cache involvement. *rows_per_s and *bytes_per_s receive the rates over
+ * the host's steady clock. The roofline of the storage tier (Sec. 4.3: F on
+ * solid-state drives, one read per missed row). Synchronous; a failed read
+ * returns SCONE_ERR_CUDA, a failed buffer allocation SCONE_ERR_NOMEM.
+ */
+int scone_rowstore_probe_reads(scone_rowstore* store, int64_t n_reads, uint64_t seed,
+                               double* rows_per_s, double* bytes_per_s);
 
 /*
  * Decode (Sec. 3.2: T stays on the accelerator "for decoding", F is looked

@@ -49,7 +49,8 @@ EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noal
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
            "scone_embed_varlen", "scone_rowstore_open", "scone_rowstore_gather",
-           "scone_rowstore_get_stats", "scone_rowstore_close", "scone_gemm_bf16",
+           "scone_rowstore_get_stats", "scone_rowstore_close", "scone_rowstore_probe_reads",
+           "scone_gemm_bf16",
            "scone_gemm_bf16_variant", "scone_fgram_model_create",
            "scone_fgram_model_destroy", "scone_fgram_precompute", "scone_fgram_discover",
            "scone_discover_create", "scone_discover_destroy", "scone_discover_set_table_slack",
@@ -129,6 +130,9 @@ def load_library():
     lib.scone_rowstore_gather.argtypes = [_vp, _vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_rowstore_get_stats.argtypes = [_vp, ctypes.POINTER(scone_rowstore_stats)]
     lib.scone_rowstore_close.argtypes = [_vp]
+    lib.scone_rowstore_probe_reads.argtypes = [_vp, _i64, ctypes.c_uint64,
+                                               ctypes.POINTER(ctypes.c_double),
+                                               ctypes.POINTER(ctypes.c_double)]
     lib.scone_gemm_bf16.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp]
     lib.scone_gemm_bf16_variant.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                                             _vp, _vp]
@@ -462,6 +466,15 @@ def scone_rowstore_close(store: RowStore) -> None:
 
 def scone_rowstore_get_stats(store: RowStore) -> dict:
     return store.stats()
+
+
+def scone_rowstore_probe_reads(store: RowStore, n_reads: int, seed: int = 1) -> dict:
+    """Random-row read rate of the store's file with its own threads and I/O mode."""
+    rows, nbytes = ctypes.c_double(), ctypes.c_double()
+    _check(load_library().scone_rowstore_probe_reads(store.handle, n_reads, seed,
+                                                     ctypes.byref(rows), ctypes.byref(nbytes)),
+           "scone_rowstore_probe_reads")
+    return {"rows_per_s": rows.value, "bytes_per_s": nbytes.value}
 
 
 def scone_rowstore_gather(store: RowStore, table: Table, tok, row, out, stream=None) -> None:

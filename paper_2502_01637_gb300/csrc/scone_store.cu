@@ -20,6 +20,8 @@
 
 #include <algorithm>
 #include <atomic>
+#include <chrono>
+#include <cstdlib>
 #include <condition_variable>
 #include <cstring>
 #include <functional>
@@ -431,5 +433,31 @@ extern "C" int scone_rowstore_gather(scone_rowstore* st, const scone_table* tb,
     return SCONE_ERR_CUDA;
   st->stats.rows_read += nu;
   st->stats.bytes_read += nu * st->row_bytes;
+  return SCONE_OK;
+}
+
+extern "C" int scone_rowstore_probe_reads(scone_rowstore* st, int64_t n_reads, uint64_t seed,
+                                          double* rows_per_s, double* bytes_per_s) {
+  if (!st || n_reads < 1 || !rows_per_s || !bytes_per_s) return SCONE_ERR_INVALID_ARG;
+  // landing buffers, 4096-aligned for O_DIRECT; contents are discarded, so
+  // reads that share a buffer may overlap
+  const int64_t n_buf = n_reads < 256 ? n_reads : 256;
+  void* buf = nullptr;
+  if (posix_memalign(&buf, 4096, (size_t)(n_buf * st->row_bytes)) != 0) return SCONE_ERR_NOMEM;
+  std::vector<int64_t> rows((size_t)n_reads);
+  for (int64_t i = 0; i < n_reads; ++i)
+    rows[(size_t)i] = (int64_t)(host_fmix64(seed + (uint64_t)i * 0x9E3779B97F4A7C15ull) %
+                                (uint64_t)st->n_rows);
+  std::atomic<bool> io_ok(true);
+  const auto t0 = std::chrono::steady_clock::now();
+  st->pool->run(n_reads, [&](int64_t i) {
+    uint8_t* dst = static_cast<uint8_t*>(buf) + (i % n_buf) * st->row_bytes;
+    if (!read_row(st, rows[(size_t)i], dst)) io_ok = false;
+  });
+  const double sec = std::chrono::duration<double>(std::chrono::steady_clock::now() - t0).count();
+  free(buf);
+  if (!io_ok) return SCONE_ERR_CUDA;
+  *rows_per_s = (double)n_reads / sec;
+  *bytes_per_s = (double)n_reads * (double)st->row_bytes / sec;
   return SCONE_OK;
 }

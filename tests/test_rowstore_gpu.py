@@ -170,3 +170,20 @@ def test_long_keys_and_k8(tmp_path):
     assert (exp_len == 8).any()
     store.close()
     table.close()
+
+
+def test_probe_reads_reports_the_file_rate(case):
+    """The storage probe reads rows of the store's own file (no GPU work, no
+    cache change) and reports positive rates that agree with each other."""
+    store = scone.RowStore(case.path, W.n_fgrams, W.d, 64, threads=4)
+    before = store.stats()
+    r = scone.scone_rowstore_probe_reads(store, 2000, seed=3)
+    assert r["rows_per_s"] > 0
+    assert abs(r["bytes_per_s"] / r["rows_per_s"] - W.d * 2) < 1e-6 * W.d * 2
+    assert store.stats() == before                 # the gather statistics are untouched
+    out = gather(case, store, case.tok)            # the store still gathers exactly
+    o_out, _, _, _ = case.expected()
+    assert np.array_equal(out, o_out.reshape(out.shape))
+    with pytest.raises(scone.SconeError):
+        scone.scone_rowstore_probe_reads(store, 0)
+    store.close()
