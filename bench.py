@@ -269,7 +269,8 @@ def bench_prefill(args, world, rank, local):
     scone.scone_table_set_copy_mode(table, {"auto": scone.SCONE_COPY_AUTO,
                                             "registers": scone.SCONE_COPY_REGISTERS,
                                             "bulk": scone.SCONE_COPY_BULK,
-                                            "split": scone.SCONE_COPY_SPLIT}[args.copy])
+                                            "split": scone.SCONE_COPY_SPLIT,
+                                            "pipelined": scone.SCONE_COPY_PIPELINED}[args.copy])
     info = table.info()
     setup_s = time.time() - t0
     batches = [torch.from_numpy(b).to(dev) for b in batches_np]
@@ -1566,7 +1567,8 @@ def main():
     ap.add_argument("--no-extras", action="store_true",
                     help="without --workload: measure large_hbm only")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--copy", default="auto", choices=["auto", "registers", "bulk", "split"],
+    ap.add_argument("--copy", default="auto",
+                    choices=["auto", "registers", "bulk", "split", "pipelined"],
                     help="row copy method of the fused kernel (results are identical)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)

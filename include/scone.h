@@ -192,8 +192,11 @@ enum scone_copy_mode {
   SCONE_COPY_BULK = 2,       /* cp.async.bulk (TMA) through a shared-memory ring; needs rows of a
                                 multiple of 16 bytes, 16-byte aligned F, T and out, and F in
                                 device memory, else scone_embed returns SCONE_ERR_UNSUPPORTED */
-  SCONE_COPY_SPLIT = 3       /* register copies by warps that only copy, fed through a
+  SCONE_COPY_SPLIT = 3,      /* register copies by warps that only copy, fed through a
                                 shared-memory ring by warps that only match */
+  SCONE_COPY_PIPELINED = 4   /* register copies with the next tile's match interleaved into
+                                the current tile's copy; for 16-byte slots, K <= 5 and
+                                16-byte-aligned rows, else as SCONE_COPY_REGISTERS */
 };
 
 int scone_table_set_copy_mode(scone_table* table, int32_t mode);

@@ -37,6 +37,7 @@ SCONE_COPY_AUTO = 0
 SCONE_COPY_REGISTERS = 1
 SCONE_COPY_BULK = 2
 SCONE_COPY_SPLIT = 3
+SCONE_COPY_PIPELINED = 4
 SCONE_GEMM_STORE = 0
 SCONE_GEMM_RESIDUAL = 1
 SCONE_GEMM_SWIGLU = 2

@@ -258,6 +258,9 @@ extern "C" int scone_embed(const scone_table* tb, const int32_t* tok, int32_t B,
   if (tb->copy_mode == SCONE_COPY_SPLIT)
     return launch_embed_split(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
                               (cudaStream_t)stream);
+  if (tb->copy_mode == SCONE_COPY_PIPELINED && pipe_eligible(tb, out))
+    return launch_embed_pipe(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
+                             (cudaStream_t)stream);
   const int width = row_copy_width(tb->view, out);
   const EmbedFn fn = pick_embed(tb->fmt, tb->view.K, width);
   const int grid = copy_grid((const void*)fn, n);

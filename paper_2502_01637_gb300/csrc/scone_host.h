@@ -51,6 +51,12 @@ int launch_embed_bulk(const scone_table* tb, const int32_t* tok, int64_t n, int3
 int launch_embed_split(const scone_table* tb, const int32_t* tok, int64_t n, int32_t L,
                        uint8_t* out, int32_t* row, uint8_t* len, cudaStream_t stream);
 
+// Fused embed with the next tile's match interleaved into the copy
+// (SCONE_COPY_PIPELINED): eligibility (FMT16, K <= 5, 16-byte copies) and launch.
+bool pipe_eligible(const scone_table* tb, const void* out);
+int launch_embed_pipe(const scone_table* tb, const int32_t* tok, int64_t n, int32_t L,
+                      uint8_t* out, int32_t* row, uint8_t* len, cudaStream_t stream);
+
 // Widest copy unit (16, 8, 4 or 2 bytes) that the row size, T, F, the output
 // and `extra` (another base address or size, 0 if none) all allow.
 inline int row_copy_width(const TableView& t, const void* out, uintptr_t extra = 0) {

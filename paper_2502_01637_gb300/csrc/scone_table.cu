@@ -412,7 +412,7 @@ extern "C" int scone_table_set_probe_limit(scone_table* t, int64_t max_buckets) 
 }
 
 extern "C" int scone_table_set_copy_mode(scone_table* t, int32_t mode) {
-  if (!t || mode < SCONE_COPY_AUTO || mode > SCONE_COPY_SPLIT) return SCONE_ERR_INVALID_ARG;
+  if (!t || mode < SCONE_COPY_AUTO || mode > SCONE_COPY_PIPELINED) return SCONE_ERR_INVALID_ARG;
   t->copy_mode = mode;
   return SCONE_OK;
 }

@@ -393,16 +393,20 @@ SPLIT_CASES = [
 ]
 
 
+@pytest.mark.parametrize("mode", ["split", "pipelined"])
 @pytest.mark.parametrize("name,K,vocab,d,B,L,quotas,inject", SPLIT_CASES)
-def test_split_copy_parity(name, K, vocab, d, B, L, quotas, inject):
+def test_split_copy_parity(name, K, vocab, d, B, L, quotas, inject, mode):
     """SCONE_COPY_SPLIT (match warps hand row addresses to copy warps through
-    a shared-memory ring): bit-exact against the oracle, for both key
+    a shared-memory ring) and SCONE_COPY_PIPELINED (the next tile's match
+    interleaved into the current tile's copy; other key formats and widths
+    take the register kernel): bit-exact against the oracle, for both key
     formats, ragged tile tails and a single-row batch."""
     w = synth.Workload(name, 80 + K, vocab, 1.05, B, L, quotas, K, d, inject_p=inject,
                        n_phrases=512 if inject else 0, phrase_len=(K, K + 2))
     case = SmallCase(w)
     table = case.build()
-    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_SPLIT)
+    scone.scone_table_set_copy_mode(table, {"split": scone.SCONE_COPY_SPLIT,
+                                            "pipelined": scone.SCONE_COPY_PIPELINED}[mode])
     for offset in (0, 1):                    # 16-byte and 2-byte copy widths
         out, row, ln = run_embed(table, case.tok, d, out_offset=offset)
         assert_parity(case, out, row, ln)
@@ -411,14 +415,33 @@ def test_split_copy_parity(name, K, vocab, d, B, L, quotas, inject):
     assert scone.scone_status(table) == 0
 
 
-def test_split_copy_error_positions_get_zero_rows():
+@pytest.mark.parametrize("mode", [3, 4])          # SCONE_COPY_SPLIT, SCONE_COPY_PIPELINED
+def test_split_copy_error_positions_get_zero_rows(mode):
     w = TINY.scaled("split_bad", B=3, L=300, quotas=((2, 3000), (3, 2000)))
     tok = synth.query_tokens(w)
     tok[0, 3] = -1
     tok[2, 299] = w.vocab + 5
+    tok[1, 40] = w.vocab                       # also inside another position's window
     case = SmallCase(w, tok=tok)
     table = case.build()
-    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_SPLIT)
+    scone.scone_table_set_copy_mode(table, mode)
     out, row, ln = run_embed(table, case.tok, w.d)
     assert_parity(case, out, row, ln)
     assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+
+
+def test_pipelined_probe_limit_reports_and_zero_rows():
+    """With one bucket per lookup allowed, the stages report the probe-limit
+    error exactly where the register kernel does."""
+    w = TINY.scaled("pipe_probe", B=4, L=400, quotas=((2, 30000), (3, 20000)))
+    case = SmallCase(w)
+    table = case.build(load_factor=0.85)
+    scone.scone_table_set_probe_limit(table, 1)
+    ref = run_embed(table, case.tok, w.d)
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_PROBE_LIMIT
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_PIPELINED)
+    got = run_embed(table, case.tok, w.d)
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_PROBE_LIMIT
+    for a, b in zip(ref, got):
+        assert np.array_equal(a, b)
+    assert (ref[2] == 0).any()
