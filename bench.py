@@ -252,6 +252,8 @@ def bench_prefill(args, world, rank, local):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     w = workload(args.workload)
+    if getattr(args, "load_factor", None):
+        w = w.scaled(w.name, load_factor=args.load_factor)
     n_tok = w.B * w.L
     t0 = time.time()
     fg_tok, fg_len, used = synth.fgram_set(w)
@@ -1567,6 +1569,8 @@ def main():
     ap.add_argument("--no-extras", action="store_true",
                     help="without --workload: measure large_hbm only")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--load-factor", type=float, default=None,
+                    help="prefill workloads: the table's load factor (default: the workload's)")
     ap.add_argument("--copy", default="auto",
                     choices=["auto", "registers", "bulk", "split", "pipelined"],
                     help="row copy method of the fused kernel (results are identical)")
