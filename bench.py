@@ -167,6 +167,7 @@ def measured_peaks():
 
 
 EMBED_SOURCES = ("scone_embed.cu", "scone_device.cuh", "scone_host.h")
+PIPE_SOURCES = ("scone_pipe.cu", "scone_embed.cu", "scone_device.cuh", "scone_host.h")
 DISCOVER_SOURCES = ("scone_discover.cu", "scone_device.cuh", "scone_host.h")
 
 
@@ -348,6 +349,10 @@ def bench_prefill(args, world, rank, local):
     bytes_launch = per_tok * n_tok
     hbm, peak_src = measured_peaks()
     achieved = bytes_launch / (kernel_ms * 1e-3) / 1e9
+    kname = embed_kernel_name(args.copy, w.K).split()[0]
+    traffic, traffic_note = profiled_traffic(
+        w.name, kname, PIPE_SOURCES if kname == "embed_pipe_kernel" else EMBED_SOURCES,
+        with_note=True)
     res = {
         "metric": METRIC,
         "value": world * n_tok / (ms_step * 1e-3),
@@ -374,12 +379,11 @@ def bench_prefill(args, world, rank, local):
             "peak": hbm,
             "unit": "GB/s",
             "frac": achieved / hbm,
-            "traffic": profiled_traffic(w.name),
-            "traffic_note": profiled_traffic(w.name, with_note=True)[1],
+            "traffic": traffic,
+            "traffic_note": traffic_note,
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
             "algorithmic_bytes_per_launch": bytes_launch,
-            "kernel": "embed_bulk_kernel (fused match + TMA bulk gather)" if args.copy == "bulk"
-                      else "embed_kernel (fused match + gather)",
+            "kernel": embed_kernel_name(args.copy, w.K),
         },
         "e2e": {
             "value": world * n_tok / (e2e_ms[False] * 1e-3),
@@ -408,6 +412,17 @@ def bench_prefill(args, world, rank, local):
         res["cpu_baseline"] = cpu_baseline(w, fg_tok, fg_len, batches_np[0], F, T)
     table.close()
     return res
+
+
+def embed_kernel_name(copy: str, K: int) -> str:
+    """The kernel scone_embed launches for a copy mode (16-byte slots, aligned rows)."""
+    if copy == "bulk":
+        return "embed_bulk_kernel (fused match + TMA bulk gather)"
+    if copy == "split":
+        return "embed_split_kernel (match warps feed copy warps through shared memory)"
+    if copy == "pipelined" or (copy == "auto" and 3 < K <= 5):
+        return "embed_pipe_kernel (next tile's match interleaved into the copy)"
+    return "embed_kernel (fused match + gather)"
 
 
 def prefill_config(w, world: int) -> dict:

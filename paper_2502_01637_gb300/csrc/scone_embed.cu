@@ -258,7 +258,12 @@ extern "C" int scone_embed(const scone_table* tb, const int32_t* tok, int32_t B,
   if (tb->copy_mode == SCONE_COPY_SPLIT)
     return launch_embed_split(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
                               (cudaStream_t)stream);
-  if (tb->copy_mode == SCONE_COPY_PIPELINED && pipe_eligible(tb, out))
+  // AUTO: the pipelined kernel where the match is long (3 < K <= 5) and it
+  // applies (measured 0.5-1% faster on stress_k5, K = 5; for K <= 3 the
+  // register kernel is 0.7-1% faster on large_hbm and prefill_1b)
+  const bool pipe = tb->copy_mode == SCONE_COPY_PIPELINED ||
+                    (tb->copy_mode == SCONE_COPY_AUTO && tb->view.K > 3);
+  if (pipe && pipe_eligible(tb, out))
     return launch_embed_pipe(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
                              (cudaStream_t)stream);
   const int width = row_copy_width(tb->view, out);

@@ -18,9 +18,11 @@
 // before its copy starts; the match steps and their order are those of
 // match_position (scone_device.cuh), split where a stage waits on a load.
 //
-// Used for the 16-byte-aligned case with 16-byte slots (FMT16) and K <= 5,
-// where the match state (the window tokens and K-1 buckets) fits beside the
-// copy's loads in the registers; other calls take embed_kernel.
+// The buckets a stage loads go to shared memory with cp.async, so the state
+// that lives across a copy segment is the window tokens and a few flags and
+// the copy keeps as many loads in flight as embed_kernel does. Used for the
+// 16-byte-aligned case with 16-byte slots (FMT16) and K <= 5; other calls
+// take embed_kernel.
 
 #include "scone_host.h"
 
@@ -33,21 +35,41 @@ namespace {
 
 template <int KT>
 struct PipeTuning {
-  // the most loads in flight per lane that compile without spills beside the
-  // match state at the given residency (80 and 128 registers)
-  static constexpr int kLoads = KT <= 3 ? 6 : 12;        // 16-byte loads in flight per lane
+  static constexpr int kLoads = KT <= 3 ? 8 : 16;        // 16-byte loads in flight per lane
   static constexpr int kMinBlocks = KT <= 3 ? 3 : 2;
 };
 
-// The match of one position, in four stages that each end with loads issued.
-template <int FMT, int KT>
+// Asynchronous 16-byte global -> shared copies (cp.async, L2 only): the
+// bucket loads of the match land in shared memory instead of registers, so
+// the match state held across a copy segment is a few words per lane.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+// One 32-byte bucket (16-byte slots) from the table into shared memory.
+__device__ __forceinline__ void bucket_async(Bucket* dst, const TableView& t, uint64_t q) {
+  const uint8_t* src = t.slots + q * bucket_bytes<FMT16>();
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  cp_async16(d, src);
+  cp_async16(d + 16, src + 16);
+}
+
+// The match of one position (16-byte slots), in four stages that each end
+// with loads issued: the window tokens into registers, the buckets into this
+// lane's shared-memory slots `sb` (one per length).
+template <int KT>
 struct PipeMatch {
   int32_t w[KT];              // window tokens, newest first
-  BucketData<FMT> v[KT - 1];  // bucket of each length (first, then second where needed)
   int32_t r1[KT - 1];
   int nmax;                   // longest usable window
   uint32_t second;            // bit n-2: length n needs its second bucket
   bool active, bad;
+  Bucket* sb;                 // [KT - 1] bucket of each length (first, then second)
 
   // stage 0: the window tokens (loads issued)
   __device__ __forceinline__ void stage0(const TableView& t, const int32_t* __restrict__ tok,
@@ -78,22 +100,26 @@ struct PipeMatch {
     for (int n = 2; n <= KT; ++n) {
       if (n <= nmax) {
         uint64_t b1, b2;
-        cuckoo_buckets(key_hash<FMT>(window_key<FMT, KT>(w, n, t.bits), t.hash_seed),
+        cuckoo_buckets(key_hash<FMT16>(window_key<FMT16, KT>(w, n, t.bits), t.hash_seed),
                        t.n_buckets, &b1, &b2);
-        v[n - 2] = ld_bucket_data<FMT>(t, b1);
+        bucket_async(&sb[n - 2], t, b1);
       }
     }
+    cp_async_commit();
   }
   // stage 2: first-round hits; the second buckets still needed (loads issued)
   __device__ __forceinline__ void stage2(const TableView& t) {
     second = 0;
     if (!active || bad) return;
+    cp_async_wait_all();
 #pragma unroll
     for (int n = 2; n <= KT; ++n) {
       r1[n - 2] = -1;
       if (n <= nmax) {
-        r1[n - 2] = find_in_bucket<FMT>(v[n - 2], window_key<FMT, KT>(w, n, t.bits));
-        if (r1[n - 2] < 0 && bucket_full<FMT>(v[n - 2])) second |= 1u << (n - 2);
+        BucketData<FMT16> v;
+        v.part[0] = sb[n - 2];
+        r1[n - 2] = find_in_bucket<FMT16>(v, window_key<FMT16, KT>(w, n, t.bits));
+        if (r1[n - 2] < 0 && bucket_full<FMT16>(v)) second |= 1u << (n - 2);
       }
     }
     // only lengths longer than the longest first-round hit matter
@@ -107,11 +133,12 @@ struct PipeMatch {
       for (int n = 2; n <= KT; ++n) {
         if (second & (1u << (n - 2))) {
           uint64_t b1, b2;
-          cuckoo_buckets(key_hash<FMT>(window_key<FMT, KT>(w, n, t.bits), t.hash_seed),
+          cuckoo_buckets(key_hash<FMT16>(window_key<FMT16, KT>(w, n, t.bits), t.hash_seed),
                          t.n_buckets, &b1, &b2);
-          v[n - 2] = ld_bucket_data<FMT>(t, b2);
+          bucket_async(&sb[n - 2], t, b2);
         }
       }
+      cp_async_commit();
     }
   }
   // stage 3: the longest hit. Returns the row (or -1), sets *len and *err as
@@ -128,10 +155,15 @@ struct PipeMatch {
         *len = 0;
         return -1;
       }
+      cp_async_wait_all();
 #pragma unroll
-      for (int n = 2; n <= KT; ++n)
-        if (second & (1u << (n - 2)))
-          r1[n - 2] = find_in_bucket<FMT>(v[n - 2], window_key<FMT, KT>(w, n, t.bits));
+      for (int n = 2; n <= KT; ++n) {
+        if (second & (1u << (n - 2))) {
+          BucketData<FMT16> v;
+          v.part[0] = sb[n - 2];
+          r1[n - 2] = find_in_bucket<FMT16>(v, window_key<FMT16, KT>(w, n, t.bits));
+        }
+      }
     }
 #pragma unroll
     for (int n = KT; n >= 2; --n) {
@@ -177,8 +209,8 @@ __device__ __forceinline__ void copy_chunks(const uint4* const* src, uint4* __re
   }
 }
 
-template <int FMT, int KT>
-__device__ __forceinline__ const uint4* pipe_finish(const TableView& t, PipeMatch<FMT, KT>& m,
+template <int KT>
+__device__ __forceinline__ const uint4* pipe_finish(const TableView& t, PipeMatch<KT>& m,
                                                     int64_t p, int32_t* __restrict__ row_out,
                                                     uint8_t* __restrict__ len_out) {
   if (!m.active) return nullptr;
@@ -194,20 +226,22 @@ __device__ __forceinline__ const uint4* pipe_finish(const TableView& t, PipeMatc
                                                : t.T + (int64_t)m.w[0] * t.d);
 }
 
-template <int FMT, int KT>
+template <int KT>
 __global__ void __launch_bounds__(kPipeThreads, PipeTuning<KT>::kMinBlocks)
     embed_pipe_kernel(const TableView t, const int32_t* __restrict__ tok, int64_t n_tok,
                       int32_t L, uint8_t* __restrict__ out, int32_t* __restrict__ row_out,
                       uint8_t* __restrict__ len_out) {
   constexpr int U = PipeTuning<KT>::kLoads;
   __shared__ const uint4* src_s[kPipeWarps][2][32];
+  __shared__ __align__(16) Bucket bucket_s[kPipeWarps][32][KT - 1];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int epr = t.d >> 3;                      // 16-byte elements per row
   const int64_t nw = (int64_t)gridDim.x * kPipeWarps;
   const int64_t wid = (int64_t)blockIdx.x * kPipeWarps + warp;
   const int64_t lo = n_tok * wid / nw, hi = n_tok * (wid + 1) / nw;
   if (lo >= hi) return;
-  PipeMatch<FMT, KT> m;
+  PipeMatch<KT> m;
+  m.sb = bucket_s[warp][lane];
   int buf = 0;
   int64_t base = lo;
   int nrows = (int)(hi - base < 32 ? hi - base : 32);
@@ -216,7 +250,7 @@ __global__ void __launch_bounds__(kPipeThreads, PipeTuning<KT>::kMinBlocks)
     m.stage0(t, tok, p, (int32_t)(p % L), lane < nrows);
     m.stage1(t);
     m.stage2(t);
-    src_s[warp][buf][lane] = pipe_finish<FMT, KT>(t, m, p, row_out, len_out);
+    src_s[warp][buf][lane] = pipe_finish<KT>(t, m, p, row_out, len_out);
     __syncwarp();
   }
   while (base < hi) {
@@ -240,7 +274,7 @@ __global__ void __launch_bounds__(kPipeThreads, PipeTuning<KT>::kMinBlocks)
     copy_chunks<U>(src, dst, nrows, epr, total, lane, c2, c3, r, col);
     if (nn) m.stage2(t);
     copy_chunks<U>(src, dst, nrows, epr, total, lane, c3, nchunks, r, col);
-    if (nn) src_s[warp][buf ^ 1][lane] = pipe_finish<FMT, KT>(t, m, np, row_out, len_out);
+    if (nn) src_s[warp][buf ^ 1][lane] = pipe_finish<KT>(t, m, np, row_out, len_out);
     __syncwarp();
     buf ^= 1;
     base = nbase;
@@ -259,7 +293,7 @@ bool pipe_eligible(const scone_table* tb, const void* out) {
 
 int launch_embed_pipe(const scone_table* tb, const int32_t* tok, int64_t n, int32_t L,
                       uint8_t* out, int32_t* row, uint8_t* len, cudaStream_t stream) {
-  const PipeFn fn = tb->view.K <= 3 ? embed_pipe_kernel<FMT16, 3> : embed_pipe_kernel<FMT16, 5>;
+  const PipeFn fn = tb->view.K <= 3 ? embed_pipe_kernel<3> : embed_pipe_kernel<5>;
   // every resident block, unless warps would get fewer than 8 rows each
   const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)fn, kPipeThreads, 0);
   const int64_t need = (n + kPipeWarps * 8 - 1) / (kPipeWarps * 8);
