@@ -1289,6 +1289,25 @@ def bench_gemm(args, world, rank, local):
         b.record(stream)
     torch.cuda.synchronize()
     ms1 = statistics.mean(a.elapsed_time(b) for a, b in ev1)
+    # context: cuBLAS (torch.matmul, bf16, plain store) on the same shape, and on
+    # the 8192^3 shape the measured peak is quoted on
+    def cublas_tflops(m, n, k, reps=10):
+        a = torch.randn((m, k), dtype=torch.bfloat16, device=dev)
+        b = torch.randn((n, k), dtype=torch.bfloat16, device=dev)
+        for _ in range(3):
+            torch.matmul(a, b.t())
+        e = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+             for _ in range(reps)]
+        for x, y in e:
+            x.record(stream)
+            torch.matmul(a, b.t())
+            y.record(stream)
+        torch.cuda.synchronize()
+        best = min(x.elapsed_time(y) for x, y in e)
+        return 2.0 * m * n * k / (best * 1e-3) / 1e12
+
+    cublas_same = cublas_tflops(M, N, K)
+    cublas_8192 = cublas_tflops(8192, 8192, 8192)
     peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) \
         if os.path.exists(os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
     peak = float(peaks.get("bf16_tflops", 1900.0))
@@ -1312,6 +1331,10 @@ def bench_gemm(args, world, rank, local):
         "gpu_launches": args.steps, "clocks": clocks.summary(),
         "variants": {"sm_pairs_256x256 (default)": tf,
                      "one_sm_128x256": flops / (ms1 * 1e-3) / 1e12},
+        "cublas_context": {"same_shape_plain_store_tflops": cublas_same,
+                           "shape_8192_cubed_tflops": cublas_8192,
+                           "what": "torch.matmul bf16, best of 10, CUDA events; context for "
+                                   "the roofline, whose peak stays MEASURED_PEAKS.json's"},
     }
 
 
