@@ -17,7 +17,8 @@
 //   * warps 2..5 read the other accumulator back with tcgen05.ld (warp w owns
 //     tensor-memory lanes 32 (w % 4) .. + 31, i.e. rows) and apply the
 //     epilogue: store, add a residual, or SwiGLU of interleaved gate/up
-//     column pairs; then they release the accumulator.
+//     column pairs; they stage the bf16 results in swizzled shared-memory
+//     boxes that TMA stores to C, and release the accumulator.
 // So the epilogue of one tile overlaps the main loop of the next.
 // Every mbarrier wait is bounded (kGemmSpin polls); past it the CTA records
 // SCONE_ERR_CUDA, stops issuing, waits for what it issued, frees its tensor
@@ -53,7 +54,8 @@ constexpr uint32_t kStageB = kBN * kBK * 2;   // 32 KB
 constexpr uint32_t kStageBytes = kStageA + kStageB;
 constexpr uint32_t kTmemCols = 2 * kBN;       // two fp32 accumulators of 256 columns x 128 lanes
 constexpr uint32_t kGemmSpin = 1u << 22;   // polls; each try_wait may also suspend briefly
-constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + 1024 /* align */ + 256 /* barriers */;
+constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + 1024 /* align */ + 256 /* barriers */ +
+                             (size_t)kEpiWarps * 2 * 32 * 128 /* epilogue boxes */;
 
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   return mbar_wait_bounded(bar, parity, kGemmSpin);
@@ -183,6 +185,121 @@ __device__ __forceinline__ void store_chunk(const float (&v)[32], int row, int c
   }
 }
 
+// The epilogue writes C through shared memory and TMA: each epilogue warp
+// stages its 32 rows of 64 output columns (128 bytes a row: two 32-column
+// chunks of the accumulator, or four under SwiGLU, whose output is half as
+// wide) as a box [32 rows x 128 bytes] with the 128-byte swizzle (16-byte
+// unit u of row r at unit u ^ (r % 8), so the lanes' row writes spread over
+// the banks), and one lane stores the box with cp.async.bulk.tensor. C is
+// then written in whole 128-byte lines instead of 32 scattered pieces per
+// warp store. Two boxes per warp alternate; a box is rewritten only after
+// the store that read it has finished reading (bulk wait_group.read 1).
+// Rows past M are clipped by the store.
+constexpr uint32_t kEpiBox = 32 * 128;                        // bytes per staged box
+constexpr uint32_t kEpiSmem = kEpiWarps * 2 * kEpiBox;        // 32 KB per CTA
+constexpr int kEpiBoxCols = 64;                               // bf16 output columns per box
+template <int EPI>
+__host__ __device__ constexpr int epi_chunks_per_box() {
+  return EPI == GEMM_EPI_SWIGLU ? 4 : 2;
+}
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(x), "r"(y), "r"(src)
+      : "memory");
+}
+__device__ __forceinline__ void epi_commit() { asm volatile("cp.async.bulk.commit_group;"); }
+__device__ __forceinline__ void epi_wait_read_1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void epi_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// This lane's row of one chunk (accumulator columns col .. col+31) as the
+// epilogue's bf16 output: 16-byte units u0 .. u0+3 (u0 .. u0+1 under SwiGLU)
+// of the lane's swizzled box row. Rows past M read no residual (the store
+// clips them).
+template <int EPI>
+__device__ __forceinline__ void stage_chunk(const float (&v)[32], int row, int M, int col,
+                                            const uint16_t* __restrict__ R, int ldc,
+                                            uint8_t* box_row, int u0, int lane) {
+  const int sw = lane & 7;
+  auto put = [&](int u, uint4 w) {
+    *reinterpret_cast<uint4*>(box_row + (((u0 + u) ^ sw) << 4)) = w;
+  };
+  if constexpr (EPI == GEMM_EPI_SWIGLU) {
+    uint32_t o[8];
+#pragma unroll
+    for (int j = 0; j < 16; j += 2) {
+      const float g0 = v[j], g1 = v[j + 1], u_0 = v[16 + j], u_1 = v[17 + j];
+      o[j / 2] = pack_bf16(g0 / (1.f + expf(-g0)) * u_0, g1 / (1.f + expf(-g1)) * u_1);
+    }
+    put(0, make_uint4(o[0], o[1], o[2], o[3]));
+    put(1, make_uint4(o[4], o[5], o[6], o[7]));
+  } else {
+    uint32_t o[16];
+    if constexpr (EPI == GEMM_EPI_RESIDUAL) {
+      const uint4* src = reinterpret_cast<const uint4*>(R + (int64_t)row * ldc + col);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 r4 = row < M ? src[q] : make_uint4(0, 0, 0, 0);
+        const uint32_t rw[4] = {r4.x, r4.y, r4.z, r4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int j = q * 8 + e * 2;
+          o[q * 4 + e] = pack_bf16(v[j] + bf16_lo(rw[e]), v[j + 1] + bf16_hi(rw[e]));
+        }
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; j += 2) o[j / 2] = pack_bf16(v[j], v[j + 1]);
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) put(q, make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]));
+  }
+}
+
+// One epilogue warp's pass over its 32 rows of an accumulator: 8 chunks of
+// 32 columns read with tcgen05.ld, staged into boxes, each full box stored
+// by TMA. `nbox` counts the warp's boxes across tiles (it picks the buffer).
+template <int EPI>
+__device__ __forceinline__ void epilogue_rows(uint32_t t_row, int row0, int M, int col0,
+                                              const uint16_t* __restrict__ R, int ldc,
+                                              const CUtensorMap* map_c, uint8_t* boxes,
+                                              int lane, int& nbox) {
+  constexpr int CPB = epi_chunks_per_box<EPI>();
+  constexpr int UPC = 8 / CPB;               // 16-byte units per chunk in a box row
+#pragma unroll 1
+  for (int c0 = 0; c0 < kBN; c0 += 32) {
+    float v[32];
+    tmem_ld32(t_row + c0, v);   // every lane takes part (.sync.aligned)
+    const int cib = (c0 / 32) % CPB;
+    uint8_t* box = boxes + (nbox & 1) * kEpiBox;
+    if (cib == 0 && nbox >= 2) {   // the store that read this box two boxes ago
+      if (lane == 0) epi_wait_read_1();
+      __syncwarp();
+    }
+    stage_chunk<EPI>(v, row0 + lane, M, col0 + c0, R, ldc, box + lane * 128, cib * UPC, lane);
+    if (cib == CPB - 1) {
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const int first = col0 + c0 - (CPB - 1) * 32;   // the box's first accumulator column
+        const int x = EPI == GEMM_EPI_SWIGLU ? first / 2 : first;
+        tma_store_2d(map_c, saddr(box), x, row0);
+        epi_commit();
+      }
+      ++nbox;
+    }
+  }
+}
+
 // Persistent, warp-specialized: warp 0 loads (TMA), warp 1 issues the MMAs
 // into one of two tensor-memory accumulators, warps 2..5 drain the other
 // accumulator through the epilogue, so the epilogue of tile i overlaps the
@@ -190,13 +307,15 @@ __device__ __forceinline__ void store_chunk(const float (&v)[32], int row, int c
 template <int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap map_a,
-                     const __grid_constant__ CUtensorMap map_b, int M, int N, int K,
+                     const __grid_constant__ CUtensorMap map_b,
+                     const __grid_constant__ CUtensorMap map_c, int M, int N, int K,
                      const uint16_t* __restrict__ R, uint16_t* __restrict__ C, int ldc,
                      int* status) {
   extern __shared__ uint8_t gsm_raw[];
   // 1024-byte alignment: the 128-byte swizzle pattern repeats every 1024 bytes
   uint8_t* gsm = reinterpret_cast<uint8_t*>(((uintptr_t)gsm_raw + 1023) & ~(uintptr_t)1023);
-  uint64_t* full = reinterpret_cast<uint64_t*>(gsm + kStages * kStageBytes);
+  uint8_t* epi_boxes = gsm + kStages * kStageBytes;   // [kEpiWarps][2] boxes, 1024-aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi_boxes + kEpiSmem);
   uint64_t* empty = full + kStages;
   uint64_t* tfull = empty + kStages;     // [2] accumulator ready (MMA -> epilogue)
   uint64_t* tempty = tfull + 2;          // [2] accumulator drained (epilogue -> MMA)
@@ -297,7 +416,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   } else {
     // epilogue warps: warp w reads tensor-memory lanes 32 (w % 4) .. + 31
     const int q = warp & 3;
-    int lt = 0;
+    uint8_t* boxes = epi_boxes + q * 2 * kEpiBox;
+    int lt = 0, nbox = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
       const int acc = lt & 1;
       const bool ok = mbar_wait(saddr(&tfull[acc]), (lt >> 1) & 1);
@@ -308,18 +428,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       int mt, nt;
       tile_coords<kGroupRows / kBM>(t, num_m, num_n, &mt, &nt);
-      const int row = mt * kBM + q * 32 + lane;
       const uint32_t t_row = tmem + acc * kBN + ((uint32_t)(q * 32) << 16);
-#pragma unroll 1
-      for (int c0 = 0; c0 < kBN; c0 += 32) {
-        float v[32];
-        tmem_ld32(t_row + c0, v);   // every lane takes part (.sync.aligned)
-        if (row < M) store_chunk<EPI>(v, row, nt * kBN + c0, R, C, ldc);
-      }
+      epilogue_rows<EPI>(t_row, mt * kBM + q * 32, M, nt * kBN, R, ldc, &map_c, boxes, lane,
+                         nbox);
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       __syncwarp();
       if (lane == 0) mbar_arrive(saddr(&tempty[acc]));
     }
+    if (lane == 0) epi_wait_all();   // the boxes are read before the CTA leaves
   }
   __syncthreads();
   if (*vfailed && threadIdx.x == 0) atomicCAS(status, 0, (int)SCONE_ERR_CUDA);
@@ -344,7 +460,7 @@ constexpr int kPairAccs = 2;                                 // accumulators per
 constexpr uint32_t kPairTmemCols = kPairAccs * kBN;
 constexpr uint32_t kPStageHalf = 128 * kBK * 2;             // 16 KB: A or B half
 constexpr uint32_t kPStageBytes = 2 * kPStageHalf;          // per CTA
-constexpr size_t kPairSmem = (size_t)kPStages * kPStageBytes + 1024 + 256;
+constexpr size_t kPairSmem = (size_t)kPStages * kPStageBytes + 1024 + 256 + kEpiSmem;
 constexpr uint32_t kIdescPair = (1u << 4) | (1u << 7) | (1u << 10) |
                                 ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(256 >> 4) << 24);
 
@@ -376,12 +492,14 @@ __device__ __forceinline__ void umma_commit_pair(uint32_t bar) {
 template <int EPI>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_bf16_pair_kernel(const __grid_constant__ CUtensorMap map_a,
-                          const __grid_constant__ CUtensorMap map_b, int M, int N, int K,
+                          const __grid_constant__ CUtensorMap map_b,
+                          const __grid_constant__ CUtensorMap map_c, int M, int N, int K,
                           const uint16_t* __restrict__ R, uint16_t* __restrict__ C, int ldc,
                           int* status) {
   extern __shared__ uint8_t gsm_raw[];
   uint8_t* gsm = reinterpret_cast<uint8_t*>(((uintptr_t)gsm_raw + 1023) & ~(uintptr_t)1023);
-  uint64_t* full = reinterpret_cast<uint64_t*>(gsm + kPStages * kPStageBytes);
+  uint8_t* epi_boxes = gsm + kPStages * kPStageBytes;   // [kEpiWarps][2] boxes, 1024-aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi_boxes + kEpiSmem);
   uint64_t* empty = full + kPStages;
   uint64_t* tfull = empty + kPStages;
   uint64_t* tempty = tfull + 2;
@@ -486,7 +604,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     const int q = warp & 3;
     const uint32_t tempty_leader0 = map_to_rank(saddr(&tempty[0]), 0);
     const uint32_t tempty_leader1 = map_to_rank(saddr(&tempty[1]), 0);
-    int lt = 0;
+    uint8_t* boxes = epi_boxes + q * 2 * kEpiBox;
+    int lt = 0, nbox = 0;
     for (int t = pair; t < tiles; t += pairs, ++lt) {
       const int acc = lt % kPairAccs;
       if (!mbar_wait(saddr(&tfull[acc]), (lt / kPairAccs) & 1) || *vfailed) {
@@ -496,18 +615,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       int mt, nt;
       tile_coords<kGroupRows / 256>(t, num_m, num_n, &mt, &nt);
-      const int row = mt * 256 + (int)rank * 128 + q * 32 + lane;
       const uint32_t t_row = tmem + acc * kBN + ((uint32_t)(q * 32) << 16);
-#pragma unroll 1
-      for (int c0 = 0; c0 < kBN; c0 += 32) {
-        float v[32];
-        tmem_ld32(t_row + c0, v);
-        if (row < M) store_chunk<EPI>(v, row, nt * kBN + c0, R, C, ldc);
-      }
+      epilogue_rows<EPI>(t_row, mt * 256 + (int)rank * 128 + q * 32, M, nt * kBN, R, ldc,
+                         &map_c, boxes, lane, nbox);
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(acc ? tempty_leader1 : tempty_leader0);
     }
+    if (lane == 0) epi_wait_all();   // the boxes are read before the CTA leaves
   }
   // every MMA of the pair has completed before either CTA frees its tensor memory
   if (threadIdx.x == 32) mbar_wait(saddr(done), 0);
@@ -552,6 +667,21 @@ bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int box_rows
          CUDA_SUCCESS;
 }
 
+// 2-D map of C [rows x ldc] for the epilogue's stores: box 64 columns x 32
+// rows, 128-byte swizzle (as the boxes are staged); rows past the end are
+// clipped.
+bool make_map_c(CUtensorMap* m, void* base, int rows, int ldc) {
+  const auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)ldc, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)ldc * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)kEpiBoxCols, 32};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int EPI>
 bool set_smem_attr() {
   static std::once_flag once;
@@ -581,11 +711,27 @@ template <int EPI>
 int launch_pair(const CUtensorMap& ma, const CUtensorMap& mb, int M, int N, int K,
                 const uint16_t* R, uint16_t* C, int ldc, int* status, cudaStream_t s) {
   if (!set_pair_smem_attr<EPI>()) return SCONE_ERR_CUDA;
+  CUtensorMap mc;
+  if (!make_map_c(&mc, C, M, ldc)) return SCONE_ERR_CUDA;
   const int64_t tiles = (int64_t)((M + 255) / 256) * (N / kBN);
   const int64_t pairs = sm_count() / 2;
   const unsigned grid = (unsigned)(2 * (tiles < pairs ? tiles : pairs));
-  gemm_bf16_pair_kernel<EPI><<<grid, kGemmThreads, kPairSmem, s>>>(ma, mb, M, N, K, R, C, ldc,
-                                                                   status);
+  gemm_bf16_pair_kernel<EPI><<<grid, kGemmThreads, kPairSmem, s>>>(ma, mb, mc, M, N, K, R, C,
+                                                                   ldc, status);
+  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
+}
+
+template <int EPI>
+int launch_single(const CUtensorMap& ma, const CUtensorMap& mb, int M, int N, int K,
+                  const uint16_t* R, uint16_t* C, int ldc, int* status, cudaStream_t s) {
+  if (!set_smem_attr<EPI>()) return SCONE_ERR_CUDA;
+  CUtensorMap mc;
+  if (!make_map_c(&mc, C, M, ldc)) return SCONE_ERR_CUDA;
+  const int64_t tiles = (int64_t)((M + kBM - 1) / kBM) * (N / kBN);
+  const int64_t sms = sm_count();
+  const dim3 grid((unsigned)(tiles < sms ? tiles : sms));
+  gemm_bf16_kernel<EPI><<<grid, kGemmThreads, kGemmSmem, s>>>(ma, mb, mc, M, N, K, R, C, ldc,
+                                                             status);
   return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
 }
 
@@ -621,29 +767,16 @@ int gemm_bf16_variant(const uint16_t* A, const uint16_t* B, const uint16_t* R, u
   }
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, M, K, kBM) || !make_map(&mb, B, N, K, kBN)) return SCONE_ERR_CUDA;
-  const int64_t tiles = (int64_t)((M + kBM - 1) / kBM) * (N / kBN);
-  const int64_t sms = sm_count();
-  const dim3 grid((unsigned)(tiles < sms ? tiles : sms));
   switch (epi) {
     case GEMM_EPI_STORE:
-      if (!set_smem_attr<GEMM_EPI_STORE>()) return SCONE_ERR_CUDA;
-      gemm_bf16_kernel<GEMM_EPI_STORE><<<grid, kGemmThreads, kGemmSmem, s>>>(ma, mb, M, N, K, R,
-                                                                            C, ldc, status);
-      break;
+      return launch_single<GEMM_EPI_STORE>(ma, mb, M, N, K, R, C, ldc, status, s);
     case GEMM_EPI_RESIDUAL:
-      if (!set_smem_attr<GEMM_EPI_RESIDUAL>()) return SCONE_ERR_CUDA;
-      gemm_bf16_kernel<GEMM_EPI_RESIDUAL><<<grid, kGemmThreads, kGemmSmem, s>>>(
-          ma, mb, M, N, K, R, C, ldc, status);
-      break;
+      return launch_single<GEMM_EPI_RESIDUAL>(ma, mb, M, N, K, R, C, ldc, status, s);
     case GEMM_EPI_SWIGLU:
-      if (!set_smem_attr<GEMM_EPI_SWIGLU>()) return SCONE_ERR_CUDA;
-      gemm_bf16_kernel<GEMM_EPI_SWIGLU><<<grid, kGemmThreads, kGemmSmem, s>>>(ma, mb, M, N, K, R,
-                                                                             C, ldc, status);
-      break;
+      return launch_single<GEMM_EPI_SWIGLU>(ma, mb, M, N, K, R, C, ldc, status, s);
     default:
       return SCONE_ERR_INVALID_ARG;
   }
-  return cudaGetLastError() == cudaSuccess ? SCONE_OK : SCONE_ERR_CUDA;
 }
 
 }  // namespace scone

@@ -69,3 +69,23 @@ def test_rejects_bad_shapes():
     C = torch.empty((128, 200), dtype=torch.bfloat16, device=DEV)
     with pytest.raises(scone.SconeError):
         scone.scone_gemm_bf16(A, B, C)
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+@pytest.mark.parametrize("epilogue", [0, 1, 2])      # store, residual, SwiGLU
+def test_rows_past_m_are_not_written(variant, epilogue):
+    """The epilogue stores whole 32-row boxes; rows past M must stay untouched
+    (the store clips them), for every epilogue and a ragged M."""
+    M, N, K = 333, 512, 128
+    A, B = rand((M, K), 8), rand((N, K), 9)
+    ncol = N // 2 if epilogue == scone.SCONE_GEMM_SWIGLU else N
+    full = torch.full((M + 64, ncol), 7.0, dtype=torch.bfloat16, device=DEV)
+    C = full[:M]
+    R = None
+    if epilogue == scone.SCONE_GEMM_RESIDUAL:
+        C.copy_(rand((M, ncol), 10))
+        R = C
+    want_tail = full[M:].clone()
+    scone.scone_gemm_bf16(A, B, C, R=R, epilogue=epilogue, variant=variant)
+    torch.cuda.synchronize()
+    assert torch.equal(full[M:], want_tail)
