@@ -1476,7 +1476,9 @@ def bench_discover(args, world, rank, local):
                 "h2d_bytes_per_step": 4 * n,
                 "d2h_bytes_per_step": n_sel * (4 * w.K + 1 + 4),
                 "what": "pinned corpus -> device, scone_fgram_discover, f-gram list -> "
-                        "pinned host"},
+                        "pinned host",
+                "per_call_ms": [round(1e3 * x, 2) for x in e2e_t],
+                "spread": max(e2e_t) / min(e2e_t) - 1.0},
         # per call: bin, hotflush, bincount, flagbin, unsort, scan and assign
         # per scan; then 4 radix-select histograms (only when the cut falls
         # inside the list), select_count, two scans and emit
