@@ -323,13 +323,15 @@ def bench_prefill(args, world, rank, local):
     dev_tok = torch.empty_like(batches[0])
     e2e_steps = max(3, min(args.steps, 50))
 
+    raw_stream = stream.cuda_stream    # the caller's stream handle, passed to each call
+
     def e2e_step(k, staged):
         if staged:
             dev_tok.copy_(host_tok[k % N_BATCHES], non_blocking=True)
-            scone.scone_embed(table, dev_tok, out)
+            scone.scone_embed(table, dev_tok, out, stream=raw_stream)
         else:
-            scone.scone_embed(table, host_tok[k % N_BATCHES], out)
-        scone.scone_status(table)      # syncs the stream, reads the 4-byte status word
+            scone.scone_embed(table, host_tok[k % N_BATCHES], out, stream=raw_stream)
+        scone.scone_status(table, raw_stream)   # syncs the stream, reads the status word
 
     e2e_ms = {}
     for staged in (False, True):
@@ -681,6 +683,7 @@ def bench_decode(args, world, rank, local):
     tok_d = torch.empty(S, dtype=torch.int32, device=dev)
     e2e_n = min(steps, 64)
     e2e_ms = {}
+    raw_stream = torch.cuda.current_stream().cuda_stream
     for staged in (False, True):
         e2e_t = []
         for k in range(e2e_n + 3):
@@ -688,10 +691,10 @@ def bench_decode(args, world, rank, local):
             t1 = time.perf_counter()
             if staged:
                 tok_d.copy_(host_new[k % steps], non_blocking=True)
-                scone.scone_decode_step(st, tok_d, out)
+                scone.scone_decode_step(st, tok_d, out, stream=raw_stream)
             else:
-                scone.scone_decode_step(st, host_new[k % steps], out)
-            scone.scone_status(table)
+                scone.scone_decode_step(st, host_new[k % steps], out, stream=raw_stream)
+            scone.scone_status(table, raw_stream)
             if k >= 3:
                 e2e_t.append(time.perf_counter() - t1)
         e2e_ms[staged] = max_over_ranks(1e3 * statistics.mean(e2e_t), world)
