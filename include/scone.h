@@ -187,7 +187,8 @@ int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
 
 /* How scone_embed moves rows (a tuning knob; results are identical). */
 enum scone_copy_mode {
-  SCONE_COPY_AUTO = 0,       /* the library picks per call */
+  SCONE_COPY_AUTO = 0,       /* the library picks per call: PIPELINED for 3 < K <= 5 where it
+                                applies, REGISTERS otherwise */
   SCONE_COPY_REGISTERS = 1,  /* 16-byte loads and streaming stores through registers */
   SCONE_COPY_BULK = 2,       /* cp.async.bulk (TMA) through a shared-memory ring; needs rows of a
                                 multiple of 16 bytes, 16-byte aligned F, T and out, and F in
