@@ -633,6 +633,9 @@ def bench_decode(args, world, rank, local):
                                     F_location=scone.SCONE_ROWS_HOST_MAPPED)
     setup_s = time.time() - t0
     link = host_link_bandwidth(dev, table, w.n_fgrams, w.d)
+    # decode steps move rows with register loads (AUTO) or TMA bulk copies (--copy bulk)
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_BULK if args.copy == "bulk"
+                                    else scone.SCONE_COPY_AUTO)
     hist, hl, new = synth.decode_inputs(w)
     S, steps = w.dec_S, w.dec_steps
     new_d = torch.from_numpy(new).to(dev)
@@ -738,7 +741,8 @@ def bench_decode(args, world, rank, local):
             "decode_rows": step_rows,
             "host_bytes_per_step": host_bytes_step,
             "hbm_bytes_per_step": hbm_bytes_step,
-            "kernel": "decode_kernel (one warp per sequence)",
+            "kernel": ("decode_kernel (one warp per sequence, TMA bulk row copies)"
+                       if args.copy == "bulk" else "decode_kernel (one warp per sequence)"),
         },
         "e2e": {"value": world * S / (e2e_ms[False] * 1e-3), "unit": "tokens/s",
                 "h2d_bytes_per_step": 4 * S, "d2h_bytes_per_step": 4,

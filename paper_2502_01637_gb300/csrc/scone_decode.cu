@@ -28,24 +28,43 @@
 #include <new>
 
 #include "scone_host.h"
+#include "scone_ptx.cuh"
 
 namespace scone {
 
 constexpr int kDecThreads = 128;
 constexpr int kDecWarps = kDecThreads / 32;
+constexpr uint32_t kDecSpinLimit = 1u << 22;
+constexpr int kDecBulkMaxSmem = 192 * 1024;   // rows of a block's warps staged for bulk copies
 
 namespace {
 
-template <int FMT, int W>
+// W: row copy width (16 or 0 = generic) for register copies. BULK: with
+// SCONE_COPY_BULK the selected row moves by TMA bulk copies instead: lane 0
+// copies it host/global -> shared (one cp.async.bulk, completion counted in
+// bytes on the warp's mbarrier) -> output (cp.async.bulk store), so a row is
+// one DMA request per direction and holds no registers. Every wait is
+// bounded: past kDecSpinLimit polls the warp records SCONE_ERR_CUDA and
+// stops copying.
+template <int FMT, int W, bool BULK>
 __global__ void __launch_bounds__(kDecThreads)
     decode_kernel(const TableView t, int32_t* __restrict__ hist, int32_t* __restrict__ hist_len,
                   const int32_t* __restrict__ new_tok, int32_t S, int32_t H,
                   uint8_t* __restrict__ out, int32_t* __restrict__ row_out,
-                  uint8_t* __restrict__ len_out, int width) {
+                  uint8_t* __restrict__ len_out, int width, const uint8_t* __restrict__ zero_row) {
   constexpr int NW = Fmt<FMT>::kWords;
   __shared__ const void* src_s[kDecWarps][1];
+  __shared__ __align__(8) uint64_t bulk_bar[kDecWarps];
+  extern __shared__ __align__(128) uint8_t dec_rows[];   // [kDecWarps][row_bytes] (BULK)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int row_bytes = t.d * 2;
+  if (BULK && threadIdx.x == 0) {
+    for (int w = 0; w < kDecWarps; ++w) mbar_init(saddr(&bulk_bar[w]), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (BULK) __syncthreads();
+  uint32_t phase = 0;
+  bool broken = false;
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;");
   for (int64_t s = (int64_t)blockIdx.x * kDecWarps + warp; s < S;
@@ -105,18 +124,58 @@ __global__ void __launch_bounds__(kDecThreads)
       src_s[warp][0] = src;
     }
     __syncwarp();
-    if (out)   // NULL: selection only (the rows are gathered elsewhere, e.g. from a row store)
-      warp_copy_rows_w<W>(src_s[warp], out + s * (int64_t)row_bytes, 1, row_bytes, width, lane);
+    if (out) {   // NULL: selection only (the rows are gathered elsewhere, e.g. from a row store)
+      if constexpr (BULK) {
+        if (lane == 0 && !broken) {
+          const void* from = src_s[warp][0] ? src_s[warp][0] : (const void*)zero_row;
+          uint8_t* buf = dec_rows + warp * row_bytes;
+          const uint32_t bar = saddr(&bulk_bar[warp]);
+          bulk_wait_read_all();   // this warp's previous row store has read the buffer
+          mbar_expect_tx(bar, (uint32_t)row_bytes);
+          bulk_load(saddr(buf), from, (uint32_t)row_bytes, bar);
+          if (mbar_wait_bounded(bar, phase, kDecSpinLimit)) {
+            bulk_store(out + s * (int64_t)row_bytes, saddr(buf), (uint32_t)row_bytes);
+            bulk_commit();
+            phase ^= 1;
+          } else {
+            record_error(t.status, SCONE_ERR_CUDA);
+            broken = true;
+          }
+        }
+      } else {
+        warp_copy_rows_w<W>(src_s[warp], out + s * (int64_t)row_bytes, 1, row_bytes, width,
+                            lane);
+      }
+    }
     __syncwarp();
+  }
+  if constexpr (BULK) {
+    if (lane == 0) {
+      if (broken) mbar_wait_bounded(saddr(&bulk_bar[warp]), phase, kDecSpinLimit);
+      bulk_wait_all();   // the row stores complete before the grid does
+    }
   }
 }
 
 using DecodeFn = void (*)(TableView, int32_t*, int32_t*, const int32_t*, int32_t, int32_t,
-                          uint8_t*, int32_t*, uint8_t*, int);
+                          uint8_t*, int32_t*, uint8_t*, int, const uint8_t*);
 
-DecodeFn pick_decode(int fmt, int width) {
-  if (fmt == FMT16) return width == 16 ? decode_kernel<FMT16, 16> : decode_kernel<FMT16, 0>;
-  return width == 16 ? decode_kernel<FMT32, 16> : decode_kernel<FMT32, 0>;
+DecodeFn pick_decode(int fmt, int width, bool bulk) {
+  if (bulk) return fmt == FMT16 ? decode_kernel<FMT16, 16, true> : decode_kernel<FMT32, 16, true>;
+  if (fmt == FMT16)
+    return width == 16 ? decode_kernel<FMT16, 16, false> : decode_kernel<FMT16, 0, false>;
+  return width == 16 ? decode_kernel<FMT32, 16, false> : decode_kernel<FMT32, 0, false>;
+}
+
+// Bulk row copies need 16-byte rows and addresses and room for a row per warp.
+bool decode_bulk_ok(const scone_table* tb, const void* out) {
+  const TableView& t = tb->view;
+  const int64_t row_bytes = (int64_t)t.d * 2;
+  if (tb->copy_mode != SCONE_COPY_BULK || !out || !tb->zero_row) return false;
+  if (row_bytes % 16 || row_bytes * kDecWarps > kDecBulkMaxSmem) return false;
+  uintptr_t a = (uintptr_t)t.T | (uintptr_t)out | (uintptr_t)tb->zero_row;
+  if (t.n_fgrams > 0) a |= (uintptr_t)t.F;
+  return (a & 15) == 0;
 }
 
 }  // namespace
@@ -169,14 +228,22 @@ extern "C" int scone_decode_step(scone_decode* st, const int32_t* new_tok, scone
   const scone_table* tb = st->table;
   DeviceGuard g(tb->device);
   const int width = row_copy_width(tb->view, out);
-  const DecodeFn fn = pick_decode(tb->fmt, width);
+  const bool bulk = decode_bulk_ok(tb, out);
+  const DecodeFn fn = pick_decode(tb->fmt, width, bulk);
+  const size_t smem = bulk ? (size_t)kDecWarps * tb->view.d * 2 : 0;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute((const void*)fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem) != cudaSuccess) {
+    cudaGetLastError();
+    return SCONE_ERR_CUDA;
+  }
   const int64_t need = (st->S + kDecWarps - 1) / kDecWarps;
-  const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)fn, kDecThreads, 0);
+  const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)fn, kDecThreads, smem);
   const int grid = (int)(need < cap ? need : cap);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kDecThreads);
-  cfg.dynamicSmemBytes = 0;
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = (cudaStream_t)stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -185,7 +252,7 @@ extern "C" int scone_decode_step(scone_decode* st, const int32_t* new_tok, scone
   cfg.numAttrs = 1;
   const cudaError_t e = cudaLaunchKernelEx(&cfg, fn, tb->view, st->hist, st->hist_len, new_tok,
                                            st->S, st->H, reinterpret_cast<uint8_t*>(out), row,
-                                           len, width);
+                                           len, width, (const uint8_t*)tb->zero_row);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return SCONE_ERR_CUDA;

@@ -445,3 +445,40 @@ def test_pipelined_probe_limit_reports_and_zero_rows():
     for a, b in zip(ref, got):
         assert np.array_equal(a, b)
     assert (ref[2] == 0).any()
+
+
+@pytest.mark.parametrize("K,host_F", [(3, False), (5, False), (3, True), (5, True)])
+def test_decode_bulk_row_copies(K, host_F):
+    """SCONE_COPY_BULK decode steps move each row by TMA bulk copies (global or
+    host-mapped F -> shared -> output); rows, lengths and bytes equal the
+    oracle's, including the zero rows of invalid tokens."""
+    S, steps, vocab, d = 70, 10, 2000, 128          # 256-byte rows
+    ft, fl, hist, hl, new, F, T = _decode_case(K, S, steps, vocab, d, seed=30 + K)
+    new[4, 9] = -2
+    o = oracle.Oracle(ft, fl, K, vocab)
+    o_out, o_row, o_len, _ = o.decode(hist, hl, new, F, T)
+    buf = None
+    if host_F:
+        buf = scone.scone_host_alloc(F.nbytes)
+        buf.numpy(np.uint16)[:F.size] = F.reshape(-1)
+        table = scone.scone_table_build(ft, fl, K, vocab, d, buf.ptr, dev_rows(T),
+                                        F_location=scone.SCONE_ROWS_HOST_MAPPED)
+    else:
+        table = scone.scone_table_build(ft, fl, K, vocab, d, dev_rows(F), dev_rows(T))
+    scone.scone_table_set_copy_mode(table, scone.SCONE_COPY_BULK)
+    st = scone.scone_decode_create(table, hist, hl)
+    new_d = torch.from_numpy(new).to(DEV)
+    out = torch.empty((S, d), dtype=torch.int16, device=DEV)
+    row = torch.empty(S, dtype=torch.int32, device=DEV)
+    ln = torch.empty(S, dtype=torch.uint8, device=DEV)
+    for k in range(steps):
+        out.fill_(-1)
+        scone.scone_decode_step(st, new_d[k], out, row, ln)
+        assert np.array_equal(ln.cpu().numpy(), o_len[k]), k
+        assert np.array_equal(row.cpu().numpy(), o_row[k].astype(np.int32)), k
+        assert np.array_equal(out.cpu().numpy().view(np.uint16), o_out[k]), k
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+    st.close()
+    table.close()
+    if buf is not None:
+        buf.free()
