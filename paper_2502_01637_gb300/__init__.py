@@ -173,6 +173,11 @@ def _stream(stream) -> int:
     import torch
 
     if stream is None:
+        # the raw handle of the current stream, without building a Stream object
+        # (a few microseconds per call, which a decode step feels)
+        raw = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+        if raw is not None:
+            return raw(torch.cuda.current_device())
         return torch.cuda.current_stream().cuda_stream
     if isinstance(stream, int):
         return stream

@@ -482,3 +482,13 @@ def test_decode_bulk_row_copies(K, host_F):
     table.close()
     if buf is not None:
         buf.free()
+
+
+def test_default_stream_is_the_current_stream():
+    """Calls without a stream argument enqueue on torch's current stream, also
+    inside a stream context."""
+    assert scone._stream(None) == torch.cuda.current_stream().cuda_stream
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        assert scone._stream(None) == s.cuda_stream
+    assert scone._stream(None) == torch.cuda.current_stream().cuda_stream
