@@ -96,6 +96,61 @@ def test_fullsize_prefill(name):
     table.close()
 
 
+def test_fullsize_mixed_serving():
+    """The serving batch the benchmark's mixed_serving times (65,536 tokens:
+    48 ragged prompt chunks and 512 one-token decode chunks, each continuing
+    one of 2,048 decode-state slots, prefill_1b's table), two batches in a row
+    so the second continues the histories the first left. Every position
+    against the oracle run over each sequence's whole known prefix (its slot's
+    history ++ its chunk): rows, lengths, and output rows at the oracle's ids."""
+    import bench
+
+    w = synth.WORKLOADS["prefill_1b"]
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    F = gpu_rows(synth.F_seed(w), w.n_fgrams, w.d)
+    T = gpu_rows(synth.T_seed(w), w.vocab, w.d)
+    table = scone.scone_table_build(fg_tok, fg_len, w.K, w.vocab, w.d, F, T)
+    S, H = 2048, w.K - 1
+    hist = synth.query_tokens(w.scaled("mixed_hist", B=S, L=H))
+    state = scone.scone_decode_create(table, hist, np.full(S, H, np.int32))
+    o = oracle.Oracle(fg_tok, fg_len, w.K, w.vocab)
+    known = {s: list(hist[s]) for s in range(S)}          # each slot's tokens so far
+    for k in range(2):
+        tok, cu, slots = bench.mixed_batch(w, k)
+        n = tok.size
+        out = torch.empty((n, w.d), dtype=torch.int16, device=DEV)
+        row_d = torch.empty(n, dtype=torch.int32, device=DEV)
+        ln_d = torch.empty(n, dtype=torch.uint8, device=DEV)
+        scone.scone_embed_varlen(table, torch.from_numpy(tok).to(DEV),
+                                 torch.from_numpy(cu).to(DEV), out, state=state,
+                                 seq_slot=torch.from_numpy(slots).to(DEV), row=row_d, len=ln_d)
+        assert scone.scone_status(table) == 0
+        o_row = np.empty(n, np.int64)
+        o_len = np.empty(n, np.uint8)
+        for b in range(cu.size - 1):
+            chunk = tok[cu[b]:cu[b + 1]]
+            if chunk.size == 0:
+                continue
+            seq = np.asarray(known[int(slots[b])] + chunk.tolist(), np.int32)[None, :]
+            r, l_, _, rc = o.select(seq)
+            assert rc == 0
+            h = seq.shape[1] - chunk.size
+            o_row[cu[b]:cu[b + 1]] = r[0, h:]
+            o_len[cu[b]:cu[b + 1]] = l_[0, h:]
+            known[int(slots[b])] = seq[0].tolist()[-H:]
+        row, ln = row_d.cpu().numpy(), ln_d.cpu().numpy()
+        bad = np.flatnonzero((row != o_row) | (ln != o_len))
+        assert bad.size == 0, f"batch {k}: {bad.size} positions differ, first at {bad[0]}"
+        r64 = torch.from_numpy(o_row).to(DEV)
+        exp = T.index_select(0, torch.from_numpy(tok).to(DEV).to(torch.int64))
+        idx = torch.nonzero(r64 >= 0).reshape(-1)
+        exp[idx] = F.index_select(0, r64[idx])
+        assert bool((out == exp).all()), f"batch {k}: output rows differ"
+        assert (o_len == 3).any() and (o_len == 1).any()
+    state.close()
+    table.close()
+
+
 def test_fullsize_offload_decode():
     """2e7 f-grams, F (82 GB) in host-pinned mapped memory; 512 sequences x 256
     steps. Rows and lengths of every step are checked against the oracle (decode
