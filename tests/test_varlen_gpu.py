@@ -152,7 +152,7 @@ def test_mixed_batch_with_slot_map(case):
     st = scone.scone_decode_create(case.table, np.zeros((S, H), np.int32), np.zeros(S, np.int32))
     rng = np.random.default_rng(3)
     seqs = {s: list(stream_tokens(int(rng.integers(1, 40)), 400 + s)) for s in range(S)}
-    # round 1: slots 0..11 prefill in a shuffled order
+    # first batch: slots 0..11 prefill in a shuffled order
     order = rng.permutation(S)
     run_varlen(case, [np.array(seqs[s], np.int32) for s in order], state=st, slots=order)
     for rnd in range(4):
