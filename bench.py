@@ -351,10 +351,11 @@ def bench_prefill(args, world, rank, local):
     bytes_launch = per_tok * n_tok
     hbm, peak_src = measured_peaks()
     achieved = bytes_launch / (kernel_ms * 1e-3) / 1e9
-    kname = embed_kernel_name(args.copy, w.K).split()[0]
+    kname_full = embed_kernel_name(args.copy, w.K, bool(info["suffix_index"]))
+    kname = kname_full.split()[0]
     traffic, traffic_note = profiled_traffic(
-        w.name, kname, PIPE_SOURCES if kname == "embed_pipe_kernel" else EMBED_SOURCES,
-        with_note=True)
+        w.name, kname, PIPE_SOURCES if kname in ("embed_pipe_kernel", "embed_walk_kernel")
+        else EMBED_SOURCES, with_note=True)
     res = {
         "metric": METRIC,
         "value": world * n_tok / (ms_step * 1e-3),
@@ -385,7 +386,7 @@ def bench_prefill(args, world, rank, local):
             "traffic_note": traffic_note,
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
             "algorithmic_bytes_per_launch": bytes_launch,
-            "kernel": embed_kernel_name(args.copy, w.K),
+            "kernel": kname_full,
         },
         "e2e": {
             "value": world * n_tok / (e2e_ms[False] * 1e-3),
@@ -407,7 +408,8 @@ def bench_prefill(args, world, rank, local):
         "match_len_hist": {str(i): int(c) for i, c in enumerate(hist)},
         "avg_match_len": float((hist * np.arange(len(hist))).sum() / max(1, hist.sum())),
         "table": {k: info[k] for k in ("n_slots", "slot_bytes", "table_bytes",
-                                       "max_insert_probe", "F_bytes", "T_bytes")},
+                                       "max_insert_probe", "F_bytes", "T_bytes", "n_markers",
+                                       "suffix_index")},
         "setup_s": setup_s,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -416,13 +418,17 @@ def bench_prefill(args, world, rank, local):
     return res
 
 
-def embed_kernel_name(copy: str, K: int) -> str:
+def embed_kernel_name(copy: str, K: int, suffix_index: bool = False) -> str:
     """The kernel scone_embed launches for a copy mode (16-byte slots, aligned rows)."""
     if copy == "bulk":
         return "embed_bulk_kernel (fused match + TMA bulk gather)"
     if copy == "split":
         return "embed_split_kernel (match warps feed copy warps through shared memory)"
-    if copy == "pipelined" or (copy == "auto" and 3 < K <= 5):
+    pipe = copy == "pipelined" or (copy == "auto" and K <= 5 and (K > 3 or suffix_index))
+    if pipe and suffix_index:
+        return ("embed_walk_kernel (the lengths walked one bucket at a time over the suffix "
+                "index, interleaved into the copy)")
+    if pipe:
         return "embed_pipe_kernel (next tile's match interleaved into the copy)"
     return "embed_kernel (fused match + gather)"
 

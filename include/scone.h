@@ -97,11 +97,45 @@ enum scone_rows_location {
  * failed (not expected below load factor 0.85). Errors: INVALID_ARG (bad
  * list, length, token or pointer), DUPLICATE_FGRAM, TABLE_FULL,
  * UNSUPPORTED (key does not fit: K*ceil(log2 vocab) > 220), NOMEM, CUDA.
+ *
+ * Tables with 16-byte slots and 3 <= K <= 5 also get a suffix index (see
+ * scone_fgram_suffix_index): every suffix of length >= 2 of a listed f-gram
+ * is findable, as an f-gram or as a marker slot without a row, and carries
+ * a bit saying that a longer f-gram ends with it. The fused embed can then
+ * look the lengths up one at a time and stop at the first absent window.
+ * The markers count towards the load factor (scone_table_info.n_markers);
+ * results are the same with or without the index.
  */
 int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_len, int64_t n_fgrams,
                       int32_t K, int32_t vocab, int32_t d, const scone_bf16* F,
                       int32_t F_location, const scone_bf16* T, float load_factor, void* stream,
                       scone_table** out);
+
+/*
+ * scone_fgram_suffix_index — the suffix index that scone_table_build adds to
+ * a table (host only, no GPU needed). Algorithm 1 (Sec. 3) takes the longest
+ * window ending at a position that is an f-gram. If every suffix of length
+ * >= 2 of every listed f-gram can be found, with a bit saying that a longer
+ * f-gram ends with it, a lookup may try n = 2, 3, ... and stop at the first
+ * window that is absent or lacks the bit: no longer window is an f-gram.
+ *
+ *  fgram_tok, fgram_len, n_fgrams, K  the list, as for scone_table_build.
+ *  ext         host uint8 [n_fgrams] or NULL: ext[r] = 1 when f-gram r is a
+ *              suffix of a longer listed f-gram, else 0.
+ *  marker_tok  host int32 [marker_cap * K] or NULL: the suffixes that are not
+ *              listed, each once, padded with -1 (oldest token first).
+ *  marker_len  host uint8 [marker_cap] or NULL: their lengths.
+ *  marker_cap  markers the caller has room for (0: count only); the first
+ *              min(cap, count) markers are written.
+ *  n_markers   receives the number of markers.
+ *
+ * Markers are listed in the order the f-grams reach them (f-gram order,
+ * longest suffix first). Errors: INVALID_ARG (bad pointer, K or length),
+ * DUPLICATE_FGRAM, UNSUPPORTED (more than 2^32 - 2 entries), NOMEM.
+ */
+int scone_fgram_suffix_index(const int32_t* fgram_tok, const uint8_t* fgram_len,
+                             int64_t n_fgrams, int32_t K, uint8_t* ext, int32_t* marker_tok,
+                             uint8_t* marker_len, int64_t marker_cap, int64_t* n_markers);
 
 /* Frees the slot array and status word (after a device synchronize). NULL is a no-op. */
 int scone_table_destroy(scone_table* table);
@@ -117,7 +151,9 @@ int scone_table_destroy(scone_table* table);
  *
  * It reuses the table's own slot array, so the new list must fit it: at most
  * 0.85 * n_slots f-grams (see scone_table_get_info). K, vocab, d, T and the F
- * location stay those of the original build. The build kernels' scratch (a
+ * location stay those of the original build. The rebuilt table has no
+ * suffix index (n_markers 0: computing one needs host memory), so the fused
+ * embed looks every length up; results are the same. The build kernels' scratch (a
  * device copy of the list plus three flags) lives in one file-scope device
  * array of SCONE_REBUILD_SCRATCH_BYTES, which every GPU that loads the library
  * holds until the process exits. A list of n f-grams needs
@@ -173,6 +209,8 @@ typedef struct scone_table_info {
   int64_t table_bytes;       /* slot array */
   int64_t F_bytes;           /* n_fgrams * d * 2 (borrowed) */
   int64_t T_bytes;           /* vocab * d * 2 (borrowed) */
+  int64_t n_markers;         /* marker slots of the suffix index (0 without one) */
+  int32_t suffix_index;      /* 1: the table has a suffix index (see scone_table_build) */
 } scone_table_info;
 
 int scone_table_get_info(const scone_table* table, scone_table_info* info);
@@ -187,8 +225,8 @@ int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
 
 /* How scone_embed moves rows (a tuning knob; results are identical). */
 enum scone_copy_mode {
-  SCONE_COPY_AUTO = 0,       /* the library picks per call: PIPELINED for 3 < K <= 5 where it
-                                applies, REGISTERS otherwise */
+  SCONE_COPY_AUTO = 0,       /* the library picks per call: PIPELINED where it applies and the
+                                table has a suffix index or 3 < K <= 5, REGISTERS otherwise */
   SCONE_COPY_REGISTERS = 1,  /* 16-byte loads and streaming stores through registers */
   SCONE_COPY_BULK = 2,       /* cp.async.bulk (TMA) through a shared-memory ring; needs rows of a
                                 multiple of 16 bytes, 16-byte aligned F, T and out, and F in
@@ -196,8 +234,10 @@ enum scone_copy_mode {
   SCONE_COPY_SPLIT = 3,      /* register copies by warps that only copy, fed through a
                                 shared-memory ring by warps that only match */
   SCONE_COPY_PIPELINED = 4   /* register copies with the next tile's match interleaved into
-                                the current tile's copy; for 16-byte slots, K <= 5 and
-                                16-byte-aligned rows, else as SCONE_COPY_REGISTERS */
+                                the current tile's copy (on a table with a suffix index the
+                                match walks the lengths one bucket at a time); for 16-byte
+                                slots, K <= 5 and 16-byte-aligned rows, else as
+                                SCONE_COPY_REGISTERS */
 };
 
 int scone_table_set_copy_mode(scone_table* table, int32_t mode);

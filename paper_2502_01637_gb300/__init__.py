@@ -45,6 +45,7 @@ SCONE_FGRAM_POS_ABSOLUTE = 0
 SCONE_FGRAM_POS_ROTARY = 1
 
 EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noalloc",
+           "scone_fgram_suffix_index",
            "scone_table_get_info", "scone_table_set_probe_limit", "scone_table_set_copy_mode",
            "scone_match", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
@@ -74,7 +75,7 @@ class scone_table_info(ctypes.Structure):
                 ("slot_bytes", _i32), ("key_bits", _i32), ("bits_per_token", _i32),
                 ("K", _i32), ("vocab", _i32), ("d", _i32), ("F_location", _i32),
                 ("max_insert_probe", _i32), ("table_bytes", _i64), ("F_bytes", _i64),
-                ("T_bytes", _i64)]
+                ("T_bytes", _i64), ("n_markers", _i64), ("suffix_index", _i32)]
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}
@@ -118,6 +119,8 @@ def load_library():
     lib.scone_table_build.argtypes = [_vp, _vp, _i64, _i32, _i32, _i32, _vp, _i32, _vp,
                                       ctypes.c_float, _vp, ctypes.POINTER(_vp)]
     lib.scone_table_destroy.argtypes = [_vp]
+    lib.scone_fgram_suffix_index.argtypes = [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _i64,
+                                             ctypes.POINTER(_i64)]
     lib.scone_table_rebuild_noalloc.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_table_get_info.argtypes = [_vp, ctypes.POINTER(scone_table_info)]
     lib.scone_table_set_probe_limit.argtypes = [_vp, _i64]
@@ -246,6 +249,29 @@ def scone_table_build(fgram_tok: np.ndarray, fgram_len: np.ndarray, K: int, voca
                                ctypes.byref(h))
     _check(rc, "scone_table_build")
     return Table(h, (F, T))
+
+
+def scone_fgram_suffix_index(fgram_tok: np.ndarray, fgram_len: np.ndarray, K: int):
+    """The suffix index scone_table_build gives a table (host only): returns
+    (ext [N] uint8, marker_tok [M, K] int32 padded with -1, marker_len [M] uint8)."""
+    lib = load_library()
+    ft = np.ascontiguousarray(fgram_tok, dtype=np.int32).reshape(-1)
+    fl = np.ascontiguousarray(fgram_len, dtype=np.uint8).reshape(-1)
+    n = fl.shape[0]
+    if ft.shape[0] != n * K:
+        raise ValueError("fgram_tok must be [n_fgrams, K]")
+    ext = np.zeros(n, np.uint8)
+    count = _i64(0)
+    args = (_ptr(ft) if n else None, _ptr(fl) if n else None, n, K)
+    _check(lib.scone_fgram_suffix_index(*args, _ptr(ext) if n else None, None, None, 0,
+                                        ctypes.byref(count)), "scone_fgram_suffix_index")
+    m = count.value
+    mt = np.full((m, K), -1, np.int32)
+    ml = np.zeros(m, np.uint8)
+    if m:
+        _check(lib.scone_fgram_suffix_index(*args, None, _ptr(mt), _ptr(ml), m,
+                                            ctypes.byref(count)), "scone_fgram_suffix_index")
+    return ext, mt, ml
 
 
 def scone_table_destroy(table: Table) -> None:

@@ -24,6 +24,16 @@
 //          64..127, 128..191, key 192..223 | row << 32}; 64-byte buckets.
 //
 // The row word of an empty slot is 0xFFFFFFFF (row -1).
+//
+// Suffix index (tables built with one, TableView::suffix_index = 1): bit 31 of
+// a row word is the extension bit, set when the slot's n-gram is the suffix
+// of a longer listed f-gram; bits 0..30 hold the row, or kMarkerRow for a
+// marker: an n-gram that is no f-gram itself but is such a suffix. Every
+// suffix (length >= 2) of every listed f-gram is then present, so a lookup
+// can take the lengths 2, 3, ... in turn and stop at the first window that
+// is absent or has no extension bit: no longer window can be an f-gram.
+// find_in_bucket hides both (a marker reads as absent), so every lookup that
+// takes the lengths independently works on either kind of table.
 
 #pragma once
 
@@ -38,6 +48,10 @@ constexpr int FMT16 = 0;
 constexpr int FMT32 = 1;
 constexpr int kSlotsPerBucket = 2;
 constexpr uint32_t kEmptyRow = 0xFFFFFFFFu;
+constexpr uint32_t kExtBit = 0x80000000u;     // row word: a longer f-gram ends with this n-gram
+constexpr uint32_t kRowMask = 0x7FFFFFFFu;
+constexpr uint32_t kMarkerRow = 0x7FFFFFFEu;  // row bits of a marker (no f-gram row)
+constexpr uint32_t kMarkerWord = kExtBit | kMarkerRow;
 constexpr uint64_t kHashSeed = 0x6A09E667F3BCC908ull;  // frac(sqrt 2), first 64 bits
 
 template <int FMT>
@@ -73,6 +87,7 @@ struct TableView {
   int32_t bits;
   int32_t vocab;
   int32_t d;
+  int32_t suffix_index;      // 1: extension bits and markers present (see above)
 };
 
 template <int NW>
@@ -164,24 +179,38 @@ __device__ __forceinline__ bool bucket_full(const BucketData<FMT>& v) {
   }
 }
 
-// The key's row if one of the bucket's slots holds it, else -1.
+// The row word of the slot holding the key, or kEmptyRow if the bucket
+// does not hold it (an empty slot's key bits are all ones, never a key).
 template <int FMT>
-__device__ __forceinline__ int32_t find_in_bucket(const BucketData<FMT>& v,
-                                                  const KeyBits<Fmt<FMT>::kWords>& k) {
+__device__ __forceinline__ uint32_t find_word_in_bucket(const BucketData<FMT>& v,
+                                                        const KeyBits<Fmt<FMT>::kWords>& k) {
   if constexpr (FMT == FMT16) {
     const Bucket& x = v.part[0];
-    if (x.a == k.w[0] && (uint32_t)x.b == (uint32_t)k.w[1]) return (int32_t)(x.b >> 32);
-    if (x.c == k.w[0] && (uint32_t)x.e == (uint32_t)k.w[1]) return (int32_t)(x.e >> 32);
-    return -1;
+    if (x.a == k.w[0] && (uint32_t)x.b == (uint32_t)k.w[1]) return (uint32_t)(x.b >> 32);
+    if (x.c == k.w[0] && (uint32_t)x.e == (uint32_t)k.w[1]) return (uint32_t)(x.e >> 32);
+    return kEmptyRow;
   } else {
 #pragma unroll
     for (int s = 0; s < 2; ++s) {
       const Bucket& x = v.part[s];
       if (x.a == k.w[0] && x.b == k.w[1] && x.c == k.w[2] && (uint32_t)x.e == (uint32_t)k.w[3])
-        return (int32_t)(x.e >> 32);
+        return (uint32_t)(x.e >> 32);
     }
-    return -1;
+    return kEmptyRow;
   }
+}
+
+// The f-gram row of a row word, or -1 (absent, or a marker).
+__device__ __forceinline__ int32_t row_of_word(uint32_t word) {
+  const uint32_t r = word & kRowMask;
+  return (word == kEmptyRow || r == kMarkerRow) ? -1 : (int32_t)r;
+}
+
+// The key's row if one of the bucket's slots holds it as an f-gram, else -1.
+template <int FMT>
+__device__ __forceinline__ int32_t find_in_bucket(const BucketData<FMT>& v,
+                                                  const KeyBits<Fmt<FMT>::kWords>& k) {
+  return row_of_word(find_word_in_bucket<FMT>(v, k));
 }
 
 // Looks a key up: the first bucket, then the second only if the first is

@@ -258,11 +258,14 @@ extern "C" int scone_embed(const scone_table* tb, const int32_t* tok, int32_t B,
   if (tb->copy_mode == SCONE_COPY_SPLIT)
     return launch_embed_split(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
                               (cudaStream_t)stream);
-  // AUTO: the pipelined kernel where the match is long (3 < K <= 5) and it
-  // applies (measured 0.5-1% faster on stress_k5, K = 5; for K <= 3 the
-  // register kernel is 0.7-1% faster on large_hbm and prefill_1b)
+  // AUTO: the pipelined kernel where it applies and either walks the lengths
+  // (tables with a suffix index: 6% faster than the register kernel on
+  // stress_k5, K = 5, and 0.2-0.7% on the K = 3 workloads) or has a long
+  // match to hide (3 < K <= 5: 0.5-1% faster on stress_k5 than the register
+  // kernel; for K <= 3 without the index the register kernel is 0.7-1% faster)
   const bool pipe = tb->copy_mode == SCONE_COPY_PIPELINED ||
-                    (tb->copy_mode == SCONE_COPY_AUTO && tb->view.K > 3);
+                    (tb->copy_mode == SCONE_COPY_AUTO &&
+                     (tb->view.K > 3 || tb->view.suffix_index));
   if (pipe && pipe_eligible(tb, out))
     return launch_embed_pipe(tb, tok, n, L, reinterpret_cast<uint8_t*>(out), row, len,
                              (cudaStream_t)stream);

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstdint>
+#include <vector>
 #include <cuda_runtime.h>
 
 #include "scone.h"
@@ -41,6 +42,24 @@ struct DeviceGuard {
     if (prev >= 0 && prev != want) cudaSetDevice(prev);
   }
 };
+
+// Suffix index of an f-gram list (scone_suffix.cu): ext[r] = 1 when f-gram
+// r is the suffix of a longer listed f-gram; the markers are the suffixes
+// (length >= 2) of listed f-grams that are not listed themselves, each once
+// ([n_markers x K] tokens padded with -1, and their lengths). Returns
+// SCONE_OK, DUPLICATE_FGRAM, UNSUPPORTED (too many entries) or NOMEM.
+struct SuffixIndex {
+  std::vector<uint8_t> ext;
+  std::vector<int32_t> marker_tok;
+  std::vector<uint8_t> marker_len;
+  int64_t n_markers = 0;
+};
+int suffix_index(const int32_t* tok, const uint8_t* len, int64_t n, int K, SuffixIndex* out);
+
+// Whether a table of this key format and K gets a suffix index at build:
+// the kernels that walk the lengths (the pipelined embed) take 16-byte slots
+// and K <= 5; for K = 2 there are no suffixes to index.
+inline bool wants_suffix_index(int fmt, int K) { return fmt == FMT16 && K >= 3 && K <= 5; }
 
 // Bulk (TMA) fused embed: eligibility for a call and launch.
 bool bulk_eligible(const scone_table* tb, const void* out);

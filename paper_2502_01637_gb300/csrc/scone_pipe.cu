@@ -23,6 +23,18 @@
 // the copy keeps as many loads in flight as embed_kernel does. Used for the
 // 16-byte-aligned case with 16-byte slots (FMT16) and K <= 5; other calls
 // take embed_kernel.
+//
+// On a table with a suffix index (scone_device.cuh) the match walks the
+// lengths instead: n = 2, 3, ... one bucket at a time, stopping at the first
+// window that is absent or has no extension bit. The K-1 first buckets of a
+// position are mostly distinct cold sectors, and random sectors cost far
+// more DRAM time than their bytes; the walk reads about 1.7 lookups per
+// position on Zipf text at K = 5 instead of K-1. It takes more dependent
+// round trips, so a round runs after every chunk of the copy (one chunk is
+// one batch of row loads in flight), and rounds left when the copy ends run
+// back to back. The walk ends at the same longest f-gram: every suffix of
+// that f-gram is present with its extension bit, and no window longer than
+// an absent or unextended one can be an f-gram.
 
 #include "scone_host.h"
 
@@ -177,6 +189,95 @@ struct PipeMatch {
   }
 };
 
+// The walk over the lengths for one position (tables with a suffix index):
+// `state` 1 = window tokens loaded, 2 = a bucket of length n in flight into
+// this lane's shared-memory slot; 0 = done. Each round() consumes what the
+// previous one issued and issues at most one bucket, so a lane takes at
+// most 1 + 2 (K - 1) rounds.
+template <int KT>
+struct PipeWalk {
+  int32_t w[KT];      // window tokens, newest first
+  int nmax, n, state;
+  bool second;        // the bucket in flight is the key's second one
+  uint64_t b2;
+  int32_t row;        // longest f-gram found so far, or -1
+  int len, err;
+  Bucket* sb;
+
+  __device__ __forceinline__ void start(const TableView& t, const int32_t* __restrict__ tok,
+                                        int64_t p, int32_t i, bool act) {
+    state = act ? 1 : 0;
+    row = -1;
+    len = 1;
+    err = 0;
+    nmax = 0;
+    if (!act) return;
+    w[0] = __ldg(tok + p);
+    nmax = t.K < i + 1 ? t.K : i + 1;
+#pragma unroll
+    for (int j = 1; j < KT; ++j) w[j] = (j < nmax) ? __ldg(tok + p - j) : 0;
+  }
+  __device__ __forceinline__ void issue_first(const TableView& t) {
+    uint64_t b1;
+    cuckoo_buckets(key_hash<FMT16>(window_key<FMT16, KT>(w, n, t.bits), t.hash_seed),
+                   t.n_buckets, &b1, &b2);
+    bucket_async(sb, t, b1);
+    cp_async_commit();
+    second = false;
+    state = 2;
+  }
+  __device__ __forceinline__ void round(const TableView& t) {
+    if (state == 1) {
+      state = 0;
+      if (!valid_token(w[0], t.vocab)) {
+        err = SCONE_ERR_TOKEN_RANGE;
+        len = 0;
+        return;
+      }
+      // a window is usable only if all its tokens are valid
+      int nvalid = 1;
+#pragma unroll
+      for (int j = 1; j < KT; ++j)
+        if (nvalid == j && j < nmax && valid_token(w[j], t.vocab)) nvalid = j + 1;
+      nmax = nvalid;
+      if (nmax < 2) return;
+      n = 2;
+      issue_first(t);
+    } else if (state == 2) {
+      cp_async_wait_all();
+      BucketData<FMT16> v;
+      v.part[0] = *sb;
+      const uint32_t word = find_word_in_bucket<FMT16>(v, window_key<FMT16, KT>(w, n, t.bits));
+      if (word != kEmptyRow) {
+        const int32_t r = row_of_word(word);
+        if (r >= 0) {
+          row = r;
+          len = n;
+        }
+        if ((word & kExtBit) && n < nmax) {
+          ++n;
+          issue_first(t);
+        } else {
+          state = 0;
+        }
+      } else if (!second && bucket_full<FMT16>(v)) {
+        if (t.probe_limit < 2) {
+          err = SCONE_ERR_PROBE_LIMIT;
+          row = -1;
+          len = 0;
+          state = 0;
+          return;
+        }
+        bucket_async(sb, t, b2);
+        cp_async_commit();
+        second = true;
+      } else {
+        state = 0;
+      }
+    }
+  }
+};
+
 // Chunks [c_begin, c_end) of a warp's copy of nrows rows of epr 16-byte
 // elements (src[r] to dst + r * epr; NULL writes zeros): chunk c covers the
 // elements [32 U c, 32 U (c + 1)) in order, lane l taking every 32nd one.
@@ -224,6 +325,90 @@ __device__ __forceinline__ const uint4* pipe_finish(const TableView& t, PipeMatc
   }
   return reinterpret_cast<const uint4*>(r >= 0 ? t.F + (int64_t)r * t.d
                                                : t.T + (int64_t)m.w[0] * t.d);
+}
+
+// The source row of a finished walk (NULL for an error position), with the
+// row and length written out as pipe_finish does.
+template <int KT>
+__device__ __forceinline__ const uint4* walk_finish(const TableView& t, const PipeWalk<KT>& m,
+                                                    int64_t p, int32_t* __restrict__ row_out,
+                                                    uint8_t* __restrict__ len_out) {
+  if (row_out) row_out[p] = m.row;
+  if (len_out) len_out[p] = (uint8_t)m.len;
+  if (m.err) {
+    record_error(t.status, m.err);
+    return nullptr;
+  }
+  return reinterpret_cast<const uint4*>(m.row >= 0 ? t.F + (int64_t)m.row * t.d
+                                                   : t.T + (int64_t)m.w[0] * t.d);
+}
+
+// The walk's match state is small (no bucket per length in registers), so
+// for every K it runs with 8 loads in flight per lane at 3 blocks per SM (80
+// registers, no spills); on stress_k5 (K = 5) that measured 124.6 us against
+// 125.6 for 16 loads at 2 blocks, and 12 x 3 or 6 x 4 spill and were slower.
+// A warp's first tile is 8 positions: its rounds run before any row moves
+// and the slowest of its lanes sets how many (123.1 us against 124.6 for a
+// first tile of 32).
+constexpr int kWalkLoads = 8;
+constexpr int kWalkMinBlocks = 3;
+constexpr int kWalkFirst = 8;
+
+// The walk variant of the kernel below: same tiles, copies and output.
+template <int KT>
+__global__ void __launch_bounds__(kPipeThreads, kWalkMinBlocks)
+    embed_walk_kernel(const TableView t, const int32_t* __restrict__ tok, int64_t n_tok,
+                      int32_t L, uint8_t* __restrict__ out, int32_t* __restrict__ row_out,
+                      uint8_t* __restrict__ len_out) {
+  constexpr int U = kWalkLoads;
+  __shared__ const uint4* src_s[kPipeWarps][2][32];
+  __shared__ __align__(16) Bucket bucket_s[kPipeWarps][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int epr = t.d >> 3;                      // 16-byte elements per row
+  const int64_t nw = (int64_t)gridDim.x * kPipeWarps;
+  const int64_t wid = (int64_t)blockIdx.x * kPipeWarps + warp;
+  const int64_t lo = n_tok * wid / nw, hi = n_tok * (wid + 1) / nw;
+  if (lo >= hi) return;
+  PipeWalk<KT> m;
+  m.sb = &bucket_s[warp][lane];
+  int buf = 0;
+  int64_t base = lo;
+  int nrows = (int)(hi - base < kWalkFirst ? hi - base : kWalkFirst);
+  {  // the warp's first tile: its rounds back to back
+    const int64_t p = base + lane;
+    m.start(t, tok, p, (int32_t)(p % L), lane < nrows);
+    while (__any_sync(0xFFFFFFFFu, m.state != 0)) m.round(t);
+    src_s[warp][buf][lane] = lane < nrows ? walk_finish<KT>(t, m, p, row_out, len_out) : nullptr;
+    __syncwarp();
+  }
+  while (base < hi) {
+    const int64_t nbase = base + nrows;
+    const int nn = nbase < hi ? (int)(hi - nbase < 32 ? hi - nbase : 32) : 0;
+    const int64_t np = nbase + lane;
+    const int64_t total = (int64_t)nrows * epr;
+    const int nchunks = (int)((total + 32 * U - 1) / (32 * U));
+    const uint4* const* src = src_s[warp][buf];
+    uint4* dst = reinterpret_cast<uint4*>(out) + base * epr;
+    int r = 0, col = lane;
+    while (col >= epr) {
+      col -= epr;
+      ++r;
+    }
+    if (nn) m.start(t, tok, np, (int32_t)(np % L), lane < nn);
+    for (int c = 0; c < nchunks; ++c) {
+      copy_chunks<U>(src, dst, nrows, epr, total, lane, c, c + 1, r, col);
+      if (nn) m.round(t);
+    }
+    if (nn) {
+      while (__any_sync(0xFFFFFFFFu, m.state != 0)) m.round(t);
+      src_s[warp][buf ^ 1][lane] = lane < nn ? walk_finish<KT>(t, m, np, row_out, len_out)
+                                             : nullptr;
+    }
+    __syncwarp();
+    buf ^= 1;
+    base = nbase;
+    nrows = nn;
+  }
 }
 
 template <int KT>
@@ -293,7 +478,11 @@ bool pipe_eligible(const scone_table* tb, const void* out) {
 
 int launch_embed_pipe(const scone_table* tb, const int32_t* tok, int64_t n, int32_t L,
                       uint8_t* out, int32_t* row, uint8_t* len, cudaStream_t stream) {
-  const PipeFn fn = tb->view.K <= 3 ? embed_pipe_kernel<3> : embed_pipe_kernel<5>;
+  // the walk needs the suffix index; with a one-bucket probe limit (a
+  // diagnostic) the staged match reports errors where embed_kernel does
+  const bool walk = tb->view.suffix_index && tb->view.probe_limit >= 2;
+  const PipeFn fn = walk ? (tb->view.K <= 3 ? embed_walk_kernel<3> : embed_walk_kernel<5>)
+                         : (tb->view.K <= 3 ? embed_pipe_kernel<3> : embed_pipe_kernel<5>);
   // every resident block, unless warps would get fewer than 8 rows each
   const int64_t cap = (int64_t)sm_count() * blocks_per_sm((const void*)fn, kPipeThreads, 0);
   const int64_t need = (n + kPipeWarps * 8 - 1) / (kPipeWarps * 8);

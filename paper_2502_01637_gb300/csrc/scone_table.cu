@@ -16,6 +16,10 @@
 //   4. one thread per f-gram looks its key up in the finished table: it must
 //      find its own row. Finding another row means the list holds the same
 //      n-gram twice (also when two copies raced past the checks in step 2).
+// With a suffix index (scone_device.cuh) the entries placed are the listed
+// f-grams followed by the marker n-grams computed on the host
+// (scone_suffix.cu); step 3 writes each slot's final row word (row and
+// extension bit, or the marker word) and step 4 checks those words.
 
 #include <sys/mman.h>
 #include <unistd.h>
@@ -126,9 +130,17 @@ __global__ void insert_kernel(uint8_t* slots, uint64_t n_buckets, uint64_t seed,
   }
 }
 
+// The final row word of entry e: a listed f-gram's row (with its extension
+// bit when ext is given), or the marker word for the entries past n_real.
+__device__ __forceinline__ uint32_t entry_word(uint32_t e, const uint8_t* ext, int64_t n_real) {
+  if ((int64_t)e >= n_real) return kMarkerWord;
+  return e | (ext && ext[e] ? kExtBit : 0u);
+}
+
 template <int FMT>
 __global__ void fill_keys_kernel(uint8_t* slots, uint64_t n_slots, const int32_t* ftok,
-                                 const uint8_t* flen, int K, int bits) {
+                                 const uint8_t* flen, int K, int bits, const uint8_t* ext,
+                                 int64_t n_real) {
   constexpr int SLOT = Fmt<FMT>::kSlotBytes;
   constexpr int NW = Fmt<FMT>::kWords;
   for (uint64_t s = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; s < n_slots;
@@ -139,20 +151,33 @@ __global__ void fill_keys_kernel(uint8_t* slots, uint64_t n_slots, const int32_t
     const auto k = key_of_listed<FMT>(ftok, flen, (int64_t)row, K, bits);
 #pragma unroll
     for (int q = 0; q < NW - 1; ++q) w[q] = k.w[q];
-    w[NW - 1] = (uint64_t)(uint32_t)k.w[NW - 1] | ((uint64_t)row << 32);
+    w[NW - 1] = (uint64_t)(uint32_t)k.w[NW - 1] |
+                ((uint64_t)entry_word(row, ext, n_real) << 32);
   }
+}
+
+// The row word stored with the key (first bucket, then the second if the
+// first is full without it), or kEmptyRow.
+template <int FMT>
+__device__ __forceinline__ uint32_t lookup_word(const TableView& t,
+                                                const KeyBits<Fmt<FMT>::kWords>& k) {
+  uint64_t b1, b2;
+  cuckoo_buckets(key_hash<FMT>(k, t.hash_seed), t.n_buckets, &b1, &b2);
+  const BucketData<FMT> v1 = ld_bucket_data<FMT>(t, b1);
+  const uint32_t w = find_word_in_bucket<FMT>(v1, k);
+  if (w != kEmptyRow || !bucket_full<FMT>(v1)) return w;
+  return find_word_in_bucket<FMT>(ld_bucket_data<FMT>(t, b2), k);
 }
 
 template <int FMT>
 __global__ void verify_kernel(TableView t, const int32_t* ftok, const uint8_t* flen, int64_t n,
-                              int K, BuildFlags* flags) {
+                              int K, const uint8_t* ext, int64_t n_real, BuildFlags* flags) {
   for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n;
        r += (int64_t)gridDim.x * blockDim.x) {
     const auto k = key_of_listed<FMT>(ftok, flen, r, K, t.bits);
-    int err = 0;
-    const int32_t found = cuckoo_lookup<FMT>(t, k, &err);
-    if (found < 0) atomicExch(&flags->full, 1);             // lost in a failed chain
-    else if (found != (int32_t)r) atomicExch(&flags->duplicate, 1);
+    const uint32_t found = lookup_word<FMT>(t, k);
+    if (found == kEmptyRow) atomicExch(&flags->full, 1);     // lost in a failed chain
+    else if (found != entry_word((uint32_t)r, ext, n_real)) atomicExch(&flags->duplicate, 1);
   }
 }
 
@@ -182,11 +207,14 @@ bool is_device_accessible(const void* p) {
 }
 
 
-// Steps 1-4 of the build into t->slots for a list already on the device.
-// Tries kMaxAttempts hash seeds; sets t->view.hash_seed and *out_flags.
-// Synchronizes the stream. Returns SCONE_OK, DUPLICATE_FGRAM, TABLE_FULL or CUDA.
-int build_slots(scone_table* t, const int32_t* d_tok, const uint8_t* d_len, BuildFlags* d_flags,
-                int64_t n, cudaStream_t s, BuildFlags* out_flags) {
+// Steps 1-4 of the build into t->slots for n entries already on the device:
+// the listed f-grams (the first n_real) and then the markers; d_ext (or
+// NULL) holds the f-grams' extension bits. Tries kMaxAttempts hash seeds;
+// sets t->view.hash_seed and *out_flags. Synchronizes the stream. Returns
+// SCONE_OK, DUPLICATE_FGRAM, TABLE_FULL or CUDA.
+int build_slots(scone_table* t, const int32_t* d_tok, const uint8_t* d_len, const uint8_t* d_ext,
+                int64_t n_real, BuildFlags* d_flags, int64_t n, cudaStream_t s,
+                BuildFlags* out_flags) {
   const uint64_t nb = (uint64_t)t->info.n_buckets;
   const uint64_t n_slots = (uint64_t)t->info.n_slots;
   const int K = t->view.K, bits = t->view.bits;
@@ -207,14 +235,16 @@ int build_slots(scone_table* t, const int32_t* d_tok, const uint8_t* d_len, Buil
         insert_kernel<FMT16><<<grid_for(n, th), th, 0, s>>>(t->slots, nb, seed, d_tok, d_len, n,
                                                             K, bits, d_flags);
         fill_keys_kernel<FMT16><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
-            t->slots, n_slots, d_tok, d_len, K, bits);
-        verify_kernel<FMT16><<<grid_for(n, th), th, 0, s>>>(v, d_tok, d_len, n, K, d_flags);
+            t->slots, n_slots, d_tok, d_len, K, bits, d_ext, n_real);
+        verify_kernel<FMT16><<<grid_for(n, th), th, 0, s>>>(v, d_tok, d_len, n, K, d_ext, n_real,
+                                                          d_flags);
       } else {
         insert_kernel<FMT32><<<grid_for(n, th), th, 0, s>>>(t->slots, nb, seed, d_tok, d_len, n,
                                                             K, bits, d_flags);
         fill_keys_kernel<FMT32><<<grid_for((int64_t)n_slots, th), th, 0, s>>>(
-            t->slots, n_slots, d_tok, d_len, K, bits);
-        verify_kernel<FMT32><<<grid_for(n, th), th, 0, s>>>(v, d_tok, d_len, n, K, d_flags);
+            t->slots, n_slots, d_tok, d_len, K, bits, d_ext, n_real);
+        verify_kernel<FMT32><<<grid_for(n, th), th, 0, s>>>(v, d_tok, d_len, n, K, d_ext, n_real,
+                                                          d_flags);
       }
       if (cudaGetLastError() != cudaSuccess ||
           cudaMemcpyAsync(&flags, d_flags, sizeof(BuildFlags), cudaMemcpyDeviceToHost, s) !=
@@ -267,6 +297,14 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
     for (int j = 0; j < n; ++j)
       if (fgram_tok[r * K + j] < 0 || fgram_tok[r * K + j] >= vocab) return SCONE_ERR_INVALID_ARG;
   }
+  // the suffix index: extension bits of the listed f-grams and the markers
+  SuffixIndex si;
+  const bool indexed = wants_suffix_index(fmt, K);
+  if (indexed && n_fgrams > 0) {
+    const int rc = suffix_index(fgram_tok, fgram_len, n_fgrams, K, &si);
+    if (rc != SCONE_OK) return rc;
+  }
+  const int64_t n_entries = n_fgrams + si.n_markers;
   if (!is_device_accessible(T)) return SCONE_ERR_INVALID_ARG;
   const uint16_t* F_dev = reinterpret_cast<const uint16_t*>(F);
   if (n_fgrams > 0) {
@@ -282,8 +320,8 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
     }
   }
 
-  int64_t n_slots = (int64_t)std::ceil((double)n_fgrams / (double)load_factor);
-  if (n_slots < n_fgrams + 1) n_slots = n_fgrams + 1;
+  int64_t n_slots = (int64_t)std::ceil((double)n_entries / (double)load_factor);
+  if (n_slots < n_entries + 1) n_slots = n_entries + 1;
   int64_t n_buckets = (n_slots + kSlotsPerBucket - 1) / kSlotsPerBucket;
   if (n_buckets < 2) n_buckets = 2;   // two distinct candidate buckets
   n_slots = n_buckets * kSlotsPerBucket;
@@ -328,6 +366,7 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   v.bits = bits;
   v.vocab = vocab;
   v.d = d;
+  v.suffix_index = indexed ? 1 : 0;
   scone_table_info& in = t->info;
   in.n_fgrams = n_fgrams;
   in.n_slots = n_slots;
@@ -342,10 +381,13 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   in.table_bytes = n_buckets * bucket;
   in.F_bytes = n_fgrams * (int64_t)d * 2;
   in.T_bytes = (int64_t)vocab * d * 2;
+  in.n_markers = si.n_markers;
+  in.suffix_index = v.suffix_index;
 
   int rc = SCONE_OK;
   int32_t* d_tok = nullptr;
   uint8_t* d_len = nullptr;
+  uint8_t* d_ext = nullptr;
   BuildFlags* d_flags = nullptr;
   BuildFlags flags = {0, 0, 0};
   do {
@@ -354,9 +396,12 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
       rc = SCONE_ERR_CUDA;
       break;
     }
-    if (n_fgrams > 0) {
-      if (cudaMalloc(&d_tok, (size_t)n_fgrams * K * sizeof(int32_t)) != cudaSuccess ||
-          cudaMalloc(&d_len, (size_t)n_fgrams) != cudaSuccess ||
+    if (n_entries > 0) {
+      // entries: the listed f-grams, then the markers
+      const int64_t nm = si.n_markers;
+      if (cudaMalloc(&d_tok, (size_t)n_entries * K * sizeof(int32_t)) != cudaSuccess ||
+          cudaMalloc(&d_len, (size_t)n_entries) != cudaSuccess ||
+          (indexed && cudaMalloc(&d_ext, (size_t)n_fgrams) != cudaSuccess) ||
           cudaMalloc(&d_flags, sizeof(BuildFlags)) != cudaSuccess) {
         rc = SCONE_ERR_NOMEM;
         break;
@@ -364,15 +409,25 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
       if (cudaMemcpyAsync(d_tok, fgram_tok, (size_t)n_fgrams * K * sizeof(int32_t),
                           cudaMemcpyHostToDevice, s) != cudaSuccess ||
           cudaMemcpyAsync(d_len, fgram_len, (size_t)n_fgrams, cudaMemcpyHostToDevice, s) !=
-              cudaSuccess) {
+              cudaSuccess ||
+          (nm > 0 && cudaMemcpyAsync(d_tok + n_fgrams * K, si.marker_tok.data(),
+                                     (size_t)nm * K * sizeof(int32_t), cudaMemcpyHostToDevice,
+                                     s) != cudaSuccess) ||
+          (nm > 0 && cudaMemcpyAsync(d_len + n_fgrams, si.marker_len.data(), (size_t)nm,
+                                     cudaMemcpyHostToDevice, s) != cudaSuccess) ||
+          (d_ext && cudaMemcpyAsync(d_ext, si.ext.data(), (size_t)n_fgrams,
+                                    cudaMemcpyHostToDevice, s) != cudaSuccess)) {
         rc = SCONE_ERR_CUDA;
         break;
       }
     }
-    rc = build_slots(t, d_tok, d_len, d_flags, n_fgrams, s, &flags);
+    // (build_slots synchronizes the stream, so the host vectors outlive the copies)
+    rc = build_slots(t, d_tok, d_len, d_ext, n_fgrams, d_flags, n_entries, s, &flags);
   } while (0);
+  if (rc != SCONE_OK) cudaStreamSynchronize(s);   // copies may still read the host vectors
   if (d_tok) cudaFree(d_tok);
   if (d_len) cudaFree(d_len);
+  if (d_ext) cudaFree(d_ext);
   if (d_flags) cudaFree(d_flags);
   if (rc != SCONE_OK) {
     cudaGetLastError();
@@ -673,8 +728,13 @@ extern "C" int scone_table_rebuild_noalloc(scone_table* t, const int32_t* fgram_
     }
   }
   // the array keeps the previous call's contents: build_slots clears the
-  // flags (which must start at zero) before every attempt
-  rc = build_slots(t, d_tok, d_len, d_flags, n_fgrams, s, &flags);
+  // flags (which must start at zero) before every attempt. The rebuilt
+  // slots carry no suffix index (computing one needs host memory): from here
+  // on launches take every length independently.
+  t->view.suffix_index = 0;
+  t->info.n_markers = 0;
+  t->info.suffix_index = 0;
+  rc = build_slots(t, d_tok, d_len, nullptr, n_fgrams, d_flags, n_fgrams, s, &flags);
   if (rc == SCONE_ERR_CUDA) {
     // the slot array may hold part of the new list while view.F, n_fgrams and
     // the hash seed still describe the old one: one best-effort attempt to

@@ -492,3 +492,62 @@ def test_default_stream_is_the_current_stream():
     with torch.cuda.stream(s):
         assert scone._stream(None) == s.cuda_stream
     assert scone._stream(None) == torch.cuda.current_stream().cuda_stream
+
+
+# ------------------------------------------------- suffix index and the walk
+def _unclosed_case(K, vocab, d, B, L, drop, seed, bad=()):
+    """A workload whose shorter f-grams are partly dropped from the list, so
+    that many suffixes of the longer ones are not f-grams (marker slots)."""
+    quotas = tuple((n, 6000) for n in range(2, K + 1))
+    w = synth.Workload(f"unclosed_k{K}", 60 + K, vocab, 1.05, B, L, quotas, K, d, inject_p=0.05,
+                       n_phrases=512, phrase_len=(K, K + 2))
+    ft, fl, _ = synth.fgram_set(w)
+    keep = ~((fl < K) & (np.random.default_rng(seed).random(fl.shape[0]) < drop))
+    tok = synth.query_tokens(w)
+    for (b, i, x) in bad:
+        tok[b, i] = x
+    return SmallCase(w, fgrams=(ft[keep], fl[keep]), tok=tok)
+
+
+@pytest.mark.parametrize("K,vocab,d,B,L,drop", [
+    (5, 3000, 512, 5, 20011, 0.6),      # warps hold two tiles: rounds inside the copy
+    (4, 3000, 256, 3, 9001, 0.9),
+    (3, 3000, 256, 10, 20011, 0.7),
+])
+def test_suffix_walk_on_unclosed_lists(K, vocab, d, B, L, drop):
+    """The table's marker count is the host index's; the walk over the lengths
+    (AUTO for K = 4, 5 and PIPELINED) and the kernels that look every length
+    up (REGISTERS, SPLIT) all give the oracle's rows, lengths and bytes."""
+    case = _unclosed_case(K, vocab, d, B, L, drop, seed=K)
+    _, _, ml = scone.scone_fgram_suffix_index(case.fg_tok, case.fg_len, K)
+    assert len(ml) > 100
+    table = case.build()
+    info = table.info()
+    assert info["n_markers"] == len(ml)
+    assert info["n_slots"] >= int(np.ceil((info["n_fgrams"] + len(ml)) / 0.5))
+    o_out, o_row, o_len, _ = case.expected()
+    n = case.tok.size
+    for mode in (scone.SCONE_COPY_AUTO, scone.SCONE_COPY_PIPELINED, scone.SCONE_COPY_REGISTERS,
+                 scone.SCONE_COPY_SPLIT):
+        scone.scone_table_set_copy_mode(table, mode)
+        out, row, ln = run_embed(table, case.tok, d)
+        assert np.array_equal(ln, o_len.reshape(n)), mode
+        assert np.array_equal(row, o_row.reshape(n).astype(np.int32)), mode
+        assert np.array_equal(out, o_out.reshape(n, d)), mode
+        out2, _, _ = run_embed(table, case.tok, d, mode="fused_noaux")
+        assert np.array_equal(out2, out)
+    assert (o_len.reshape(n) == K).any()
+    assert scone.scone_status(table) == 0
+
+
+def test_suffix_walk_error_positions():
+    """Invalid tokens (at a position, and inside later positions' windows)
+    end the walk as they end the staged match: zero rows, len 0, status."""
+    bad = ((0, 3, -1), (1, 40, 3000), (2, 20010, 3005), (4, 0, -7), (3, 33, 2999))
+    case = _unclosed_case(5, 3000, 512, 5, 20011, 0.6, seed=5, bad=bad)
+    table = case.build()
+    assert table.info()["n_markers"] > 0
+    out, row, ln = run_embed(table, case.tok, 512)
+    assert_parity(case, out, row, ln)
+    assert (ln == 0).sum() == 4
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE

@@ -282,3 +282,33 @@ def test_rebuild_noalloc_scratch_limit():
     for x, y in zip(a, c):
         assert np.array_equal(x, y)
     table.close()
+
+
+def test_rebuild_noalloc_drops_the_suffix_index():
+    """A built K = 3 table carries a suffix index (here with marker slots, as
+    a third of the 2-grams are left out of the list); the rebuilt table has
+    none, and every copy mode, the pipelined one included, still gives the
+    oracle's answer on both."""
+    fg1_tok, fg1_len, _ = synth.fgram_set(BASE)
+    keep = ~((fg1_len == 2) & (np.arange(fg1_len.shape[0]) % 3 == 0))
+    fg1_tok, fg1_len = fg1_tok[keep], fg1_len[keep]
+    fg2_tok, fg2_len, _ = synth.fgram_set(OTHER)
+    T_host = synth.rows_cpu(synth.T_seed(BASE), BASE.d, np.arange(BASE.vocab))
+    F1_host = synth.rows_cpu(synth.F_seed(BASE), BASE.d, np.arange(fg1_len.shape[0]))
+    F2_host = synth.rows_cpu(synth.F_seed(OTHER), OTHER.d, np.arange(OTHER.n_fgrams))
+    T, F1, F2 = dev_rows(T_host), dev_rows(F1_host), dev_rows(F2_host)
+    tok = synth.query_tokens(BASE)
+    table = scone.scone_table_build(fg1_tok, fg1_len, BASE.K, BASE.vocab, BASE.d, F1, T)
+    _, _, ml = scone.scone_fgram_suffix_index(fg1_tok, fg1_len, BASE.K)
+    assert len(ml) > 0 and table.info()["n_markers"] == len(ml)
+    modes = (scone.SCONE_COPY_AUTO, scone.SCONE_COPY_PIPELINED, scone.SCONE_COPY_REGISTERS)
+    for mode in modes:
+        scone.scone_table_set_copy_mode(table, mode)
+        _same_as_oracle(run_embed(table, tok, BASE.d), fg1_tok, fg1_len, F1_host, T_host, tok)
+    assert _rebuild_via_c_abi(table, fg2_tok, fg2_len, F2) == scone.SCONE_OK
+    assert table.info()["n_markers"] == 0
+    for mode in modes:
+        scone.scone_table_set_copy_mode(table, mode)
+        _same_as_oracle(run_embed(table, tok, BASE.d), fg2_tok, fg2_len, F2_host, T_host, tok)
+    assert scone.scone_status(table) == scone.SCONE_OK
+    table.close()
