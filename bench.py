@@ -167,7 +167,8 @@ def measured_peaks():
 
 
 EMBED_SOURCES = ("scone_embed.cu", "scone_device.cuh", "scone_host.h")
-PIPE_SOURCES = ("scone_pipe.cu", "scone_embed.cu", "scone_device.cuh", "scone_host.h")
+PIPE_SOURCES = ("scone_pipe.cu", "scone_walk.cuh", "scone_embed.cu", "scone_device.cuh",
+                "scone_host.h")
 DISCOVER_SOURCES = ("scone_discover.cu", "scone_device.cuh", "scone_host.h")
 
 
@@ -1106,7 +1107,9 @@ def bench_mixed(args, world, rank, local):
             "traffic": None,
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
             "algorithmic_bytes_per_launch": bytes_launch,
-            "kernel": "varlen_embed_kernel (fused match + gather over packed sequences)",
+            "kernel": ("varlen_walk_kernel (fused match + gather over packed sequences, the "
+                       "lengths walked over the suffix index)" if table.info()["suffix_index"]
+                       else "varlen_embed_kernel (fused match + gather over packed sequences)"),
         },
         "e2e": {
             "value": world * n_tok / (e2e_ms * 1e-3),

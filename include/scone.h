@@ -223,7 +223,9 @@ int scone_table_get_info(const scone_table* table, scone_table_info* info);
  */
 int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
 
-/* How scone_embed moves rows (a tuning knob; results are identical). */
+/* How scone_embed moves rows (a tuning knob; results are identical). scone_embed_varlen
+   reads it too: REGISTERS keeps its register kernel, AUTO and PIPELINED take the walk
+   over the suffix index where that applies, BULK and SPLIT act as REGISTERS there. */
 enum scone_copy_mode {
   SCONE_COPY_AUTO = 0,       /* the library picks per call: PIPELINED where it applies and the
                                 table has a suffix index or 3 < K <= 5, REGISTERS otherwise */

@@ -193,12 +193,14 @@ def test_error_positions(case):
     st.close()
 
 
-def ragged_continued(w, seed, rounds=6, per_seq=400):
+def ragged_continued(w, seed, rounds=6, per_seq=400, mode=None, fgrams=None):
     """Six rounds of ragged chunks (some empty) that continue S slots, the
     last round flushing each sequence's rest; every chunk's rows match the
     oracle on the sequence's whole prefix."""
-    c = SmallCase(w, tok=np.zeros((1, 1), np.int32))
+    c = SmallCase(w, fgrams=fgrams, tok=np.zeros((1, 1), np.int32))
     c.table = c.build()
+    if mode is not None:
+        scone.scone_table_set_copy_mode(c.table, mode)
     S, H = 6, w.K - 1
     st = scone.scone_decode_create(c.table, np.zeros((S, H), np.int32), np.zeros(S, np.int32))
     full = [synth.zipf_tokens(w, seed + s, per_seq) for s in range(S)]
@@ -241,14 +243,32 @@ def ragged_continued(w, seed, rounds=6, per_seq=400):
     return matched, info
 
 
-def test_k5_ragged_and_continued():
+@pytest.mark.parametrize("mode", [scone.SCONE_COPY_AUTO, scone.SCONE_COPY_REGISTERS])
+def test_k5_ragged_and_continued(mode):
     """K = 5 over the stress law, with phrases injected often enough that 4-
-    and 5-gram matches occur (and cross chunk boundaries)."""
+    and 5-gram matches occur (and cross chunk boundaries); AUTO walks the
+    lengths over the table's suffix index, REGISTERS looks every length up."""
     w5 = synth.WORKLOADS["stress_k5"].scaled("varlen_k5", B=1, L=64, d=64,
                                              quotas=((2, 3000), (3, 3000), (4, 1500), (5, 1500)),
                                              inject_p=0.05, n_phrases=256, phrase_len=(5, 7))
-    matched, _ = ragged_continued(w5, 900)
+    matched, info = ragged_continued(w5, 900, mode=mode)
     assert matched[4] and matched[5]
+    assert info["suffix_index"] == 1
+
+
+@pytest.mark.parametrize("mode", [scone.SCONE_COPY_AUTO, scone.SCONE_COPY_REGISTERS])
+def test_unclosed_list_ragged_and_continued(mode):
+    """A K = 4 list with half of its shorter f-grams left out, so that the
+    table holds many marker slots: the walk and the register kernel both
+    follow the oracle over ragged, continued chunks."""
+    w = synth.Workload("varlen_unclosed", 71, 3000, 1.05, 1, 64,
+                       ((2, 3000), (3, 3000), (4, 3000)), 4, 64, inject_p=0.05, n_phrases=256,
+                       phrase_len=(4, 6))
+    ft, fl, _ = synth.fgram_set(w)
+    keep = ~((fl < 4) & (np.arange(fl.shape[0]) % 2 == 0))
+    matched, info = ragged_continued(w, 1300, mode=mode, fgrams=(ft[keep], fl[keep]))
+    assert info["n_markers"] > 100
+    assert matched[2] and matched[4]
 
 
 @pytest.mark.parametrize("name,K,vocab,slot_bytes", [
@@ -266,3 +286,60 @@ def test_key_formats_ragged_and_continued(name, K, vocab, slot_bytes):
     matched, info = ragged_continued(w, 1000 + K)
     assert info["slot_bytes"] == slot_bytes
     assert matched[2] and matched[K]
+
+
+@pytest.mark.parametrize("K,mode", [(3, scone.SCONE_COPY_AUTO), (3, scone.SCONE_COPY_REGISTERS),
+                                    (5, scone.SCONE_COPY_AUTO), (5, scone.SCONE_COPY_REGISTERS)])
+def test_many_short_chunks_across_warps(K, mode):
+    """Thousands of chunks of 0..5 tokens continuing as many slots, in three
+    launches: the chunks' first K-1 positions (the readers of a slot's old
+    history) fall across warp boundaries many times per launch, and each
+    slot's history is rewritten in the launch that reads it. Every position
+    equals the oracle on its sequence's whole prefix."""
+    quotas = tuple((n, 2000) for n in range(2, K + 1))
+    w = synth.Workload(f"short_chunks_k{K}", 90 + K, 2000, 1.05, 1, 64, quotas, K, 64,
+                       inject_p=0.05, n_phrases=256, phrase_len=(K, K + 2))
+    c = SmallCase(w, tok=np.zeros((1, 1), np.int32))
+    c.table = c.build()
+    scone.scone_table_set_copy_mode(c.table, mode)
+    S, H, rounds = 6000, K - 1, 3
+    st = scone.scone_decode_create(c.table, np.zeros((S, H), np.int32), np.zeros(S, np.int32))
+    rng = np.random.default_rng(K)
+    full = [synth.zipf_tokens(w, 5000 + s, 5 * rounds) for s in range(S)]
+    pos = np.zeros(S, np.int64)
+    for rnd in range(rounds):
+        order = rng.permutation(S)                 # slots in a new order every launch
+        lens = rng.integers(0, 6, S)
+        chunks = [full[s][pos[s]:pos[s] + lens[k]] for k, s in enumerate(order)]
+        cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        flat = np.concatenate(chunks).astype(np.int32)
+        n = flat.size
+        out = torch.empty((n, w.d), dtype=torch.int16, device=DEV)
+        row = torch.empty(n, dtype=torch.int32, device=DEV)
+        ln = torch.empty(n, dtype=torch.uint8, device=DEV)
+        scone.scone_embed_varlen(c.table, torch.from_numpy(flat).to(DEV),
+                                 torch.from_numpy(cu).to(DEV), out, state=st,
+                                 seq_slot=torch.from_numpy(order.astype(np.int32)).to(DEV),
+                                 row=row, len=ln)
+        torch.cuda.synchronize()
+        g_out = out.cpu().numpy().view(np.uint16)
+        g_row, g_len = row.cpu().numpy(), ln.cpu().numpy()
+        for k, s in enumerate(order):
+            if lens[k] == 0:
+                continue
+            a, b = int(pos[s]), int(pos[s] + lens[k])
+            e_out, e_row, e_len, _ = c.oracle.embed(np.asarray(full[s][:b], np.int32)[None, :],
+                                                    c.F, c.T)
+            sl = slice(cu[k], cu[k + 1])
+            assert np.array_equal(g_len[sl], e_len[0, a:b]), (rnd, s)
+            assert np.array_equal(g_row[sl], e_row[0, a:b].astype(np.int32)), (rnd, s)
+            assert np.array_equal(g_out[sl], e_out[0, a:b]), (rnd, s)
+            pos[s] = b
+    hist, hlen = scone.scone_decode_get_history(st)
+    for s in range(S):                         # the histories the launches left behind
+        m = int(min(H, pos[s]))
+        assert hlen[s] == m
+        assert np.array_equal(hist[s, H - m:], np.asarray(full[s][pos[s] - m:pos[s]]))
+    assert scone.scone_status(c.table) == 0
+    st.close()
+    c.table.close()
