@@ -225,7 +225,9 @@ int scone_table_set_probe_limit(scone_table* table, int64_t max_buckets);
 
 /* How scone_embed moves rows (a tuning knob; results are identical). scone_embed_varlen
    reads it too: REGISTERS keeps its register kernel, AUTO and PIPELINED take the walk
-   over the suffix index where that applies, BULK and SPLIT act as REGISTERS there. */
+   over the suffix index where that applies, BULK and SPLIT act as REGISTERS there. So
+   does scone_match: REGISTERS looks every length up, any other mode walks the lengths
+   on a table with a suffix index. */
 enum scone_copy_mode {
   SCONE_COPY_AUTO = 0,       /* the library picks per call: PIPELINED where it applies and the
                                 table has a suffix index or 3 < K <= 5, REGISTERS otherwise */
@@ -248,10 +250,14 @@ int scone_table_set_copy_mode(scone_table* table, int32_t mode);
  * scone_match — the selection step of Algorithm 1 (Sec. 3): for each
  * position, the length of the longest f-gram ending there and its row of F.
  * Probes lengths 2..min(K, i+1), i.e. at most K-1 lookups per token, the
- * bound Sec. 4.3 states ("up to four queries per token" for K = 5). All
- * lengths read their first buckets in one round trip; the lengths whose
- * first bucket is full without the key, and that are longer than the best
- * first-round hit, read their second buckets in a second one. Async.
+ * bound Sec. 4.3 states ("up to four queries per token" for K = 5). On a
+ * table with a suffix index and tokens in device memory the lengths are
+ * walked in turn, stopping at the first absent or unextended window (fewer
+ * lookups; see the copy modes).
+ * Otherwise all lengths read their first buckets in one round trip, and the
+ * lengths whose first bucket is full without the key, and that are longer
+ * than the best first-round hit, read their second buckets in a second one.
+ * Async.
  *
  *  tok  int32 [B * L]; row int32 [B * L] (F row, or -1 when T is used or on
  *  error); len uint8 [B * L] or NULL (n in 2..K for an f-gram, 1 for the

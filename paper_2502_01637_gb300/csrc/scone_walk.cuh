@@ -204,3 +204,53 @@ constexpr int kWalkMinBlocks = 3;
 constexpr int kWalkFirst = 8;
 
 }  // namespace scone
+
+namespace scone {
+
+// The walk for one position in one thread, with blocking loads (for kernels
+// that hide latency with many threads instead of interleaving a copy, such
+// as the match kernel): tokens, then n = 2, 3, ... one bucket (or two) at a
+// time. Same result, len and err as match_position; the default probe
+// limit is assumed (the callers take the all-length lookups otherwise).
+template <int KT>
+__device__ __forceinline__ int32_t walk_position(const TableView& t,
+                                                 const int32_t* __restrict__ tok, int64_t p,
+                                                 int32_t i, int32_t x, int* len, int* err) {
+  if (!valid_token(x, t.vocab)) {
+    *err = SCONE_ERR_TOKEN_RANGE;
+    *len = 0;
+    return -1;
+  }
+  int nmax = t.K < i + 1 ? t.K : i + 1;
+  int32_t w[KT];
+  w[0] = x;
+#pragma unroll
+  for (int j = 1; j < KT; ++j) w[j] = (j < nmax) ? __ldg(tok + p - j) : 0;
+  // a window is usable only if all its tokens are valid
+  int nvalid = 1;
+#pragma unroll
+  for (int j = 1; j < KT; ++j)
+    if (nvalid == j && j < nmax && valid_token(w[j], t.vocab)) nvalid = j + 1;
+  nmax = nvalid;
+  int32_t row = -1;
+  *len = 1;
+  for (int n = 2; n <= nmax; ++n) {
+    const auto k = window_key<FMT16, KT>(w, n, t.bits);
+    uint64_t b1, b2;
+    cuckoo_buckets(key_hash<FMT16>(k, t.hash_seed), t.n_buckets, &b1, &b2);
+    const BucketData<FMT16> v = ld_bucket_data<FMT16>(t, b1);
+    uint32_t word = find_word_in_bucket<FMT16>(v, k);
+    if (word == kEmptyRow && bucket_full<FMT16>(v))
+      word = find_word_in_bucket<FMT16>(ld_bucket_data<FMT16>(t, b2), k);
+    if (word == kEmptyRow) break;
+    const int32_t r = row_of_word(word);
+    if (r >= 0) {
+      row = r;
+      *len = n;
+    }
+    if (!(word & kExtBit)) break;
+  }
+  return row;
+}
+
+}  // namespace scone
