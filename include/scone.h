@@ -272,6 +272,35 @@ int scone_match(const scone_table* table, const int32_t* tok, int32_t B, int32_t
                 int32_t* row, uint8_t* len, void* stream);
 
 /*
+ * scone_prescan — the training-time pre-scan of Appendix F (tag every token
+ * of a corpus with its longest f-gram's length and row) for a corpus in host
+ * memory, staged through HBM: chunks of whole sequences are copied in, tagged
+ * by the match kernel (scone_match on device memory) and their tags copied
+ * out, each on its own stream, so the host link carries bulk copies in both
+ * directions while the kernel works on the chunk before. Same results as
+ * scone_match on the host addresses.
+ *
+ *  tok        host int32 [B * L]; row host int32 [B * L]; len host uint8
+ *             [B * L] or NULL. Pinned memory (scone_host_alloc or registered)
+ *             lets the copies overlap; pageable memory works, more slowly.
+ *  B, L       B sequences of L >= 1 tokens (B * L may exceed 2^31).
+ *  chunk_tokens  tokens per chunk, rounded down to whole sequences (at least
+ *             one); 0 selects 32 Mi. The first call on a table allocates two
+ *             chunks of device buffers (9 bytes per token each, 5 without
+ *             len) and three streams, which the table keeps (a later call
+ *             with larger chunks, or with len after calls without it,
+ *             reallocates them) and scone_table_destroy frees.
+ *  stream     work queued on it before the call comes first; the call
+ *             returns when the tags are in host memory (synchronous).
+ *
+ * Calls on one table must not overlap (they share its buffers). Device-
+ * detected errors are recorded in the table's status word as for
+ * scone_match. Errors: INVALID_ARG, NOMEM (the device buffers), CUDA.
+ */
+int scone_prescan(scone_table* table, const int32_t* tok, int64_t B, int32_t L, int32_t* row,
+                  uint8_t* len, int64_t chunk_tokens, void* stream);
+
+/*
  * scone_fgram_discover — constructs V_fgram from a corpus: Algorithm 3
  * ("Constructing a set of f-grams", Appendix A) by the K-1 counting scans of
  * Sec. 3.2. C_w is the number of windows equal to the n-gram w, n = 2..K,

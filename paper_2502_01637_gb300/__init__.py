@@ -47,7 +47,7 @@ SCONE_FGRAM_POS_ROTARY = 1
 EXPORTS = ("scone_table_build", "scone_table_destroy", "scone_table_rebuild_noalloc",
            "scone_fgram_suffix_index",
            "scone_table_get_info", "scone_table_set_probe_limit", "scone_table_set_copy_mode",
-           "scone_match", "scone_embed_gather", "scone_embed",
+           "scone_match", "scone_prescan", "scone_embed_gather", "scone_embed",
            "scone_decode_create", "scone_decode_step", "scone_decode_get_history",
            "scone_decode_destroy", "scone_status", "scone_host_alloc", "scone_host_free",
            "scone_embed_varlen", "scone_rowstore_open", "scone_rowstore_gather",
@@ -126,6 +126,7 @@ def load_library():
     lib.scone_table_set_probe_limit.argtypes = [_vp, _i64]
     lib.scone_table_set_copy_mode.argtypes = [_vp, _i32]
     lib.scone_match.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp]
+    lib.scone_prescan.argtypes = [_vp, _vp, _i64, _i32, _vp, _vp, _i64, _vp]
     lib.scone_embed_gather.argtypes = [_vp, _vp, _vp, _i64, _vp, _vp]
     lib.scone_embed.argtypes = [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]
     lib.scone_embed_varlen.argtypes = [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]
@@ -193,6 +194,8 @@ def _ptr(t) -> Optional[int]:
         return None
     if isinstance(t, int):
         return t
+    if isinstance(t, HostBuffer):
+        return t.ptr
     if isinstance(t, np.ndarray):
         assert t.flags["C_CONTIGUOUS"]
         return t.ctypes.data
@@ -341,6 +344,15 @@ def scone_match(table: Table, tok, row, len=None, stream=None) -> None:
     B, L = _bl(tok)
     _check(load_library().scone_match(table.handle, _ptr(tok), B, L, _ptr(row), _ptr(len),
                                       _stream(stream)), "scone_match")
+
+
+def scone_prescan(table: Table, tok, B: int, L: int, row, len=None, chunk_tokens: int = 0,
+                  stream=None) -> None:
+    """Tags a corpus in host memory (tok, row, len: host addresses or buffers of
+    B * L entries), staged through HBM in chunks of whole sequences; returns
+    when the tags are in host memory."""
+    _check(load_library().scone_prescan(table.handle, _ptr(tok), B, L, _ptr(row), _ptr(len),
+                                        chunk_tokens, _stream(stream)), "scone_prescan")
 
 
 def scone_embed_gather(table: Table, tok, row, out, stream=None) -> None:

@@ -8,6 +8,11 @@
 #include "scone.h"
 #include "scone_device.cuh"
 
+namespace scone {
+struct PrescanWork;   // scone_prescan's device buffers, streams and events (scone_prescan.cu)
+void prescan_release(PrescanWork* w);
+}  // namespace scone
+
 struct scone_table {
   int device = 0;
   int fmt = scone::FMT16;
@@ -17,6 +22,7 @@ struct scone_table {
   int* status_host_dev = nullptr;  // its device address
   uint8_t* zero_row = nullptr;  // d * 2 zero bytes: the source of error positions (bulk copies)
   int copy_mode = SCONE_COPY_AUTO;
+  scone::PrescanWork* prescan = nullptr;  // made by the first scone_prescan call, kept
   scone::TableView view{};
   scone_table_info info{};
 };

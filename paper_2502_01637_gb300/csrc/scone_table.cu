@@ -445,6 +445,7 @@ extern "C" int scone_table_destroy(scone_table* t) {
   cudaGetDevice(&prev);
   if (prev != t->device) cudaSetDevice(t->device);
   if (t->slots || t->status || t->zero_row) cudaDeviceSynchronize();
+  if (t->prescan) prescan_release(t->prescan);
   if (t->slots) cudaFree(t->slots);
   if (t->status) cudaFree(t->status);
   if (t->status_host) cudaFreeHost(t->status_host);

@@ -551,3 +551,42 @@ def test_suffix_walk_error_positions():
     assert_parity(case, out, row, ln)
     assert (ln == 0).sum() == 4
     assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+
+
+# ------------------------------------------------- pre-scan staged through HBM
+def test_prescan_staged_equals_oracle():
+    """scone_prescan on a corpus in pinned host memory, staged through HBM in
+    chunks of whole sequences (default size, several chunks with a short last
+    one, one sequence per chunk when a chunk is shorter than a sequence, and
+    no len output): the oracle's rows and lengths, the same as scone_match on
+    the host addresses."""
+    w = TINY.scaled("prescan_staged", B=37, L=1000)
+    case = SmallCase(w)
+    table = case.build()
+    n = case.tok.size
+    corpus = scone.scone_host_alloc(n * 4)
+    corpus.numpy(np.int32)[:n] = case.tok.reshape(-1)
+    rows, lens = scone.scone_host_alloc(n * 4), scone.scone_host_alloc(n)
+    _, o_row, o_len, _ = case.expected()
+    for chunk in (0, 5000, 999, 1000):
+        rows.numpy(np.int32)[:n] = -7
+        lens.numpy(np.uint8)[:n] = 99
+        scone.scone_prescan(table, corpus, w.B, w.L, rows, lens, chunk_tokens=chunk)
+        assert np.array_equal(rows.numpy(np.int32)[:n], o_row.reshape(-1).astype(np.int32)), chunk
+        assert np.array_equal(lens.numpy(np.uint8)[:n], o_len.reshape(-1)), chunk
+    rows.numpy(np.int32)[:n] = -7
+    scone.scone_prescan(table, corpus, w.B, w.L, rows, None, chunk_tokens=7000)
+    assert np.array_equal(rows.numpy(np.int32)[:n], o_row.reshape(-1).astype(np.int32))
+    zc_rows, zc_lens = scone.scone_host_alloc(n * 4), scone.scone_host_alloc(n)
+    lib = scone.load_library()
+    assert lib.scone_match(table.handle, corpus.ptr, w.B, w.L, zc_rows.ptr, zc_lens.ptr,
+                           torch.cuda.current_stream().cuda_stream) == 0
+    torch.cuda.synchronize()
+    assert np.array_equal(zc_rows.numpy(np.int32)[:n], rows.numpy(np.int32)[:n])
+    assert scone.scone_status(table) == 0
+    lib_inv = scone.SCONE_ERR_INVALID_ARG
+    assert lib.scone_prescan(table.handle, corpus.ptr, w.B, 0, rows.ptr, None, 0, None) == lib_inv
+    assert lib.scone_prescan(table.handle, None, w.B, w.L, rows.ptr, None, 0, None) == lib_inv
+    for b in (corpus, rows, lens, zc_rows, zc_lens):
+        b.free()
+    table.close()
