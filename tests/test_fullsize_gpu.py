@@ -46,10 +46,10 @@ def check_sampled(w, tok, row, ln, out, pos):
     assert np.array_equal(got, exp), "output bytes differ from the oracle's rows"
 
 
-def check_all_positions(w, tok, tok_d, row_d, ln_d, out, F, T):
+def check_all_positions(w, tok, tok_d, row_d, ln_d, out, F, T, fgrams=None):
     """Every position against the oracle: rows and lengths element by
     element, output rows against the rows at the oracle's ids."""
-    o = oracle.Oracle(*synth.fgram_set(w)[:2], w.K, w.vocab)
+    o = oracle.Oracle(*(fgrams if fgrams is not None else synth.fgram_set(w)[:2]), w.K, w.vocab)
     o_row, o_len, _, rc = o.select(tok)
     assert rc == 0
     o_row, o_len = o_row.reshape(-1), o_len.reshape(-1)
@@ -93,6 +93,36 @@ def test_fullsize_prefill(name):
     assert torch.equal(out, out2)
     pos = sample_positions(w.B, w.L, w.K, 6000, seed=len(name))
     check_sampled(w, tok, row_d.cpu().numpy(), ln_d.cpu().numpy(), out, pos)
+    table.close()
+
+
+def test_fullsize_stress_k5_with_markers():
+    """stress_k5 with every third f-gram shorter than K left out of the list,
+    so that the table's suffix index holds hundreds of thousands of marker
+    slots (suffixes of listed f-grams that are not listed): every position of
+    the full batch, through the walk the benchmark's kernel takes, against the
+    oracle of the shortened list."""
+    w = synth.WORKLOADS["stress_k5"]
+    fg_tok, fg_len, _ = synth.fgram_set(w)
+    keep = ~((fg_len < w.K) & (np.arange(fg_len.shape[0]) % 3 == 0))
+    ft, fl = fg_tok[keep], fg_len[keep]
+    F_all = gpu_rows(synth.F_seed(w), w.n_fgrams, w.d)
+    F = F_all.index_select(0, torch.from_numpy(np.flatnonzero(keep)).to(DEV))
+    del F_all
+    T = gpu_rows(synth.T_seed(w), w.vocab, w.d)
+    table = scone.scone_table_build(ft, fl, w.K, w.vocab, w.d, F, T, load_factor=w.load_factor)
+    info = table.info()
+    assert info["suffix_index"] == 1 and info["n_markers"] > 100_000
+    tok = synth.query_tokens(w)
+    tok_d = torch.from_numpy(tok).to(DEV)
+    n = tok.size
+    out = torch.empty((n, w.d), dtype=torch.int16, device=DEV)
+    row_d = torch.empty(n, dtype=torch.int32, device=DEV)
+    ln_d = torch.empty(n, dtype=torch.uint8, device=DEV)
+    scone.scone_embed(table, tok_d, out, row_d, ln_d)          # AUTO: the walk
+    assert scone.scone_status(table) == 0
+    hist = check_all_positions(w, tok, tok_d, row_d, ln_d, out, F, T, fgrams=(ft, fl))
+    assert (hist[1:] > 0).all(), f"some length never occurs: {hist}"
     table.close()
 
 
