@@ -170,6 +170,7 @@ EMBED_SOURCES = ("scone_embed.cu", "scone_device.cuh", "scone_host.h")
 PIPE_SOURCES = ("scone_pipe.cu", "scone_walk.cuh", "scone_embed.cu", "scone_device.cuh",
                 "scone_host.h")
 DISCOVER_SOURCES = ("scone_discover.cu", "scone_device.cuh", "scone_host.h")
+VARLEN_SOURCES = ("scone_varlen.cu", "scone_walk.cuh", "scone_device.cuh", "scone_host.h")
 
 
 def kernel_source_hash(files=EMBED_SOURCES) -> str:
@@ -1123,7 +1124,8 @@ def bench_mixed(args, world, rank, local):
             "peak": hbm,
             "unit": "GB/s",
             "frac": achieved / hbm,
-            "traffic": None,
+            "traffic": (profiled_traffic("mixed_serving", "varlen_walk_kernel", VARLEN_SOURCES)
+                        if table.info()["suffix_index"] else None),
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)",
             "algorithmic_bytes_per_launch": bytes_launch,
             "kernel": ("varlen_walk_kernel (fused match + gather over packed sequences, the "
