@@ -1417,7 +1417,13 @@ def bench_discover(args, world, rank, local):
     S = w.n_fgrams
     t0 = time.time()
     tok_np = synth.query_tokens(w)
-    host_tok = torch.from_numpy(tok_np).pin_memory()
+    # the corpus in pinned host memory from scone_host_alloc (a huge-page
+    # mapping): torch's pin_memory buffers (small pages) copied in at 15-112
+    # GB/s on some calls instead of 211, from address translation of the pages
+    host_buf = scone.scone_host_alloc(tok_np.nbytes)
+    host_np = host_buf.numpy(np.int32)[:tok_np.size].reshape(tok_np.shape)
+    host_np[:] = tok_np
+    host_tok = torch.from_numpy(host_np)
     tok = host_tok.to(dev)
     out_tok = torch.empty((S, w.K), dtype=torch.int32, device=dev)
     out_len = torch.empty(S, dtype=torch.uint8, device=dev)
@@ -1449,18 +1455,24 @@ def bench_discover(args, world, rank, local):
     st = stats[-1]
 
     # end to end: corpus from pinned host memory, the call, the list back to the host
-    host_out = [torch.empty_like(t, device="cpu").pin_memory() for t in (out_tok, out_len, out_cnt)]
-    e2e_t = []
+    out_bufs = [scone.scone_host_alloc(t.numel() * t.element_size()) for t in (out_tok, out_len, out_cnt)]
+    host_out = [torch.from_numpy(b.numpy(np.uint8)[:t.numel() * t.element_size()]).view(t.dtype)
+                .reshape(t.shape) for b, t in zip(out_bufs, (out_tok, out_len, out_cnt))]
+    e2e_t, e2e_h2d = [], []
     for k in range(max(2, min(args.steps, 5))):
         torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t1 = time.perf_counter()
+        e0.record(stream)
         tok.copy_(host_tok, non_blocking=True)
+        e1.record(stream)
         ft, fl, fc, _ = step(tok)
         m = fl.shape[0]
         for h, d in zip(host_out, (ft, fl, fc)):
             h[:m].copy_(d, non_blocking=True)
         torch.cuda.synchronize()
         e2e_t.append(time.perf_counter() - t1)
+        e2e_h2d.append(e0.elapsed_time(e1))
     e2e_ms = max_over_ranks(1e3 * statistics.mean(e2e_t), world)
     m = int(st["frequent"][2] + sum(st["frequent"][3:]))
     n_sel = min(S, m)
@@ -1515,6 +1527,7 @@ def bench_discover(args, world, rank, local):
                 "what": "pinned corpus -> device, scone_fgram_discover, f-gram list -> "
                         "pinned host",
                 "per_call_ms": [round(1e3 * x, 2) for x in e2e_t],
+                "corpus_h2d_ms": [round(x, 2) for x in e2e_h2d],
                 "spread": max(e2e_t) / min(e2e_t) - 1.0},
         # per call: bin, hotflush, bincount, flagbin, unsort, scan and assign
         # per scan; then 4 radix-select histograms (only when the cut falls
