@@ -55,3 +55,28 @@ def test_reference_line_keys():
 def test_reference_line_other_workload_is_explicit():
     d = run_bench("--impl", "reference", "--workload", "discover", "--steps", "1")
     assert d["impl"] == "reference" and "unavailable" in d
+
+
+def test_kernel_names_and_profile_lookup():
+    """The roofline's kernel follows the launch the copy mode and the table's
+    suffix index select, and a profile summary counts only while its source
+    hash matches the current sources."""
+    import bench
+
+    assert bench.embed_kernel_name("auto", 3, True).startswith("embed_walk_kernel")
+    assert bench.embed_kernel_name("auto", 5, True).startswith("embed_walk_kernel")
+    assert bench.embed_kernel_name("auto", 5, False).startswith("embed_pipe_kernel")
+    assert bench.embed_kernel_name("auto", 3, False).startswith("embed_kernel")
+    assert bench.embed_kernel_name("registers", 3, True).startswith("embed_kernel")
+    assert bench.embed_kernel_name("pipelined", 3, True).startswith("embed_walk_kernel")
+    assert bench.embed_kernel_name("split", 5, True).startswith("embed_split_kernel")
+    # the committed summaries of the bench's kernels were taken on these sources
+    for wl in ("large_hbm", "stress_k5", "prefill_1b"):
+        t, note = bench.profiled_traffic(wl, "embed_walk_kernel", bench.PIPE_SOURCES,
+                                         with_note=True)
+        assert t is not None and t > 0, wl
+    assert bench.profiled_traffic("mixed_serving", "varlen_walk_kernel",
+                                  bench.VARLEN_SOURCES) is not None
+    # an unknown summary reads as no traffic
+    assert bench.profiled_traffic("no_such_workload", "embed_walk_kernel",
+                                  bench.PIPE_SOURCES) is None
