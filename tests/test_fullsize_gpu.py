@@ -245,8 +245,9 @@ def test_fullsize_offload_decode():
 def test_prescan_host_mapped_corpus():
     """The training-time pre-scan (Appendix F): scone_match reads a corpus
     held in host memory and writes its tags (row, len) to host memory. Tags
-    equal those of the same launch on device copies, and every position
-    equals the oracle."""
+    equal those of the same launch on device copies (where the match walks
+    the lengths) and of scone_prescan (staged through HBM), and every
+    position equals the oracle."""
     w = synth.WORKLOADS["prescan"].scaled("prescan_test", B=4096)   # 8.4M tokens
     fg_tok, fg_len, _ = synth.fgram_set(w)
     n = w.B * w.L
@@ -275,6 +276,13 @@ def test_prescan_host_mapped_corpus():
     assert np.array_equal(h_len, o_len.reshape(-1))
     assert np.array_equal(h_row, o_row.reshape(-1).astype(np.int32))
     assert (np.bincount(h_len, minlength=4)[1:] > 0).all()
+    # the staged pre-scan (chunks through HBM, eight of them here) writes the same tags
+    tags_len.numpy(np.uint8)[:n] = 99
+    tags_row.numpy(np.int32)[:n] = -7
+    scone.scone_prescan(table, corpus, w.B, w.L, tags_row, tags_len, chunk_tokens=1 << 20)
+    assert np.array_equal(tags_len.numpy(np.uint8)[:n], h_len)
+    assert np.array_equal(tags_row.numpy(np.int32)[:n], h_row)
+    assert scone.scone_status(table) == 0
     table.close()
     for b in (corpus, tags_len, tags_row):
         b.free()
