@@ -586,7 +586,11 @@ int scone_decode_destroy(scone_decode* state);
 
 /*
  * scone_status: synchronizes `stream`, returns the first device-detected
- * error recorded since the last call (SCONE_OK if none) and clears it.
+ * error recorded since the last call (SCONE_OK if none) and clears it. The
+ * kernel that records an error also writes it to a host-mapped word of the
+ * table, so when no error was recorded the call is the sync and one read of
+ * host memory; after an error it launches one 1-thread kernel that moves the
+ * status word into that host word and clears it.
  */
 int scone_status(const scone_table* table, void* stream);
 

@@ -83,7 +83,7 @@ __global__ void __launch_bounds__(kBulkThreads)
         int len = 0, err = 0;
         const int32_t r = match_position<FMT, KT>(t, tok, p, (int32_t)(p % L), x, &len, &err);
         if (err) {
-          record_error(t.status, err);
+          record_error(t, err);
         } else {
           src = r >= 0 ? static_cast<const void*>(t.F + (int64_t)r * t.d)
                        : static_cast<const void*>(t.T + (int64_t)x * t.d);
@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kBulkThreads)
         while (!failed && !mbar_try_wait(saddr(&full[s]), parity)) {
           if (++spins >= kSpinLimit) {
             failed = true;
-            record_error(t.status, SCONE_ERR_CUDA);
+            record_error(t, SCONE_ERR_CUDA);
           }
         }
         if (!failed) {

@@ -119,8 +119,8 @@ __global__ void __launch_bounds__(kDecThreads)
       hist_len[s] = h + 1 < H ? h + 1 : H;
       if (row_out) row_out[s] = r;
       if (len_out) len_out[s] = (uint8_t)len;
-      if (!xvalid) record_error(t.status, SCONE_ERR_TOKEN_RANGE);
-      else if (probe_err) record_error(t.status, SCONE_ERR_PROBE_LIMIT);
+      if (!xvalid) record_error(t, SCONE_ERR_TOKEN_RANGE);
+      else if (probe_err) record_error(t, SCONE_ERR_PROBE_LIMIT);
       src_s[warp][0] = src;
     }
     __syncwarp();
@@ -138,7 +138,7 @@ __global__ void __launch_bounds__(kDecThreads)
             bulk_commit();
             phase ^= 1;
           } else {
-            record_error(t.status, SCONE_ERR_CUDA);
+            record_error(t, SCONE_ERR_CUDA);
             broken = true;
           }
         }

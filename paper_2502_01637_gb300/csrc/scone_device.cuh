@@ -83,6 +83,7 @@ struct TableView {
   const uint16_t* F;         // device-accessible address of F (HBM or host-mapped)
   const uint16_t* T;
   int* status;               // sticky first device-detected error
+  int* status_mirror;        // device address of a host-mapped copy of it, or NULL
   int32_t K;
   int32_t bits;
   int32_t vocab;
@@ -252,8 +253,13 @@ __device__ __forceinline__ int32_t cuckoo_lookup_eager(const TableView& t,
   return find_in_bucket<FMT>(v2, k);
 }
 
-__device__ __forceinline__ void record_error(int* status, int code) {
-  if (*reinterpret_cast<volatile int*>(status) == 0) atomicCAS(status, 0, code);
+// Records a device-detected error: the first one wins the table's status
+// word, and the thread that wins also writes it to the host-mapped mirror, so
+// that scone_status finds "no error" by reading host memory alone.
+__device__ __forceinline__ void record_error(const TableView& t, int code) {
+  if (*reinterpret_cast<volatile int*>(t.status) == 0 && atomicCAS(t.status, 0, code) == 0 &&
+      t.status_mirror)
+    *reinterpret_cast<volatile int*>(t.status_mirror) = code;
 }
 
 __device__ __forceinline__ bool valid_token(int32_t x, int32_t vocab) {

@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(kThreads)
     const int32_t x = __ldg(tok + p);
     int len = 0, err = 0;
     const int32_t r = match_position<FMT, KT>(t, tok, p, pos_in_seq(p, L), x, &len, &err);
-    if (err) record_error(t.status, err);
+    if (err) record_error(t, err);
     row_out[p] = r;
     if (len_out) len_out[p] = (uint8_t)len;
   }
@@ -104,7 +104,7 @@ __global__ void __launch_bounds__(kThreads)
     const int32_t x = __ldg(tok + p);
     int len = 0, err = 0;
     const int32_t r = walk_position<KT>(t, tok, p, pos_in_seq(p, L), x, &len, &err);
-    if (err) record_error(t.status, err);
+    if (err) record_error(t, err);
     row_out[p] = r;
     if (len_out) len_out[p] = (uint8_t)len;
   }
@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kThreads, EmbedTuning<KT>::kMinBlocks)
       int len = 0, err = 0;
       const int32_t r = match_position<FMT, KT>(t, tok, p, pos_in_seq(p, L), x, &len, &err);
       if (err) {
-        record_error(t.status, err);
+        record_error(t, err);
       } else {
         src = r >= 0 ? static_cast<const void*>(t.F + (int64_t)r * t.d)
                      : static_cast<const void*>(t.T + (int64_t)x * t.d);
@@ -176,11 +176,11 @@ __global__ void __launch_bounds__(kThreads)
       const int32_t r = __ldg(row + p);
       if (r >= 0) {
         if (r < t.n_fgrams) src = t.F + (int64_t)r * t.d;
-        else record_error(t.status, SCONE_ERR_INVALID_ARG);
+        else record_error(t, SCONE_ERR_INVALID_ARG);
       } else {
         const int32_t x = __ldg(tok + p);
         if (valid_token(x, t.vocab)) src = t.T + (int64_t)x * t.d;
-        else record_error(t.status, SCONE_ERR_TOKEN_RANGE);
+        else record_error(t, SCONE_ERR_TOKEN_RANGE);
       }
     }
     src_s[warp][lane] = src;

@@ -180,7 +180,7 @@ __device__ __forceinline__ const uint4* pipe_finish(const TableView& t, PipeMatc
   if (row_out) row_out[p] = r;
   if (len_out) len_out[p] = (uint8_t)len;
   if (err) {
-    record_error(t.status, err);
+    record_error(t, err);
     return nullptr;
   }
   return reinterpret_cast<const uint4*>(r >= 0 ? t.F + (int64_t)r * t.d

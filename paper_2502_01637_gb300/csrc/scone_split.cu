@@ -79,7 +79,7 @@ __global__ void __launch_bounds__(kSplitThreads, SplitTuning<KT>::kMinBlocks)
           !mbar_wait_bounded(saddr(&empty_bar[s]), (uint32_t)((round - 1) & 1),
                              kSplitSpinLimit)) {
         if (lane == 0) {
-          record_error(t.status, SCONE_ERR_CUDA);
+          record_error(t, SCONE_ERR_CUDA);
           *abort_v = 1;
         }
         return;
@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(kSplitThreads, SplitTuning<KT>::kMinBlocks)
         const int32_t r =
             match_position<FMT, KT>(t, tok, p, split_pos_in_seq(p, L), x, &len, &err);
         if (err) {
-          record_error(t.status, err);
+          record_error(t, err);
         } else {
           src = r >= 0 ? static_cast<const void*>(t.F + (int64_t)r * t.d)
                        : static_cast<const void*>(t.T + (int64_t)x * t.d);
@@ -116,7 +116,7 @@ __global__ void __launch_bounds__(kSplitThreads, SplitTuning<KT>::kMinBlocks)
     const int64_t round = tile / kSplitSlots;
     if (!mbar_wait_bounded(saddr(&full_bar[s]), (uint32_t)(round & 1), kSplitSpinLimit)) {
       if (lane == 0) {
-        record_error(t.status, SCONE_ERR_CUDA);
+        record_error(t, SCONE_ERR_CUDA);
         *abort_v = 1;
       }
       return;

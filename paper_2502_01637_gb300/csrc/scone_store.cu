@@ -72,9 +72,9 @@ __global__ void __launch_bounds__(kStoreThreads)
       if (r < 0) {
         const int32_t x = tok[p];
         if (valid_token(x, t.vocab)) src = t.T + (int64_t)x * t.d;
-        else record_error(t.status, SCONE_ERR_TOKEN_RANGE);
+        else record_error(t, SCONE_ERR_TOKEN_RANGE);
       } else if (r >= n_rows) {
-        record_error(t.status, SCONE_ERR_INVALID_ARG);
+        record_error(t, SCONE_ERR_INVALID_ARG);
       } else {
         const uint64_t s = slot_of_row(r, cache_rows);
         if (tag[s] == r) {

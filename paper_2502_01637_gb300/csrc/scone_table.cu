@@ -362,6 +362,7 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
   v.F = F_dev;
   v.T = reinterpret_cast<const uint16_t*>(T);
   v.status = t->status;
+  v.status_mirror = t->status_host_dev;   // NULL without a mapped mirror
   v.K = K;
   v.bits = bits;
   v.vocab = vocab;
@@ -479,8 +480,7 @@ namespace {
 // Moves the sticky status word to the host mirror and clears it, in stream
 // order: one launch instead of a copy and a memset.
 __global__ void status_fetch_kernel(int* status, int* host_mirror) {
-  *host_mirror = *status;
-  *status = 0;
+  *host_mirror = atomicExch(status, 0);
 }
 
 }  // namespace
@@ -490,6 +490,15 @@ extern "C" int scone_status(const scone_table* t, void* stream) {
   if (!t) return SCONE_ERR_INVALID_ARG;
   cudaStream_t s = (cudaStream_t)stream;
   if (t->status_host) {
+    // the kernels that record an error also write it to the mirror, so after
+    // the sync a zero mirror means no error and nothing more is launched;
+    // otherwise one kernel moves the status word into the mirror and clears
+    // it (the mirror keeps that code until the next fetch replaces it)
+    if (cudaStreamSynchronize(s) != cudaSuccess) {
+      cudaGetLastError();
+      return SCONE_ERR_CUDA;
+    }
+    if (*static_cast<volatile int*>(t->status_host) == 0) return SCONE_OK;
     scone::status_fetch_kernel<<<1, 1, 0, s>>>(t->status, t->status_host_dev);
     if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess) {
       cudaGetLastError();

@@ -247,7 +247,7 @@ __global__ void __launch_bounds__(kVThreads, VarlenTuning<KT>::kMinBlocks)
       int len = 0, err = 0;
       const int32_t r = match_varlen<FMT, KT>(t, tok, v, with_state, H, p, x, &len, &err);
       if (err) {
-        record_error(t.status, err);
+        record_error(t, err);
       } else {
         src = r >= 0 ? static_cast<const void*>(t.F + (int64_t)r * t.d)
                      : static_cast<const void*>(t.T + (int64_t)x * t.d);

@@ -185,7 +185,7 @@ __device__ __forceinline__ const uint4* walk_finish(const TableView& t, const Pi
   if (row_out) row_out[p] = m.row;
   if (len_out) len_out[p] = (uint8_t)m.len;
   if (m.err) {
-    record_error(t.status, m.err);
+    record_error(t, m.err);
     return nullptr;
   }
   return reinterpret_cast<const uint4*>(m.row >= 0 ? t.F + (int64_t)m.row * t.d

@@ -590,3 +590,33 @@ def test_prescan_staged_equals_oracle():
     for b in (corpus, rows, lens, zc_rows, zc_lens):
         b.free()
     table.close()
+
+
+def test_status_reports_the_first_error_once():
+    """scone_status returns the first device-detected error since the last
+    call and clears it; with no error it returns 0 without launching anything
+    (the kernels that record an error also write it to the table's host-mapped
+    mirror, which scone_status reads after the sync)."""
+    w = TINY.scaled("status_once", B=2, L=300, quotas=((2, 3000), (3, 2000)))
+    tok = synth.query_tokens(w)
+    bad = tok.copy()
+    bad[1, 7] = w.vocab + 3
+    case = SmallCase(w, tok=tok)
+    table = case.build()
+    for _ in range(2):
+        out, row, ln = run_embed(table, tok, w.d)
+        assert scone.scone_status(table) == 0
+        assert_parity(case, out, row, ln)
+        run_embed(table, bad, w.d)
+        assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+        assert scone.scone_status(table) == 0            # cleared by the call before
+        assert scone.scone_status(table) == 0
+    # an error in a decode step reaches the same word
+    st = scone.scone_decode_create(table, np.zeros((4, 2), np.int32), np.zeros(4, np.int32))
+    new = torch.tensor([1, 2, -5, 3], dtype=torch.int32, device=DEV)
+    out = torch.empty((4, w.d), dtype=torch.int16, device=DEV)
+    scone.scone_decode_step(st, new, out)
+    assert scone.scone_status(table, raise_on_error=False) == scone.SCONE_ERR_TOKEN_RANGE
+    assert scone.scone_status(table) == 0
+    st.close()
+    table.close()
