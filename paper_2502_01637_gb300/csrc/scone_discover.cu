@@ -409,7 +409,7 @@ bincount_kernel(const unsigned long long* __restrict__ rkey, const uint16_t* __r
   auto* ckey = reinterpret_cast<unsigned long long*>(cnt_smem);           // [kCntSlots]
   auto* ccnt = reinterpret_cast<uint32_t*>(ckey + kCntSlots);              // [kCntSlots]
   auto* cfirst = ccnt + kCntSlots;                                          // [kCntSlots]
-  __shared__ unsigned long long item_s;
+  __shared__ unsigned long long item_s[2];
   for (int h = threadIdx.x; h < kCntSlots; h += kCntThreads) {
     ckey[h] = 0;
     ccnt[h] = 0;
@@ -418,10 +418,17 @@ bincount_kernel(const unsigned long long* __restrict__ rkey, const uint16_t* __r
   const int lane = threadIdx.x & 31, warp = threadIdx.x / 32;
   const int64_t n_groups = (n_chunks + kItemChunks - 1) / kItemChunks;
   const unsigned long long n_items = (unsigned long long)n_groups * kBins;
-  for (;;) {
-    if (threadIdx.x == 0) item_s = atomicAdd(ticket, 1ull);
-    __syncthreads();
-    const unsigned long long item = item_s;
+  if (threadIdx.x == 0) item_s[0] = atomicAdd(ticket, 1ull);
+  __syncthreads();
+  // Two barriers per item: after the records (the cache is complete) and
+  // after the flush (the cache is empty, and the next ticket is in). Thread 0
+  // takes the next ticket as the flush starts, so its round trip overlaps the
+  // flush. It is not taken earlier: a block holding the next item while it
+  // counts the current one widens the span of table regions being updated at
+  // once, and the updates then miss L2 more often. item_s alternates between
+  // two slots so that the next ticket never overwrites one still being read.
+  for (int it = 0;; it ^= 1) {
+    const unsigned long long item = item_s[it];
     if (item >= n_items) break;
     const int bin = (int)(item / n_groups);
     const int64_t c0 = (int64_t)(item % n_groups) * kItemChunks + warp * 32;
@@ -484,6 +491,7 @@ bincount_kernel(const unsigned long long* __restrict__ rkey, const uint16_t* __r
         if (cold[u]) table_add(table, cap, key[u], home[u], prev[u], 1u, start[u], err);
     }
     __syncthreads();
+    if (threadIdx.x == 0) item_s[it ^ 1] = atomicAdd(ticket, 1ull);
     // add the cache to the table and empty it; every probe of a batch is
     // issued before any result is used
     constexpr int kOwn = kCntSlots / kCntThreads;
