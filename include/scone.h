@@ -589,8 +589,10 @@ int scone_decode_destroy(scone_decode* state);
  * error recorded since the last call (SCONE_OK if none) and clears it. The
  * kernel that records an error also writes it to a host-mapped word of the
  * table, so when no error was recorded the call is the sync and one read of
- * host memory; after an error it launches one 1-thread kernel that moves the
- * status word into that host word and clears it.
+ * host memory; after an error it clears that word and launches one 1-thread
+ * kernel that moves the status word to the host and clears it. An error that
+ * a kernel on another stream records during the call is returned by the next
+ * call. Calls on one table must not overlap.
  */
 int scone_status(const scone_table* table, void* stream);
 

@@ -18,7 +18,8 @@ struct scone_table {
   int fmt = scone::FMT16;
   uint8_t* slots = nullptr;  // n_buckets * 32 bytes
   int* status = nullptr;     // sticky device error word
-  int* status_host = nullptr;      // pinned, device-mapped mirror read by scone_status
+  int* status_host = nullptr;      // pinned, device-mapped [2]: the recorded error's copy and
+                                   // the fetched status word, read by scone_status
   int* status_host_dev = nullptr;  // its device address
   uint8_t* zero_row = nullptr;  // d * 2 zero bytes: the source of error positions (bulk copies)
   int copy_mode = SCONE_COPY_AUTO;

@@ -338,11 +338,14 @@ extern "C" int scone_table_build(const int32_t* fgram_tok, const uint8_t* fgram_
     scone_table_destroy(t);
     return SCONE_ERR_NOMEM;
   }
-  // the status mirror is an optimisation: without it scone_status copies the word
+  // the status mirror is an optimisation: without it scone_status copies the
+  // word. Word 0 is the copy the recording kernel writes, word 1 receives the
+  // status word when scone_status fetches it.
   void* mirror = nullptr;
-  if (cudaHostAlloc(&mirror, sizeof(int), cudaHostAllocMapped) == cudaSuccess) {
+  if (cudaHostAlloc(&mirror, 2 * sizeof(int), cudaHostAllocMapped) == cudaSuccess) {
     t->status_host = static_cast<int*>(mirror);
-    *t->status_host = 0;
+    t->status_host[0] = 0;
+    t->status_host[1] = 0;
     void* dp = nullptr;
     if (cudaHostGetDevicePointer(&dp, mirror, 0) == cudaSuccess) {
       t->status_host_dev = static_cast<int*>(dp);
@@ -477,10 +480,10 @@ extern "C" int scone_table_set_copy_mode(scone_table* t, int32_t mode) {
 namespace scone {
 namespace {
 
-// Moves the sticky status word to the host mirror and clears it, in stream
-// order: one launch instead of a copy and a memset.
-__global__ void status_fetch_kernel(int* status, int* host_mirror) {
-  *host_mirror = atomicExch(status, 0);
+// Moves the sticky status word into a host-mapped word and clears it, in
+// stream order: one launch instead of a copy and a memset.
+__global__ void status_fetch_kernel(int* status, int* host_word) {
+  *host_word = atomicExch(status, 0);
 }
 
 }  // namespace
@@ -490,21 +493,25 @@ extern "C" int scone_status(const scone_table* t, void* stream) {
   if (!t) return SCONE_ERR_INVALID_ARG;
   cudaStream_t s = (cudaStream_t)stream;
   if (t->status_host) {
-    // the kernels that record an error also write it to the mirror, so after
-    // the sync a zero mirror means no error and nothing more is launched;
-    // otherwise one kernel moves the status word into the mirror and clears
-    // it (the mirror keeps that code until the next fetch replaces it)
+    // the kernel that records an error (the one whose compare-and-swap sets
+    // the status word) also writes it to mirror word 0, so after the sync a
+    // zero there means no error and nothing is launched. Otherwise word 0 is
+    // cleared first (while the status word is set, no kernel writes it) and
+    // one kernel moves the status word into word 1 and clears it; an error
+    // recorded after that exchange sets word 0 again for the next call.
     if (cudaStreamSynchronize(s) != cudaSuccess) {
       cudaGetLastError();
       return SCONE_ERR_CUDA;
     }
-    if (*static_cast<volatile int*>(t->status_host) == 0) return SCONE_OK;
-    scone::status_fetch_kernel<<<1, 1, 0, s>>>(t->status, t->status_host_dev);
+    volatile int* m = t->status_host;
+    if (m[0] == 0) return SCONE_OK;
+    m[0] = 0;
+    scone::status_fetch_kernel<<<1, 1, 0, s>>>(t->status, t->status_host_dev + 1);
     if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess) {
       cudaGetLastError();
       return SCONE_ERR_CUDA;
     }
-    return *static_cast<volatile int*>(t->status_host);
+    return m[1];
   }
   int code = 0;
   if (cudaMemcpyAsync(&code, t->status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
