@@ -641,7 +641,8 @@ extern "C" const char* scone_strerror(int code) {
     case SCONE_ERR_DUPLICATE_FGRAM: return "duplicate f-gram in the list";
     case SCONE_ERR_TABLE_FULL: return "hash table full";
     case SCONE_ERR_PROBE_LIMIT: return "lookup exceeded the probe limit";
-    case SCONE_ERR_UNSUPPORTED: return "key does not fit (K * ceil(log2 vocab) > 220)";
+    case SCONE_ERR_UNSUPPORTED:
+      return "unsupported size (K * ceil(log2 vocab) > 220, or a suffix index over 2^32 - 2 entries)";
     case SCONE_ERR_CUDA: return "CUDA runtime error";
     case SCONE_ERR_NOMEM: return "out of memory";
     default: return "unknown error";
