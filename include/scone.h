@@ -59,8 +59,9 @@ enum scone_err {
   SCONE_ERR_DUPLICATE_FGRAM = -3, /* the f-gram list holds the same n-gram twice */
   SCONE_ERR_TABLE_FULL = -4,      /* an insert found no free slot (cannot happen below LF 1) */
   SCONE_ERR_PROBE_LIMIT = -5,     /* a lookup read more buckets than the limit (sticky) */
-  SCONE_ERR_UNSUPPORTED = -6,     /* K * ceil(log2 vocab) does not fit the key format, or a
-                                     suffix index would exceed 2^32 - 2 entries */
+  SCONE_ERR_UNSUPPORTED = -6,     /* outside what the call supports: K * ceil(log2 vocab)
+                                     wider than the key format, a size past the call's
+                                     documented limit, or a copy mode it cannot use */
   SCONE_ERR_CUDA = -7,            /* a CUDA runtime call failed */
   SCONE_ERR_NOMEM = -8            /* device or host allocation failed */
 };

@@ -642,7 +642,8 @@ extern "C" const char* scone_strerror(int code) {
     case SCONE_ERR_TABLE_FULL: return "hash table full";
     case SCONE_ERR_PROBE_LIMIT: return "lookup exceeded the probe limit";
     case SCONE_ERR_UNSUPPORTED:
-      return "unsupported size (K * ceil(log2 vocab) > 220, or a suffix index over 2^32 - 2 entries)";
+      return "unsupported by this call (key wider than 220 bits, a size past the call's limit, "
+             "or a copy mode it cannot use)";
     case SCONE_ERR_CUDA: return "CUDA runtime error";
     case SCONE_ERR_NOMEM: return "out of memory";
     default: return "unknown error";
