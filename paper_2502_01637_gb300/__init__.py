@@ -346,11 +346,29 @@ def scone_match(table: Table, tok, row, len=None, stream=None) -> None:
                                       _stream(stream)), "scone_match")
 
 
+def _nbytes(x) -> Optional[int]:
+    """Size in bytes of a buffer argument, or None for a raw address."""
+    if x is None or isinstance(x, int):
+        return None
+    if isinstance(x, HostBuffer):
+        return x.nbytes
+    if isinstance(x, np.ndarray):
+        return x.nbytes
+    return x.numel() * x.element_size()
+
+
 def scone_prescan(table: Table, tok, B: int, L: int, row, len=None, chunk_tokens: int = 0,
                   stream=None) -> None:
     """Tags a corpus in host memory (tok, row, len: host addresses or buffers of
     B * L entries), staged through HBM in chunks of whole sequences; returns
-    when the tags are in host memory."""
+    when the tags are in host memory. Buffers whose size is known are checked
+    against B * L entries first (the copies would otherwise run past them)."""
+    n = max(B, 0) * max(L, 0)
+    for name, buf, width in (("tok", tok, 4), ("row", row, 4), ("len", len, 1)):
+        size = _nbytes(buf)
+        if size is not None and size < n * width:
+            raise ValueError(f"scone_prescan: {name} holds {size} bytes, "
+                             f"B * L = {n} entries need {n * width}")
     _check(load_library().scone_prescan(table.handle, _ptr(tok), B, L, _ptr(row), _ptr(len),
                                         chunk_tokens, _stream(stream)), "scone_prescan")
 

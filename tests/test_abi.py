@@ -127,3 +127,25 @@ def test_host_tokens_must_be_pinned():
         scone._tok_ptr(torch.zeros(8, dtype=torch.int32))
     with pytest.raises(ValueError):
         scone._tok_ptr(np.zeros(8, np.int32))
+
+
+def test_prescan_buffers_checked_against_the_corpus_size():
+    """scone_prescan's wrapper refuses host buffers shorter than B * L entries
+    (4 bytes for tokens and rows, 1 for lengths) before the library is
+    called, so no copy can run past them."""
+    import numpy as np
+    import pytest
+
+    import paper_2502_01637_gb300 as scone
+
+    B, L = 3, 5
+    ok_tok, ok_row, ok_len = (np.zeros(B * L, np.int32), np.zeros(B * L, np.int32),
+                              np.zeros(B * L, np.uint8))
+    short = (np.zeros(B * L - 1, np.int32), np.zeros(B * L - 1, np.int32),
+             np.zeros(B * L - 1, np.uint8))
+    for k, name in enumerate(("tok", "row", "len")):
+        args = [ok_tok, ok_row, ok_len]
+        args[k] = short[k]
+        with pytest.raises(ValueError, match=name):
+            scone.scone_prescan(None, args[0], B, L, args[1], args[2])
+    assert scone._nbytes(ok_len) == B * L and scone._nbytes(0x1000) is None
