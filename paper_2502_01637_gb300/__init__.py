@@ -209,6 +209,14 @@ class Table:
     def __init__(self, handle: ctypes.c_void_p, keep):
         self._h = handle
         self._keep = keep   # F and T must outlive the table
+        self._d = None
+
+    @property
+    def d(self) -> int:
+        """Row width (elements), read once from the table."""
+        if self._d is None:
+            self._d = self.info()["d"]
+        return self._d
 
     @property
     def handle(self) -> ctypes.c_void_p:
@@ -342,6 +350,7 @@ def _bl(tok):
 def scone_match(table: Table, tok, row, len=None, stream=None) -> None:
     """tok [B, L] (or [n]) int32 device; row int32 and len uint8 of the same count."""
     B, L = _bl(tok)
+    _need("scone_match", ("row", row, 4 * B * L), ("len", len, B * L))
     _check(load_library().scone_match(table.handle, _ptr(tok), B, L, _ptr(row), _ptr(len),
                                       _stream(stream)), "scone_match")
 
@@ -357,6 +366,16 @@ def _nbytes(x) -> Optional[int]:
     return x.numel() * x.element_size()
 
 
+def _need(call: str, *specs) -> None:
+    """specs: (name, buffer, bytes the call reads or writes there). A buffer of
+    known size that holds fewer bytes raises ValueError before the call, so no
+    kernel or copy runs past it; raw addresses and None pass unchecked."""
+    for name, buf, need in specs:
+        size = _nbytes(buf)
+        if size is not None and size < need:
+            raise ValueError(f"{call}: {name} holds {size} bytes, needs {need}")
+
+
 def scone_prescan(table: Table, tok, B: int, L: int, row, len=None, chunk_tokens: int = 0,
                   stream=None) -> None:
     """Tags a corpus in host memory (tok, row, len: host addresses or buffers of
@@ -364,16 +383,14 @@ def scone_prescan(table: Table, tok, B: int, L: int, row, len=None, chunk_tokens
     when the tags are in host memory. Buffers whose size is known are checked
     against B * L entries first (the copies would otherwise run past them)."""
     n = max(B, 0) * max(L, 0)
-    for name, buf, width in (("tok", tok, 4), ("row", row, 4), ("len", len, 1)):
-        size = _nbytes(buf)
-        if size is not None and size < n * width:
-            raise ValueError(f"scone_prescan: {name} holds {size} bytes, "
-                             f"B * L = {n} entries need {n * width}")
+    _need("scone_prescan", ("tok", tok, 4 * n), ("row", row, 4 * n), ("len", len, n))
     _check(load_library().scone_prescan(table.handle, _ptr(tok), B, L, _ptr(row), _ptr(len),
                                         chunk_tokens, _stream(stream)), "scone_prescan")
 
 
 def scone_embed_gather(table: Table, tok, row, out, stream=None) -> None:
+    n = tok.numel()
+    _need("scone_embed_gather", ("row", row, 4 * n), ("out", out, 2 * n * table.d))
     _check(load_library().scone_embed_gather(table.handle, _ptr(tok), _ptr(row), tok.numel(),
                                              _ptr(out), _stream(stream)), "scone_embed_gather")
 
@@ -393,6 +410,8 @@ def scone_embed(table: Table, tok, out, row=None, len=None, stream=None) -> None
     """Fused Algorithm 1: out [B*L, d] bf16 rows; row / len optional. tok may
     be a pinned CPU tensor: the kernel then reads it over the host link."""
     B, L = _bl(tok)
+    n = B * L
+    _need("scone_embed", ("out", out, 2 * n * table.d), ("row", row, 4 * n), ("len", len, n))
     _check(load_library().scone_embed(table.handle, _tok_ptr(tok), B, L, _ptr(out), _ptr(row),
                                       _ptr(len), _stream(stream)), "scone_embed")
 
@@ -403,6 +422,9 @@ def scone_embed_varlen(table: Table, tok, cu_seqlens, out, state=None, seq_slot=
     (device); with a DecodeState, sequence b continues slot seq_slot[b] (or
     b) and the slots' histories advance."""
     n_seq = cu_seqlens.numel() - 1
+    n = tok.numel()
+    _need("scone_embed_varlen", ("out", out, 2 * n * table.d), ("row", row, 4 * n),
+          ("len", len, n), ("seq_slot", seq_slot, 4 * max(n_seq, 0)))
     _check(load_library().scone_embed_varlen(
         table.handle, _ptr(tok), tok.numel(), _ptr(cu_seqlens), n_seq,
         state.handle if state is not None else None, _ptr(seq_slot), _ptr(out), _ptr(row),
@@ -541,6 +563,8 @@ def scone_rowstore_probe_reads(store: RowStore, n_reads: int, seed: int = 1) -> 
 
 def scone_rowstore_gather(store: RowStore, table: Table, tok, row, out, stream=None) -> None:
     """out[t] = F[row[t]] from the store (or T[tok[t]] where row[t] < 0)."""
+    n = row.numel()
+    _need("scone_rowstore_gather", ("tok", tok, 4 * n), ("out", out, 2 * n * table.d))
     _check(load_library().scone_rowstore_gather(store.handle, table.handle, _ptr(tok), _ptr(row),
                                                 row.numel(), _ptr(out), _stream(stream)),
            "scone_rowstore_gather")
@@ -584,6 +608,10 @@ def scone_decode_create(table: Table, hist: np.ndarray, hist_len: np.ndarray) ->
 def scone_decode_step(state: DecodeState, new_tok, out, row=None, len=None, stream=None) -> None:
     """One decode step; new_tok [S] int32, a CUDA tensor or a pinned CPU tensor
     (read by the kernel over the host link)."""
+    S = state.S
+    _need("scone_decode_step", ("new_tok", new_tok, 4 * S),
+          ("out", out, 2 * S * state._table.d if out is not None else 0),
+          ("row", row, 4 * S), ("len", len, S))
     _check(load_library().scone_decode_step(state.handle, _tok_ptr(new_tok), _ptr(out),
                                             _ptr(row), _ptr(len), _stream(stream)),
            "scone_decode_step")

@@ -149,3 +149,52 @@ def test_prescan_buffers_checked_against_the_corpus_size():
         with pytest.raises(ValueError, match=name):
             scone.scone_prescan(None, args[0], B, L, args[1], args[2])
     assert scone._nbytes(ok_len) == B * L and scone._nbytes(0x1000) is None
+
+
+def test_output_buffers_checked_against_the_batch():
+    """The embed, match, gather, ragged-batch and decode wrappers refuse an
+    output (or index) buffer smaller than the batch needs before the library
+    is called: the kernels cannot see a tensor's size and would write past
+    it. Checked with host tensors and stand-in handles (no device needed)."""
+    import types
+
+    import numpy as np
+    import pytest
+    import torch
+
+    import paper_2502_01637_gb300 as scone
+
+    d, B, L = 16, 2, 3
+    n = B * L
+    table = types.SimpleNamespace(d=d, handle=None)
+    tok = torch.zeros((B, L), dtype=torch.int32)
+    out_ok = torch.zeros((n, d), dtype=torch.int16)
+    out_short = torch.zeros((n - 1, d), dtype=torch.int16)
+    row_short = torch.zeros(n - 1, dtype=torch.int32)
+    len_short = torch.zeros(n - 1, dtype=torch.uint8)
+    with pytest.raises(ValueError, match="out"):
+        scone.scone_embed(table, tok, out_short)
+    with pytest.raises(ValueError, match="row"):
+        scone.scone_embed(table, tok, out_ok, row=row_short)
+    with pytest.raises(ValueError, match="len"):
+        scone.scone_embed(table, tok, out_ok, len=len_short)
+    with pytest.raises(ValueError, match="row"):
+        scone.scone_match(table, tok, row_short)
+    with pytest.raises(ValueError, match="out"):
+        scone.scone_embed_gather(table, tok.reshape(-1), torch.zeros(n, dtype=torch.int32),
+                                 out_short)
+    cu = torch.tensor([0, 4, n], dtype=torch.int32)
+    with pytest.raises(ValueError, match="out"):
+        scone.scone_embed_varlen(table, tok.reshape(-1), cu, out_short)
+    with pytest.raises(ValueError, match="seq_slot"):
+        scone.scone_embed_varlen(table, tok.reshape(-1), cu, out_ok,
+                                 seq_slot=torch.zeros(1, dtype=torch.int32))
+    state = types.SimpleNamespace(S=4, _table=table, handle=None)
+    with pytest.raises(ValueError, match="out"):
+        scone.scone_decode_step(state, torch.zeros(4, dtype=torch.int32), out_short[:3])
+    with pytest.raises(ValueError, match="new_tok"):
+        scone.scone_decode_step(state, np.zeros(3, np.int32), None)
+    # a buffer of the right size passes the check (and then meets the host-token
+    # rule: pageable CPU tokens are refused)
+    with pytest.raises(ValueError, match="pinned"):
+        scone.scone_embed(table, tok, out_ok)
