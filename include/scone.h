@@ -523,7 +523,11 @@ int scone_fgram_precompute(scone_fgram_model* model, const int32_t* fgram_tok,
  * Synchronous. scone_rowstore_gather: out[t] = F[row[t]] (row[t] >= 0) or
  * T[tok[t]] (row[t] < 0, T from the table, whose d must equal the store's);
  * row as written by scone_match, scone_embed_varlen or scone_decode_step;
- * tok, row device [n]; out device [n * d], 16-byte aligned. Synchronous (the
+ * tok, row device [n]; out device [n * d], 16-byte aligned. A table used only
+ * to select rows for a store (scone_match, or scone_decode_step with out =
+ * NULL) never reads its F, and may be built with a placeholder F of one row;
+ * the calls that copy f-gram rows (scone_embed, scone_embed_gather,
+ * scone_embed_varlen, scone_decode_step with out) need the full F. Synchronous (the
  * host reads the misses). A row id >= n_rows or a token outside the vocab is
  * a device-detected error (zero row, sticky table status); a failed read
  * returns SCONE_ERR_CUDA.

@@ -254,6 +254,10 @@ def scone_table_build(fgram_tok: np.ndarray, fgram_len: np.ndarray, K: int, voca
     n = fl.shape[0]
     if ft.shape[0] != n * K:
         raise ValueError("fgram_tok must be [n_fgrams, K]")
+    # T is read for every position without an f-gram; F only by the calls that
+    # copy f-gram rows (a table that only selects rows for a row store may hold
+    # a one-row placeholder F)
+    _need("scone_table_build", ("T", T, 2 * max(vocab, 0) * max(d, 0)))
     h = _vp()
     rc = lib.scone_table_build(_ptr(ft) if n else None, _ptr(fl) if n else None, n, K, vocab, d,
                                _ptr(F), F_location, _ptr(T), load_factor, _stream(stream),

@@ -198,3 +198,20 @@ def test_output_buffers_checked_against_the_batch():
     # rule: pageable CPU tokens are refused)
     with pytest.raises(ValueError, match="pinned"):
         scone.scone_embed(table, tok, out_ok)
+
+
+def test_table_build_checks_T_against_the_vocabulary():
+    """scone_table_build's wrapper refuses a token table T smaller than vocab
+    rows of d bf16 before the library is called (the kernels read T[token]
+    for every position without an f-gram)."""
+    import numpy as np
+    import pytest
+    import torch
+
+    import paper_2502_01637_gb300 as scone
+
+    ft = np.array([[1, 2]], np.int32)
+    fl = np.array([2], np.uint8)
+    T_short = torch.zeros((9, 8), dtype=torch.int16)
+    with pytest.raises(ValueError, match="T"):
+        scone.scone_table_build(ft, fl, 2, 10, 8, None, T_short)
