@@ -445,6 +445,11 @@ def scone_gemm_bf16(A, B, C, R=None, epilogue: int = SCONE_GEMM_STORE, status=No
 
     M, K = A.shape
     N = B.shape[0]
+    if B.dim() != 2 or B.shape[1] != K:
+        raise ValueError(f"scone_gemm_bf16: B must be [N, {K}], got {tuple(B.shape)}")
+    c_cols = N // 2 if epilogue == SCONE_GEMM_SWIGLU else N
+    _need("scone_gemm_bf16", ("C", C, 2 * M * c_cols),
+          ("R", R if epilogue == SCONE_GEMM_RESIDUAL else None, 2 * M * N))
     own = status is None
     if own:
         status = torch.zeros(1, dtype=torch.int32, device=A.device)
@@ -505,6 +510,9 @@ def scone_fgram_precompute(model: FgramModel, fgram_tok, fgram_len, T, F,
     tensors, T [vocab, d] device, F [n, d] device tensor (or host-mapped address)."""
     n, K = fgram_tok.shape
     vocab = T.shape[0] if vocab is None else vocab
+    d = model.d
+    _need("scone_fgram_precompute", ("fgram_len", fgram_len, n), ("T", T, 2 * vocab * d),
+          ("F", F, 2 * n * d))
     _check(load_library().scone_fgram_precompute(model.handle, _ptr(fgram_tok), _ptr(fgram_len), n,
                                                  K, _ptr(T), vocab, _ptr(F), _stream(stream)),
            "scone_fgram_precompute")

@@ -215,3 +215,33 @@ def test_table_build_checks_T_against_the_vocabulary():
     T_short = torch.zeros((9, 8), dtype=torch.int16)
     with pytest.raises(ValueError, match="T"):
         scone.scone_table_build(ft, fl, 2, 10, 8, None, T_short)
+
+
+def test_gemm_and_precompute_buffers_checked():
+    """scone_gemm_bf16 refuses B of another K and a C (or R) smaller than the
+    epilogue writes (reads); scone_fgram_precompute refuses an F smaller than
+    n rows of d. Both before the library is called."""
+    import types
+
+    import pytest
+    import torch
+
+    import paper_2502_01637_gb300 as scone
+
+    A = torch.zeros((128, 64), dtype=torch.int16)
+    with pytest.raises(ValueError, match="B must be"):
+        scone.scone_gemm_bf16(A, torch.zeros((256, 32), dtype=torch.int16),
+                              torch.zeros((128, 256), dtype=torch.int16))
+    B = torch.zeros((256, 64), dtype=torch.int16)
+    with pytest.raises(ValueError, match="C"):
+        scone.scone_gemm_bf16(A, B, torch.zeros((128, 128), dtype=torch.int16))
+    with pytest.raises(ValueError, match="R"):
+        scone.scone_gemm_bf16(A, B, torch.zeros((128, 256), dtype=torch.int16),
+                              R=torch.zeros((127, 256), dtype=torch.int16),
+                              epilogue=scone.SCONE_GEMM_RESIDUAL)
+    model = types.SimpleNamespace(d=256, handle=None)
+    tok = torch.zeros((4, 3), dtype=torch.int32)
+    ln = torch.full((4,), 3, dtype=torch.uint8)
+    T = torch.zeros((10, 256), dtype=torch.int16)
+    with pytest.raises(ValueError, match="F"):
+        scone.scone_fgram_precompute(model, tok, ln, T, torch.zeros((3, 256), dtype=torch.int16))
