@@ -98,6 +98,14 @@ def test_null_handles_rejected():
     assert lib.scone_discover_create(None) == inv
     assert lib.scone_discover_destroy(None) == 0
     assert lib.scone_discover_set_table_slack(None, 2.5) == inv
+    assert lib.scone_prescan(None, None, 1, 1, None, None, 0, None) == inv
+    n_markers = ctypes.c_int64(-1)
+    assert lib.scone_fgram_suffix_index(None, None, 1, 3, None, None, None, 0,
+                                        ctypes.byref(n_markers)) == inv    # list missing
+    assert lib.scone_fgram_suffix_index(None, None, 0, 3, None, None, None, 0,
+                                        None) == inv                      # no count pointer
+    assert lib.scone_fgram_suffix_index(None, None, 0, 3, None, None, None, 0,
+                                        ctypes.byref(n_markers)) == 0 and n_markers.value == 0
 
 
 def test_key_format_boundaries():
